@@ -1,0 +1,191 @@
+/*
+ * mbe.h -- C ABI of the GB300 (sm_103a) library for the data-parallel hot path
+ * of Multi-Block Editing (MBE) for block-diffusion language models
+ * (arXiv 2607.22663).
+ *
+ * One editing pass of MBE (Sec. 4.1, Eq. 5) reopens a window of k already
+ * decoded blocks, runs the model over the window with full attention inside
+ * it while reading the committed prefix from the KV cache, and applies the
+ * token-to-token (T2T) edit rule of Eq. 2 to the window's historical part.
+ * Blocks that changed are recomputed under standard (block-causal) attention
+ * and their KV written back (Sec. 4.3, cache control). This library provides
+ * the three data-parallel steps of that pass:
+ *
+ *   mbe_window_attention   attention of the window queries over the paged
+ *                          prefix plus the window (Eq. 5; Sec. 2.2)
+ *   mbe_edit_decide        argmax / confidence / threshold-and-replace (Eq. 2)
+ *   mbe_kv_window_write    scatter of window K/V into the paged cache (Sec. 4.3)
+ *
+ * Conventions shared by every entry point
+ *   - All pointers are DEVICE pointers unless stated otherwise; the caller
+ *     owns every buffer. The library never allocates device memory.
+ *   - Every call validates its host-visible arguments synchronously and returns
+ *     a status; on any status other than MBE_OK nothing was launched.
+ *   - Work is enqueued asynchronously on `stream`. Conditions that only the
+ *     device can see (a length above the declared maximum, a page id outside
+ *     the cache, a bounded wait that ran out) set a device error word and the
+ *     affected work is skipped; mbe_get_device_error() reports and clears it.
+ *   - bf16 tensors are IEEE bfloat16 bit patterns, row-major, densely packed in
+ *     the stated shapes; every base pointer must be 16-byte aligned.
+ *   - Window tokens of all sequences are packed back to back ("ragged"):
+ *     sequence s owns rows cu_window[s] .. cu_window[s] + window_len[s] - 1.
+ *   - Query head h reads KV head h / (num_q_heads / num_kv_heads) (grouped-
+ *     query attention with contiguous groups).
+ */
+#ifndef MBE_H
+#define MBE_H
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  MBE_OK = 0,
+  MBE_ERR_INVALID_ARG = 1,   /* bad host-visible argument (null, shape, alignment) */
+  MBE_ERR_UNSUPPORTED = 2,   /* valid but not implemented (e.g. head_dim 96) */
+  MBE_ERR_CUDA = 3,          /* a CUDA runtime/driver call failed */
+  MBE_ERR_TIMEOUT = 4,       /* a bounded device wait expired (device error word) */
+  MBE_ERR_WORKSPACE = 5,     /* workspace missing or smaller than required */
+  MBE_ERR_DEVICE_CHECK = 6   /* a device-side argument check failed (device error word) */
+} mbe_status;
+
+/* Attention mask of the window part (Sec. 2.2 and Eq. 5). */
+typedef enum {
+  MBE_BLOCK_CAUSAL = 0,              /* window query i sees window key j iff floor(j/B) <= floor(i/B) */
+  MBE_MULTI_BLOCK_BIDIRECTIONAL = 1  /* every window query sees every window key (full attention in W_j) */
+} mbe_mask_mode;
+
+typedef enum { MBE_F32 = 0, MBE_BF16 = 1 } mbe_dtype;
+
+/* Bits of the device error word (see mbe_get_device_error). */
+#define MBE_DEVERR_TIMEOUT 0x1u       /* a bounded wait in a kernel expired */
+#define MBE_DEVERR_LENGTH 0x2u        /* prefix_len/window_len/mask_mode outside the declared range */
+#define MBE_DEVERR_PAGE 0x4u          /* a block_table entry outside [0, num_pages) */
+#define MBE_DEVERR_CAPACITY 0x8u      /* work list larger than the workspace was sized for */
+
+/*
+ * mbe_window_attention -- attention of one editing (or standard) pass.
+ * Paper: Eq. 5 (window W_j = [j* B, (j+1) B) with full attention inside the
+ * window), Sec. 2.2 (block j conditions on the committed prefix; blocks are
+ * decoded left to right), Sec. 4.3 (the editing pass reads cached history and
+ * writes no KV).
+ *
+ * For sequence s (P = prefix_len[s], W = window_len[s]) and window query i,
+ * query head h, KV head g = h / (num_q_heads / num_kv_heads):
+ *   out[cu_window[s] + i, h, :] = sum_j softmax_j(scale * q . k_j) v_j
+ * over the visible keys j: all P prefix keys (cache positions 0..P-1, read
+ * through block_table), and the window keys permitted by mask_mode[s].
+ *
+ *   q          bf16 [total_q_tokens, num_q_heads, head_dim]
+ *   k_win,v_win bf16 [total_q_tokens, num_kv_heads, head_dim]: K/V of this pass's
+ *              window tokens (never written to the cache by this call)
+ *   k_cache,v_cache bf16 [num_pages, num_kv_heads, page_size, head_dim]
+ *   block_table int32 [batch, max_pages_per_seq]: physical page of logical page
+ *              p of sequence s; entries past ceil(P/page_size) are not read.
+ *              An entry outside [0, num_pages) reads zeros and sets
+ *              MBE_DEVERR_PAGE.
+ *   prefix_len, window_len int32 [batch]; cu_window int32 [batch + 1] with
+ *              cu_window[0] = 0, cu_window[s+1] = cu_window[s] + window_len[s],
+ *              cu_window[batch] = total_q_tokens.
+ *   mask_mode  uint8 [batch], values of mbe_mask_mode (per sequence, so mixed
+ *              standard and editing passes run in one launch).
+ *   max_window, max_prefix  host upper bounds of window_len[] and prefix_len[]
+ *              (they size the workspace; a larger device value sets
+ *              MBE_DEVERR_LENGTH and that sequence is skipped).
+ *   softmax_scale  0 means 1/sqrt(head_dim).
+ *   out        bf16 [total_q_tokens, num_q_heads, head_dim]
+ *   lse_or_null fp32 [total_q_tokens, num_q_heads]: natural-log sum of exp of
+ *              the scaled scores, or NULL.
+ *   workspace  device scratch of at least mbe_window_attention_workspace_size()
+ *              bytes (work list and split-KV partials); not shared between
+ *              concurrent calls.
+ * Supported: head_dim in {64, 128}; num_q_heads / num_kv_heads a power of two
+ * <= 128; page_size a power of two >= 8; block_size >= 1. Rows of k_win/v_win
+ * for all total_q_tokens tokens must hold finite values.
+ * Errors: MBE_ERR_INVALID_ARG, MBE_ERR_UNSUPPORTED, MBE_ERR_WORKSPACE,
+ * MBE_ERR_CUDA (launch failure).
+ */
+mbe_status mbe_window_attention(const void* q, const void* k_win, const void* v_win, const void* k_cache,
+                                const void* v_cache, int32_t num_pages, const int32_t* block_table,
+                                int32_t max_pages_per_seq, const int32_t* prefix_len, const int32_t* window_len,
+                                const int32_t* cu_window, const uint8_t* mask_mode, int32_t batch,
+                                int32_t total_q_tokens, int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim,
+                                int32_t block_size, int32_t page_size, int32_t max_window, int32_t max_prefix,
+                                float softmax_scale, void* out, float* lse_or_null, void* workspace,
+                                size_t workspace_bytes, cudaStream_t stream);
+
+/* Bytes of device workspace mbe_window_attention needs for these bounds on the
+ * current device (depends on its SM count). Returns 0 for invalid arguments. */
+size_t mbe_window_attention_workspace_size(int32_t batch, int32_t num_q_heads, int32_t num_kv_heads,
+                                           int32_t head_dim, int32_t max_window, int32_t max_prefix);
+
+/*
+ * mbe_edit_decide -- the T2T update of Eq. 2 for every row of a pass.
+ * Paper: Eq. 2 (Delta_t: a visible token is overwritten by the highest-
+ * probability prediction when the prediction differs and its confidence
+ * exceeds omega_edit); Sec. 4.1 (edits only in the window's historical part).
+ *
+ * For row r of logits l[r, 0..vocab-1]:
+ *   argmax[r]     = x_hat = argmax_v l[r, v], the lowest index among ties
+ *   confidence[r] = c = softmax(l[r])[x_hat] = 1 / sum_v exp(l[r, v] - l[r, x_hat])   (fp32)
+ *   edit_mask[r]  = editable[r] && x_hat != committed[r] && c > tau_r
+ *   new_tokens[r] = edit_mask[r] ? x_hat : committed[r]
+ * with tau_r = tau_per_row[r] if given, else tau.
+ *
+ *   logits     [rows, row_stride] of `dtype`, the first `vocab` entries of each
+ *              row used; finite values (non-finite input gives unspecified output)
+ *   committed  int32 [rows]; new_tokens may alias committed
+ *   editable_or_null uint8 [rows] (NULL: every row editable)
+ *   new_tokens int32 [rows], edit_mask uint8 [rows], confidence fp32 [rows],
+ *   argmax_or_null int32 [rows]
+ * Errors: MBE_ERR_INVALID_ARG (null pointer, vocab < 1, row_stride < vocab),
+ * MBE_ERR_CUDA.
+ */
+mbe_status mbe_edit_decide(const void* logits, mbe_dtype dtype, int64_t row_stride, int32_t rows, int32_t vocab,
+                           const int32_t* committed, const float* tau_per_row_or_null, float tau,
+                           const uint8_t* editable_or_null, int32_t* new_tokens, uint8_t* edit_mask,
+                           float* confidence, int32_t* argmax_or_null, cudaStream_t stream);
+
+/*
+ * mbe_kv_window_write -- refresh of the cache with the window's K/V.
+ * Paper: Sec. 4.1 (modified blocks are recomputed under standard attention to
+ * refresh their KV cache) and Sec. 4.3 (cache control: only the changed blocks
+ * are written back, after editing converges).
+ *
+ * For sequence s and window token i (P = prefix_len[s]), every KV head g:
+ *   cache[block_table[s][(P+i)/page_size], g, (P+i) % page_size, :] = win[cu_window[s]+i, g, :]
+ * for K and V. With block_write_mask_or_null ([batch, max_blocks_per_seq]
+ * uint8), window block b = i / block_size is written only where the mask is
+ * non-zero. A page id outside [0, num_pages) is skipped and sets
+ * MBE_DEVERR_PAGE; a window longer than max_window sets MBE_DEVERR_LENGTH.
+ *   k_win, v_win bf16 [total tokens, num_kv_heads, head_dim]
+ *   k_cache, v_cache bf16 [num_pages, num_kv_heads, page_size, head_dim]
+ * head_dim must be a multiple of 8.
+ */
+mbe_status mbe_kv_window_write(const void* k_win, const void* v_win, void* k_cache, void* v_cache,
+                               int32_t num_pages, const int32_t* block_table, int32_t max_pages_per_seq,
+                               const int32_t* prefix_len, const int32_t* window_len, const int32_t* cu_window,
+                               const uint8_t* block_write_mask_or_null, int32_t max_blocks_per_seq, int32_t batch,
+                               int32_t max_window, int32_t num_kv_heads, int32_t head_dim, int32_t block_size,
+                               int32_t page_size, cudaStream_t stream);
+
+/* Synchronises `stream`, then reads and clears the device error word of the
+ * current device. Returns MBE_OK if it was clear, MBE_ERR_TIMEOUT if the
+ * timeout bit was set, else MBE_ERR_DEVICE_CHECK; *flags_or_null receives the
+ * MBE_DEVERR_* bits. */
+mbe_status mbe_get_device_error(cudaStream_t stream, uint32_t* flags_or_null);
+
+/* Static description of a status code. */
+const char* mbe_status_string(mbe_status status);
+
+/* Library version: major * 10000 + minor * 100 + patch. */
+int32_t mbe_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MBE_H */

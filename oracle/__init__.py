@@ -1,0 +1,169 @@
+"""CPU oracle for the MBE editing-pass hot path (test infrastructure only).
+
+This package is a plain, slow, double-precision restatement of what the hot
+path computes, written from the paper (arXiv 2607.22663):
+
+* ``window_attention``  -- Eq. 5 editing window with full attention inside the
+  window, Sec. 2.2 block-causal conditioning, over a paged cached prefix.
+* ``edit_decide``       -- the T2T edit set of Eq. 2 (argmax, confidence,
+  threshold-and-replace).
+* ``kv_window_write``   -- Sec. 4.3 targeted refresh: window K/V written to
+  the paged cache at positions [P, P+W).
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` may import it. It shares no code with the CUDA library and never
+imports it. The arithmetic lives in ``mbe_oracle.c`` (compiled with gcc, no
+fast-math); this module only marshals numpy arrays.
+
+Parity status: every function is pinned by tests in ``tests/test_oracle_*.py``
+against library routines (torch float64 SDPA / softmax), closed forms and
+invariants; nothing here is "parity unpinned".
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+from pathlib import Path
+
+import numpy as np
+
+_HERE = Path(__file__).resolve().parent
+_SRC = _HERE / "mbe_oracle.c"
+_BUILD = _HERE / "_build"
+_LIB_PATH = _BUILD / "libmbe_oracle.so"
+_lib = None
+
+STATUS = {0: "ok", 1: "bad argument", 2: "page id out of range", 3: "non-finite logit", 4: "out of memory"}
+
+
+def build(force: bool = False) -> Path:
+    """Compile the oracle's C source into a shared library (gcc, OpenMP, -O2)."""
+    _BUILD.mkdir(exist_ok=True)
+    if force or not _LIB_PATH.exists() or _LIB_PATH.stat().st_mtime < _SRC.stat().st_mtime:
+        tmp = _LIB_PATH.with_suffix(".so.tmp%d" % os.getpid())
+        cmd = ["gcc", "-O2", "-std=c11", "-fopenmp", "-fPIC", "-shared", "-o", str(tmp), str(_SRC), "-lm"]
+        subprocess.run(cmd, check=True)
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        build()
+        lib = ctypes.CDLL(str(_LIB_PATH))
+        P = ctypes.c_void_p
+        i32, i64, f32, f64 = ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_double
+        lib.oracle_num_threads.restype = ctypes.c_int
+        lib.oracle_window_attention.restype = ctypes.c_int
+        lib.oracle_window_attention.argtypes = [P, P, P, P, P, P, i32, P, P, P, P, i32, i32, i32, i32, i32, i32,
+                                                i32, f64, i32, P, P, P, P]
+        lib.oracle_edit_decide.restype = ctypes.c_int
+        lib.oracle_edit_decide.argtypes = [P, i32, i64, i32, i32, P, P, f32, P, i32, P, P, P, P, P]
+        lib.oracle_kv_window_write.restype = ctypes.c_int
+        lib.oracle_kv_window_write.argtypes = [P, P, P, P, P, i32, P, P, P, P, i32, i32, i32, i32, i32, i32, i32]
+        _lib = lib
+    return _lib
+
+
+def num_threads() -> int:
+    return int(_load().oracle_num_threads())
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _c(a, dtype):
+    return None if a is None else np.ascontiguousarray(a, dtype=dtype)
+
+
+def _check(rc):
+    if rc != 0:
+        raise RuntimeError("oracle: " + STATUS.get(rc, str(rc)))
+
+
+def window_attention(q, k_win, v_win, k_cache, v_cache, block_table, prefix_len, window_len, cu_window,
+                     mask_mode, block_size, page_size, scale=None, units=None):
+    """Window attention (Eq. 5, Sec. 2.2) in float64.
+
+    q: uint16 bf16 bits [T, Hq, D]; k_win/v_win: [T, Hkv, D];
+    k_cache/v_cache: [num_pages, Hkv, page_size, D]; block_table: int32
+    [batch, max_pages]; prefix_len/window_len: int32 [batch]; cu_window: int32
+    [batch+1]; mask_mode: uint8 [batch] (0 block_causal, 1 bidirectional).
+    units: optional list of (seq, q_head) pairs to compute (others stay NaN).
+    Returns (out float64 [T, Hq, D], lse float64 [T, Hq]).
+    """
+    lib = _load()
+    q = _c(q, np.uint16)
+    T, Hq, D = q.shape
+    Hkv = k_win.shape[1]
+    num_pages = k_cache.shape[0]
+    block_table = _c(block_table, np.int32)
+    batch = block_table.shape[0]
+    if scale is None:
+        scale = 1.0 / np.sqrt(D)
+    out = np.full((T, Hq, D), np.nan, dtype=np.float64)
+    lse = np.full((T, Hq), np.nan, dtype=np.float64)
+    if units is None:
+        n_units, us, uh = -1, None, None
+    else:
+        units = np.asarray(units, dtype=np.int32).reshape(-1, 2)
+        n_units = units.shape[0]
+        us, uh = np.ascontiguousarray(units[:, 0]), np.ascontiguousarray(units[:, 1])
+    args = [_c(k_win, np.uint16), _c(v_win, np.uint16), _c(k_cache, np.uint16), _c(v_cache, np.uint16)]
+    pl, wl, cu, mm = _c(prefix_len, np.int32), _c(window_len, np.int32), _c(cu_window, np.int32), _c(mask_mode, np.uint8)
+    rc = lib.oracle_window_attention(_ptr(q), *[_ptr(a) for a in args], _ptr(block_table), block_table.shape[1],
+                                     _ptr(pl), _ptr(wl), _ptr(cu), _ptr(mm), batch, Hq, Hkv, D, block_size,
+                                     page_size, num_pages, float(scale), n_units, _ptr(us), _ptr(uh), _ptr(out),
+                                     _ptr(lse))
+    _check(rc)
+    return out, lse
+
+
+def edit_decide(logits, committed, tau=0.0, tau_per_row=None, editable=None, rows=None, is_bf16=False):
+    """T2T edit decision of Eq. 2 in float64.
+
+    logits: float32 [R, V] or uint16 bf16 bits [R, V] (set is_bf16).
+    Returns dict of new_tokens int32, edit_mask uint8, confidence float64,
+    argmax int32 (all [R]; rows not in `rows` are left as -1 / 0 / NaN).
+    """
+    lib = _load()
+    logits = np.ascontiguousarray(logits)
+    R, V = logits.shape
+    committed = _c(committed, np.int32)
+    tpr = _c(tau_per_row, np.float32)
+    ed = _c(editable, np.uint8)
+    new = np.full(R, -1, dtype=np.int32)
+    mask = np.zeros(R, dtype=np.uint8)
+    conf = np.full(R, np.nan, dtype=np.float64)
+    am = np.full(R, -1, dtype=np.int32)
+    sel = None if rows is None else np.ascontiguousarray(rows, dtype=np.int32)
+    dtype = 1 if is_bf16 else 0
+    if not is_bf16:
+        logits = np.ascontiguousarray(logits, dtype=np.float32)
+    rc = lib.oracle_edit_decide(_ptr(logits), dtype, V, R, V, _ptr(committed), _ptr(tpr), float(tau), _ptr(ed),
+                                -1 if sel is None else sel.shape[0], _ptr(sel), _ptr(new), _ptr(mask), _ptr(conf),
+                                _ptr(am))
+    _check(rc)
+    return {"new_tokens": new, "edit_mask": mask, "confidence": conf, "argmax": am}
+
+
+def kv_window_write(k_win, v_win, k_cache, v_cache, block_table, prefix_len, window_len, cu_window, block_size,
+                    block_write_mask=None):
+    """Targeted-refresh KV write (Sec. 4.3). Returns new (k_cache, v_cache) copies."""
+    lib = _load()
+    kc = np.array(k_cache, dtype=np.uint16, copy=True)
+    vc = np.array(v_cache, dtype=np.uint16, copy=True)
+    num_pages, Hkv, page_size, D = kc.shape
+    bt = _c(block_table, np.int32)
+    batch = bt.shape[0]
+    bwm = _c(block_write_mask, np.uint8)
+    maxb = 0 if bwm is None else bwm.shape[1]
+    rc = lib.oracle_kv_window_write(_ptr(_c(k_win, np.uint16)), _ptr(_c(v_win, np.uint16)), _ptr(kc), _ptr(vc),
+                                    _ptr(bt), bt.shape[1], _ptr(_c(prefix_len, np.int32)),
+                                    _ptr(_c(window_len, np.int32)), _ptr(_c(cu_window, np.int32)), _ptr(bwm), maxb,
+                                    batch, Hkv, D, block_size, page_size, num_pages)
+    _check(rc)
+    return kc, vc

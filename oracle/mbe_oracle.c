@@ -1,0 +1,292 @@
+/*
+ * mbe_oracle.c -- plain, slow, obviously-correct CPU oracle for the hot path
+ * of Multi-Block Editing (MBE): the editing pass's window attention, the T2T
+ * edit decision, and the KV window write.
+ *
+ * TEST INFRASTRUCTURE ONLY. Nothing on the product path may call this code:
+ * only the tests, the smoke check and the benchmark's CPU-baseline leg use it.
+ * It shares no code, header, table or helper with the CUDA library.
+ *
+ * Arithmetic: inputs are bf16 (or fp32) values widened exactly to double;
+ * every sum, exponential and division is done in double precision. Masks are
+ * built explicitly as boolean arrays before any score is computed.
+ *
+ * Citations are to the paper (arXiv 2607.22663, "Multi-Block Editing"):
+ *   Sec. 2.2   block diffusion: block j spans [jB,(j+1)B) and conditions on
+ *              the committed prefix.
+ *   Eq. 2      T2T edit set: a visible token is overwritten by the argmax
+ *              prediction iff prediction != token and confidence > omega_edit.
+ *   Eq. 5      editing window W_j = [j* B, (j+1) B) with full attention inside
+ *              the window (Sec. 4.1 "Inference algorithm").
+ *   Sec. 4.3   cache control: the editing pass reads the cached history and
+ *              writes no KV; changed blocks are later recomputed under standard
+ *              (block-causal) attention and their KV written back.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+#define ORC_OK 0
+#define ORC_BAD_ARG 1
+#define ORC_BAD_PAGE 2
+#define ORC_NONFINITE 3
+#define ORC_NOMEM 4
+
+/* bf16 bit pattern -> exact double */
+static double bf16_to_double(uint16_t b) {
+  uint32_t u = ((uint32_t)b) << 16;
+  float f;
+  memcpy(&f, &u, sizeof f);
+  return (double)f;
+}
+
+int oracle_num_threads(void) {
+#ifdef _OPENMP
+  return omp_get_max_threads();
+#else
+  return 1;
+#endif
+}
+
+/*
+ * Window attention of one editing (or standard) pass, Eq. 5 and Sec. 2.2.
+ *
+ * For sequence s with committed prefix length P = prefix_len[s] and window
+ * length W = window_len[s], the key sequence is the P cached prefix tokens
+ * (read from the paged cache through block_table) followed by the W window
+ * tokens of this pass (k_win/v_win rows cu_window[s] .. cu_window[s]+W-1).
+ *
+ * Visibility of key j to window query i (both window-local for the window):
+ *   prefix key                          : always visible
+ *   window key, multi_block_bidirectional (mode 1): visible  (full attention
+ *                                          inside W_j, Eq. 5)
+ *   window key, block_causal (mode 0)   : visible iff floor(j/B) <= floor(i/B)
+ *                                          (a block sees earlier blocks and
+ *                                          itself, Sec. 2.2)
+ * Query head h reads kv head h / (Hq/Hkv).
+ *
+ * out[t, h, :] = sum_j softmax_j(scale * q.k_j) v_j over visible j  (double)
+ * lse[t, h]    = log sum_j exp(scale * q.k_j)                       (double)
+ *
+ * If n_units >= 0, only the (unit_seq[u], unit_qhead[u]) pairs are computed
+ * (all window rows of that pair); otherwise every (seq, head) is computed.
+ */
+int oracle_window_attention(const uint16_t* q, const uint16_t* k_win, const uint16_t* v_win,
+                            const uint16_t* k_cache, const uint16_t* v_cache, const int32_t* block_table,
+                            int32_t max_pages_per_seq, const int32_t* prefix_len, const int32_t* window_len,
+                            const int32_t* cu_window, const uint8_t* mask_mode, int32_t batch, int32_t Hq,
+                            int32_t Hkv, int32_t D, int32_t block_size, int32_t page_size, int32_t num_pages,
+                            double scale, int32_t n_units, const int32_t* unit_seq, const int32_t* unit_qhead,
+                            double* out, double* lse) {
+  if (batch < 0 || Hq <= 0 || Hkv <= 0 || Hq % Hkv != 0 || D <= 0 || block_size <= 0 || page_size <= 0)
+    return ORC_BAD_ARG;
+  const int64_t total = n_units >= 0 ? n_units : (int64_t)batch * Hq;
+  const int32_t group = Hq / Hkv;
+  int status = ORC_OK;
+
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int64_t u = 0; u < total; ++u) {
+    int32_t s, h;
+    if (n_units >= 0) {
+      s = unit_seq[u];
+      h = unit_qhead[u];
+    } else {
+      s = (int32_t)(u / Hq);
+      h = (int32_t)(u % Hq);
+    }
+    if (s < 0 || s >= batch || h < 0 || h >= Hq) {
+#pragma omp atomic write
+      status = ORC_BAD_ARG;
+      continue;
+    }
+    const int32_t P = prefix_len[s], W = window_len[s], t0 = cu_window[s];
+    const int32_t g = h / group;
+    const int32_t nk = P + W;
+    if (W == 0) continue;
+    if (P < 0 || W < 0 || (P + page_size - 1) / page_size > max_pages_per_seq) {
+#pragma omp atomic write
+      status = ORC_BAD_ARG;
+      continue;
+    }
+    /* key and value rows (pointers into the inputs), logical order */
+    const uint16_t** krow = (const uint16_t**)malloc(sizeof(uint16_t*) * (size_t)(nk > 0 ? nk : 1));
+    const uint16_t** vrow = (const uint16_t**)malloc(sizeof(uint16_t*) * (size_t)(nk > 0 ? nk : 1));
+    unsigned char* mask = (unsigned char*)malloc((size_t)W * (size_t)(nk > 0 ? nk : 1));
+    double* z = (double*)malloc(sizeof(double) * (size_t)(nk > 0 ? nk : 1));
+    if (!krow || !vrow || !mask || !z) {
+      free(krow); free(vrow); free(mask); free(z);
+#pragma omp atomic write
+      status = ORC_NOMEM;
+      continue;
+    }
+    int bad = 0;
+    for (int32_t j = 0; j < P; ++j) {
+      const int32_t page = block_table[(int64_t)s * max_pages_per_seq + j / page_size];
+      if (page < 0 || page >= num_pages) { bad = 1; break; }
+      const int64_t off = (((int64_t)page * Hkv + g) * page_size + (j % page_size)) * D;
+      krow[j] = k_cache + off;
+      vrow[j] = v_cache + off;
+    }
+    for (int32_t j = 0; j < W; ++j) {
+      const int64_t off = ((int64_t)(t0 + j) * Hkv + g) * D;
+      krow[P + j] = k_win + off;
+      vrow[P + j] = v_win + off;
+    }
+    if (bad) {
+      free(krow); free(vrow); free(mask); free(z);
+#pragma omp atomic write
+      status = ORC_BAD_PAGE;
+      continue;
+    }
+    /* explicit boolean mask M[i][j] */
+    for (int32_t i = 0; i < W; ++i) {
+      for (int32_t j = 0; j < nk; ++j) {
+        unsigned char vis;
+        if (j < P) {
+          vis = 1;
+        } else if (mask_mode[s] == 1) {
+          vis = 1;
+        } else {
+          const int32_t w = j - P;
+          vis = (w / block_size) <= (i / block_size);
+        }
+        mask[(int64_t)i * nk + j] = vis;
+      }
+    }
+    for (int32_t i = 0; i < W; ++i) {
+      const uint16_t* qi = q + ((int64_t)(t0 + i) * Hq + h) * D;
+      double m = -INFINITY;
+      for (int32_t j = 0; j < nk; ++j) {
+        if (!mask[(int64_t)i * nk + j]) continue;
+        double dot = 0.0;
+        for (int32_t d = 0; d < D; ++d) dot += bf16_to_double(qi[d]) * bf16_to_double(krow[j][d]);
+        z[j] = scale * dot;
+        if (z[j] > m) m = z[j];
+      }
+      double zsum = 0.0;
+      for (int32_t j = 0; j < nk; ++j)
+        if (mask[(int64_t)i * nk + j]) zsum += exp(z[j] - m);
+      double* oi = out + ((int64_t)(t0 + i) * Hq + h) * D;
+      for (int32_t d = 0; d < D; ++d) oi[d] = 0.0;
+      for (int32_t j = 0; j < nk; ++j) {
+        if (!mask[(int64_t)i * nk + j]) continue;
+        const double p = exp(z[j] - m) / zsum;
+        for (int32_t d = 0; d < D; ++d) oi[d] += p * bf16_to_double(vrow[j][d]);
+      }
+      if (lse) lse[(int64_t)(t0 + i) * Hq + h] = m + log(zsum);
+    }
+    free(krow); free(vrow); free(mask); free(z);
+  }
+  return status;
+}
+
+/*
+ * T2T edit decision of Eq. 2 for the rows of one editing pass.
+ *
+ * For row r with logits l[r, 0..V-1]:
+ *   x_hat = argmax_v l[r, v]      (ties: the lowest index)
+ *   c     = p(x_hat) = exp(l[x_hat]) / sum_v exp(l[v]) = 1 / sum_v exp(l[v] - l[x_hat])
+ *   edit  = editable[r] && x_hat != committed[r] && c > tau_r
+ *   new   = edit ? x_hat : committed[r]
+ * tau_r is tau_per_row[r] when given, else tau. The comparison c > tau_r is
+ * taken on c rounded to float, the precision of tau. editable == NULL means
+ * every row is editable (the caller restricts edits to the historical part of
+ * the window, Sec. 4.1).
+ * dtype 0: float32 logits, dtype 1: bf16 logits. If n_sel >= 0 only rows
+ * sel_rows[0..n_sel-1] are computed; outputs are indexed by row.
+ */
+int oracle_edit_decide(const void* logits, int32_t dtype, int64_t row_stride, int32_t rows, int32_t vocab,
+                       const int32_t* committed, const float* tau_per_row, float tau, const uint8_t* editable,
+                       int32_t n_sel, const int32_t* sel_rows, int32_t* new_tokens, uint8_t* edit_mask,
+                       double* confidence, int32_t* argmax_out) {
+  if (rows < 0 || vocab <= 0 || (dtype != 0 && dtype != 1) || row_stride < vocab) return ORC_BAD_ARG;
+  const int64_t total = n_sel >= 0 ? n_sel : rows;
+  int status = ORC_OK;
+#pragma omp parallel for schedule(static)
+  for (int64_t u = 0; u < total; ++u) {
+    const int32_t r = n_sel >= 0 ? sel_rows[u] : (int32_t)u;
+    if (r < 0 || r >= rows) {
+#pragma omp atomic write
+      status = ORC_BAD_ARG;
+      continue;
+    }
+    double m = -INFINITY;
+    int32_t xh = -1;
+    int finite = 1;
+    for (int32_t v = 0; v < vocab; ++v) {
+      double x;
+      if (dtype == 0) {
+        x = (double)((const float*)logits)[(int64_t)r * row_stride + v];
+      } else {
+        x = bf16_to_double(((const uint16_t*)logits)[(int64_t)r * row_stride + v]);
+      }
+      if (!isfinite(x)) finite = 0;
+      if (x > m) {
+        m = x;
+        xh = v;
+      }
+    }
+    if (!finite) {
+#pragma omp atomic write
+      status = ORC_NONFINITE;
+      continue;
+    }
+    double ssum = 0.0;
+    for (int32_t v = 0; v < vocab; ++v) {
+      double x;
+      if (dtype == 0) {
+        x = (double)((const float*)logits)[(int64_t)r * row_stride + v];
+      } else {
+        x = bf16_to_double(((const uint16_t*)logits)[(int64_t)r * row_stride + v]);
+      }
+      ssum += exp(x - m);
+    }
+    const double c = 1.0 / ssum;
+    const float tr = tau_per_row ? tau_per_row[r] : tau;
+    const int ed = (editable == NULL || editable[r] != 0) && xh != committed[r] && ((float)c > tr);
+    if (new_tokens) new_tokens[r] = ed ? xh : committed[r];
+    if (edit_mask) edit_mask[r] = (uint8_t)ed;
+    if (confidence) confidence[r] = c;
+    if (argmax_out) argmax_out[r] = xh;
+  }
+  return status;
+}
+
+/*
+ * KV window write (Sec. 4.3 targeted refresh): the K/V of window token i of
+ * sequence s is stored at logical cache position P + i, i.e. in page
+ * block_table[s][(P+i) / page_size], slot (P+i) % page_size, for every kv head.
+ * If block_write_mask is given ([batch, max_blocks_per_seq] bytes), window
+ * block b = i / block_size is written only where block_write_mask[s][b] != 0
+ * (only the blocks whose tokens changed are refreshed).
+ */
+int oracle_kv_window_write(const uint16_t* k_win, const uint16_t* v_win, uint16_t* k_cache, uint16_t* v_cache,
+                           const int32_t* block_table, int32_t max_pages_per_seq, const int32_t* prefix_len,
+                           const int32_t* window_len, const int32_t* cu_window, const uint8_t* block_write_mask,
+                           int32_t max_blocks_per_seq, int32_t batch, int32_t Hkv, int32_t D, int32_t block_size,
+                           int32_t page_size, int32_t num_pages) {
+  if (batch < 0 || Hkv <= 0 || D <= 0 || block_size <= 0 || page_size <= 0) return ORC_BAD_ARG;
+  for (int32_t s = 0; s < batch; ++s) {
+    const int32_t P = prefix_len[s], W = window_len[s], t0 = cu_window[s];
+    for (int32_t i = 0; i < W; ++i) {
+      if (block_write_mask && !block_write_mask[(int64_t)s * max_blocks_per_seq + i / block_size]) continue;
+      const int32_t pos = P + i;
+      if (pos / page_size >= max_pages_per_seq) return ORC_BAD_ARG;
+      const int32_t page = block_table[(int64_t)s * max_pages_per_seq + pos / page_size];
+      if (page < 0 || page >= num_pages) return ORC_BAD_PAGE;
+      for (int32_t g = 0; g < Hkv; ++g) {
+        const int64_t dst = (((int64_t)page * Hkv + g) * page_size + pos % page_size) * D;
+        const int64_t src = ((int64_t)(t0 + i) * Hkv + g) * D;
+        for (int32_t d = 0; d < D; ++d) {
+          k_cache[dst + d] = k_win[src + d];
+          v_cache[dst + d] = v_win[src + d];
+        }
+      }
+    }
+  }
+  return ORC_OK;
+}

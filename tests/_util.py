@@ -1,0 +1,36 @@
+"""Helpers shared by the tests: dense re-gathering of paged K/V (independent of
+both the oracle and the CUDA path) and bf16 conversions."""
+import numpy as np
+import torch
+
+from paper_2607_22663_gb300.workloads import bf16_bits
+
+
+def dense_keys(prob, s, g):
+    """Logical key/value rows [P+W, D] (float64) of sequence s, kv head g, gathered
+    with torch indexing from the paged cache and the window tensors."""
+    P, W = prob.prefix_host[s], prob.window_host[s]
+    ps = prob.page_size
+    pos = torch.arange(P)
+    pages = prob.block_table[s].cpu()[pos // ps].long()
+    kp = prob.k_cache.cpu()[pages, g, pos % ps].double()
+    vp = prob.v_cache.cpu()[pages, g, pos % ps].double()
+    t0 = int(prob.cu_window.cpu()[s])
+    kw = prob.k_win.cpu()[t0:t0 + W, g].double()
+    vw = prob.v_win.cpu()[t0:t0 + W, g].double()
+    return torch.cat([kp, kw]), torch.cat([vp, vw])
+
+
+def oracle_attention(prob, units=None, scale=None):
+    import oracle
+    return oracle.window_attention(bf16_bits(prob.q), bf16_bits(prob.k_win), bf16_bits(prob.v_win),
+                                   bf16_bits(prob.k_cache), bf16_bits(prob.v_cache),
+                                   prob.block_table.cpu().numpy(), prob.prefix_len.cpu().numpy(),
+                                   prob.window_len.cpu().numpy(), prob.cu_window.cpu().numpy(),
+                                   prob.mask_mode.cpu().numpy(), prob.block_size, prob.page_size, scale=scale,
+                                   units=units)
+
+
+def to_bf16_round(x: np.ndarray) -> np.ndarray:
+    """Round float64 values to the nearest bf16 (ties to even), returned as float64."""
+    return torch.from_numpy(np.ascontiguousarray(x)).to(torch.bfloat16).double().numpy()
