@@ -1,0 +1,456 @@
+"""Benchmark of one MBE editing pass on synthetic decoding-shaped data.
+
+A step is one editing pass of the whole hot path over one batch: window
+attention for every layer (one mbe_window_attention call per layer) followed
+by mbe_edit_decide over the pass's logits; workloads that include the cache
+refresh also run mbe_kv_window_write. Inputs are resident in HBM when the timed
+region starts. The default workload is the decode-heavy serving mix
+(128 sequences, prefix U[512,16384], window 64, 32/8 heads, head_dim 128,
+24 layers, vocabulary 131072).
+
+Prints one JSON line (rank 0). ``--impl reference`` times the CPU oracle on a
+bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "edit-pass attn TFLOP/s (% bf16 peak); edit-decide GB/s (% HBM); windows/s"
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return {k: float(d[k]) for k in PEAKS_FALLBACK}, "measured"
+    except Exception:
+        return dict(PEAKS_FALLBACK), "fallback"
+
+
+# ------------------------------------------------------------------ accounting
+def attention_flops(prefix, window, modes, num_q_heads, head_dim, block_size):
+    """Mask-aware algorithmic FLOPs: 4 * D per visible (query, key) pair and
+    query head (QK^T and PV, one multiply-add = 2 FLOPs each)."""
+    pairs = 0
+    for P, W, m in zip(prefix, window, modes):
+        if m == 1:
+            pairs += W * (P + W)
+        else:
+            for i in range(W):
+                pairs += P + min(W, (i // block_size + 1) * block_size)
+    return 4 * head_dim * num_q_heads * pairs
+
+
+def attention_bytes(prefix, window, num_q_heads, num_kv_heads, head_dim):
+    """Algorithmic HBM bytes: each prefix and window K/V row read once, Q read
+    once, O written once (bf16)."""
+    kv = sum(P + W for P, W in zip(prefix, window)) * num_kv_heads * head_dim * 2 * 2
+    qo = sum(window) * num_q_heads * head_dim * 2 * 2
+    return kv + qo
+
+
+def edit_bytes(rows, vocab, elem):
+    """Logits read once + committed read + new token, mask, confidence written."""
+    return rows * vocab * elem + rows * (4 + 4 + 1 + 4)
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={q}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        try:
+            for line in open(self.path):
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+            os.unlink(self.path)
+        except Exception:
+            pass
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        smax = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ------------------------------------------------------------------ workloads
+def build_workload(name, device, layers=None, batch=None):
+    from paper_2607_22663_gb300 import workloads as wl
+    if name == "serving128":
+        return wl.serving128(device, layers=layers or 24, batch=batch or 128)
+    return wl.WORKLOADS[name](device)
+
+
+def workload_config(w):
+    a = w["attn"][0]
+    cfg = {"workload": w["name"], "batch": a.batch, "layers": w["layers"], "attn_calls_per_step": len(w["attn"]),
+           "window": sorted(set(a.window_host)), "prefix_range": [min(a.prefix_host), max(a.prefix_host)],
+           "heads_q_kv": [a.num_q_heads, a.num_kv_heads], "head_dim": a.head_dim, "block_size": a.block_size,
+           "page_size": a.page_size}
+    if w.get("edit") is not None:
+        cfg["edit_rows_vocab"] = list(w["edit"].logits.shape)
+    return cfg
+
+
+# ------------------------------------------------------------------ GPU arm
+def run_gpu(args, rank, world):
+    from paper_2607_22663_gb300 import mbe
+    from paper_2607_22663_gb300.workloads import editable_historical
+
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(dev)
+    peaks, peak_src = load_peaks()
+    w = build_workload(args.workload, dev, args.layers, args.batch)
+    attn = w["attn"]
+    ep = w["edit"]
+    with_kv_write = args.workload == "long32k"
+    a0 = attn[0]
+    editable = editable_historical(a0.window_host, a0.block_size, dev) if ep is not None else None
+    stream = torch.cuda.current_stream()
+
+    # per-call buffers: outputs, workspaces and per-call events
+    outs = [torch.empty_like(a.q) for a in attn]
+    # one workspace serves every call: the calls run in order on one stream
+    need = max(mbe.window_attention_workspace_size(a.batch, a.num_q_heads, a.num_kv_heads, a.head_dim, a.max_window,
+                                                   a.max_prefix) for a in attn)
+    ws = torch.empty(need, dtype=torch.uint8, device=dev)
+    wss = [ws] * len(attn)
+    if ep is not None:
+        R = ep.logits.shape[0]
+        new_t = torch.empty(R, dtype=torch.int32, device=dev)
+        mask_t = torch.empty(R, dtype=torch.uint8, device=dev)
+        conf_t = torch.empty(R, dtype=torch.float32, device=dev)
+
+    def attention_call(i, a, q=None, kw=None, vw=None):
+        mbe.window_attention(a.q if q is None else q, a.k_win if kw is None else kw, a.v_win if vw is None else vw,
+                             a.k_cache, a.v_cache, a.block_table, a.prefix_len, a.window_len, a.cu_window,
+                             a.mask_mode, block_size=a.block_size, max_window=a.max_window, max_prefix=a.max_prefix,
+                             out=outs[i], workspace=wss[i])
+
+    def edit_call(logits=None, committed=None):
+        mbe.edit_decide(ep.logits if logits is None else logits, ep.committed if committed is None else committed,
+                        tau=ep.tau, tau_per_row=ep.tau_per_row, editable=editable, new_tokens=new_t,
+                        edit_mask=mask_t, confidence=conf_t, want_argmax=False)
+
+    def step(attn_events=None, edit_events=None):
+        for i, a in enumerate(attn):
+            if attn_events is not None:
+                attn_events[i][0].record(stream)
+            attention_call(i, a)
+            if attn_events is not None:
+                attn_events[i][1].record(stream)
+            if with_kv_write:
+                mbe.kv_window_write(a.k_win, a.v_win, a.k_cache, a.v_cache, a.block_table, a.prefix_len,
+                                    a.window_len, a.cu_window, block_size=a.block_size, max_window=a.max_window)
+        if ep is not None:
+            if edit_events is not None:
+                edit_events[0].record(stream)
+            edit_call()
+            if edit_events is not None:
+                edit_events[1].record(stream)
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+
+    for _ in range(args.warmup):
+        step()
+    st, flags = mbe.get_device_error()
+    if st != 0:
+        raise RuntimeError(f"device error during warm-up: status {st} flags {flags:#x}")
+
+    K = args.steps
+    ev_attn = [[[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in attn] for _ in range(K)]
+    ev_edit = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(dev.index) as clk:
+        barrier()
+        t0.record(stream)
+        for k in range(K):
+            step(ev_attn[k], ev_edit[k] if ep is not None else None)
+        t1.record(stream)
+        barrier()
+    clocks = clk.summary()
+    ms_total = t0.elapsed_time(t1)
+    if world > 1:
+        tt = torch.tensor([ms_total], device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        ms_total = float(tt.item())
+    ms_step = ms_total / K
+    attn_ms = [statistics.mean(ev_attn[k][i][0].elapsed_time(ev_attn[k][i][1]) for k in range(K))
+               for i in range(len(attn))]
+    edit_ms = statistics.mean(ev_edit[k][0].elapsed_time(ev_edit[k][1]) for k in range(K)) if ep is not None else None
+    st, flags = mbe.get_device_error()
+    if st != 0:
+        raise RuntimeError(f"device error during timing: status {st} flags {flags:#x}")
+
+    flops = [attention_flops(a.prefix_host, a.window_host, a.mode_host, a.num_q_heads, a.head_dim, a.block_size)
+             for a in attn]
+    abytes = [attention_bytes(a.prefix_host, a.window_host, a.num_q_heads, a.num_kv_heads, a.head_dim) for a in attn]
+    attn_time = sum(attn_ms)
+    attn_tflops = sum(flops) / (attn_time * 1e-3) / 1e12
+    attn_gbs = sum(abytes) / (attn_time * 1e-3) / 1e9
+    windows = a0.batch * world
+    value = windows / (ms_step * 1e-3)
+    res = {"metric": METRIC, "value": round(value, 3), "unit": "windows/s", "n_gpus": world, "steps": K,
+           "warmup": args.warmup, "ms_per_step": round(ms_step, 4), "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+           "config": {**workload_config(w), "l2": "inputs larger than L2 (per-layer KV cache and logits >> 129 MB)",
+                      "parallelism": f"replicas{world}"}}
+    res["attention"] = {"tflops": round(attn_tflops, 2),
+                        "frac_bf16_peak_sustained": round(attn_tflops / peaks["bf16_tflops_sustained"], 4),
+                        "frac_bf16_peak_burst": round(attn_tflops / peaks["bf16_tflops"], 4),
+                        "gbs": round(attn_gbs, 1), "frac_hbm": round(attn_gbs / peaks["hbm_gbs"], 4),
+                        "ms_per_call": round(attn_time / len(attn), 4), "flops_per_call": flops[0],
+                        "bytes_per_call": abytes[0]}
+    if ep is not None:
+        eb = edit_bytes(ep.logits.shape[0], ep.logits.shape[1], ep.logits.element_size())
+        res["edit_decide"] = {"gbs": round(eb / (edit_ms * 1e-3) / 1e9, 1),
+                              "frac_hbm": round(eb / (edit_ms * 1e-3) / 1e9 / peaks["hbm_gbs"], 4),
+                              "ms": round(edit_ms, 4), "bytes": eb,
+                              "edit_rate": round(float(mask_t.float().mean().item()), 5)}
+    res["roofline"] = {"bound": "hbm", "achieved": round(attn_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                       "frac": round(attn_gbs / peaks["hbm_gbs"], 4), "traffic": None,
+                       "kernel": "mbe_window_attention (schedule + attn_kernel + merge)",
+                       "peak_source": f"{peak_src} hbm_gbs"}
+    res["clocks"] = clocks
+    per_step = len(attn) * 3 + (1 if ep is not None else 0) + (len(attn) if with_kv_write else 0)
+    res["gpu_launches"] = per_step * K
+    res["e2e"] = run_e2e(args, w, attention_call, edit_call, dev, stream, world, new_t if ep is not None else None,
+                         mask_t if ep is not None else None, conf_t if ep is not None else None)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        v, desc, spent = run_cpu_sample(w, target_s=15.0)
+        res["cpu_baseline"] = {"value": round(v, 5), "unit": "windows/s", "cores": oracle.num_threads(),
+                               "kind": "oracle", "sample": desc}
+    return res
+
+
+def run_e2e(args, w, attention_call, edit_call, dev, stream, world, new_t, mask_t, conf_t):
+    """Same pass through the public API with the per-step inputs (window Q/K/V
+    of every layer, logits, committed tokens) copied from pinned host memory
+    and the step's result (new tokens, edit mask, confidence) read back. The
+    paged KV caches are resident state, as in serving. Copies of layer l+1 run
+    on a second stream while layer l computes."""
+    attn = w["attn"]
+    ep = w["edit"]
+    host = []
+    dbuf = []
+    for a in attn:
+        host.append(tuple(t.cpu().pin_memory() for t in (a.q, a.k_win, a.v_win)))
+        dbuf.append(tuple(torch.empty_like(t) for t in (a.q, a.k_win, a.v_win)))
+    if ep is not None:
+        lg_h = ep.logits.cpu().pin_memory()
+        cm_h = ep.committed.cpu().pin_memory()
+        lg_d = torch.empty_like(ep.logits)
+        cm_d = torch.empty_like(ep.committed)
+        R = ep.logits.shape[0]
+        out_h = [torch.empty(R, dtype=t.dtype, pin_memory=True) for t in (new_t, mask_t, conf_t)]
+    copy_stream = torch.cuda.Stream(dev)
+    h2d = sum(t.numel() * t.element_size() for hs in host for t in hs)
+    if ep is not None:
+        h2d += lg_h.numel() * lg_h.element_size() + cm_h.numel() * cm_h.element_size()
+    d2h = sum(t.numel() * t.element_size() for t in out_h) if ep is not None else 0
+
+    def step():
+        copied = [torch.cuda.Event() for _ in attn]
+        with torch.cuda.stream(copy_stream):
+            for i in range(len(attn)):
+                for d, h in zip(dbuf[i], host[i]):
+                    d.copy_(h, non_blocking=True)
+                copied[i].record(copy_stream)
+            if ep is not None:
+                lg_d.copy_(lg_h, non_blocking=True)
+                cm_d.copy_(cm_h, non_blocking=True)
+                done_l = torch.cuda.Event()
+                done_l.record(copy_stream)
+        for i, a in enumerate(attn):
+            stream.wait_event(copied[i])
+            attention_call(i, a, *dbuf[i])
+        if ep is not None:
+            stream.wait_event(done_l)
+            edit_call(lg_d, cm_d)
+            for h, d in zip(out_h, (new_t, mask_t, conf_t)):
+                h.copy_(d, non_blocking=True)
+        copy_stream.wait_stream(stream)
+
+    for _ in range(max(1, min(args.warmup, 3))):
+        step()
+    torch.cuda.synchronize()
+    K = max(1, min(args.steps, args.e2e_steps))
+    if world > 1:
+        torch.distributed.barrier()
+    t0 = time.perf_counter()
+    for _ in range(K):
+        step()
+    torch.cuda.synchronize()
+    el = time.perf_counter() - t0
+    if world > 1:
+        tt = torch.tensor([el], device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        el = float(tt.item())
+    windows = attn[0].batch * world
+    return {"value": round(windows * K / el, 3), "unit": "windows/s", "h2d_bytes_per_step": int(h2d),
+            "d2h_bytes_per_step": int(d2h), "steps": K,
+            "resident_state": "paged KV caches of every layer (written by earlier passes)"}
+
+
+# ------------------------------------------------------------------ CPU oracle arm
+def run_cpu_sample(w, target_s=15.0, max_seqs=None):
+    """Times the oracle on a bounded sample: a few whole sequences (all heads) of
+    one layer, scaled to the workload's layer count, plus the edit decision of
+    those sequences' rows. Returns windows/s and a description."""
+    import numpy as np
+
+    import oracle
+    from paper_2607_22663_gb300.workloads import bf16_bits
+    from paper_2607_22663_gb300.workloads import extract_sequences as subproblem
+
+    attn = w["attn"]
+    a = attn[0]
+    order = np.argsort(a.prefix_host)
+    # sequences near the median prefix, growing the sample until ~target_s
+    mid = len(order) // 2
+    picks, spent, t_attn = [], 0.0, 0.0
+    rows_timed, t_edit = 0, 0.0
+    ep = w["edit"]
+    k = 0
+    while spent < target_s and k < len(order) and (max_seqs is None or len(picks) < max_seqs):
+        s = int(order[(mid + (k // 2 + 1) * (1 if k % 2 else -1)) % len(order)]) if k else int(order[mid])
+        k += 1
+        sub = subproblem(a, [s])
+        t = time.perf_counter()
+        oracle.window_attention(bf16_bits(sub.q), bf16_bits(sub.k_win), bf16_bits(sub.v_win), bf16_bits(sub.k_cache),
+                                bf16_bits(sub.v_cache), sub.block_table.numpy(), sub.prefix_len.numpy(),
+                                sub.window_len.numpy(), sub.cu_window.numpy(), sub.mask_mode.numpy(),
+                                sub.block_size, sub.page_size)
+        dt = time.perf_counter() - t
+        t_attn += dt
+        picks.append(s)
+        spent += dt
+        if ep is not None:
+            t0 = int(a.cu_window[s])
+            rows = list(range(t0, t0 + a.window_host[s]))
+            lg = ep.logits[rows].cpu()
+            t = time.perf_counter()
+            if lg.dtype == torch.bfloat16:
+                oracle.edit_decide(bf16_bits(lg), ep.committed[rows].cpu().numpy(), tau=ep.tau, is_bf16=True)
+            else:
+                oracle.edit_decide(lg.numpy(), ep.committed[rows].cpu().numpy(), tau=ep.tau)
+            dt = time.perf_counter() - t
+            t_edit += dt
+            spent += dt
+            rows_timed += len(rows)
+    n = len(picks)
+    per_window = t_attn / n * len(attn) + (t_edit / n if ep is not None else 0.0)
+    desc = (f"{n} sequences (prefix {sorted(a.prefix_host[s] for s in picks)}), all {a.num_q_heads} heads, 1 of "
+            f"{len(attn)} layers scaled x{len(attn)}; edit-decide on their {rows_timed} rows; "
+            f"{spent:.1f} s of oracle time")
+    return 1.0 / per_window, desc, spent
+
+
+def run_reference(args, rank, world):
+    import oracle
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    w = build_workload(args.workload, dev, args.layers, args.batch)
+    cores = oracle.num_threads()
+    # each step: one bounded sample sized so warmup+steps finish in minutes
+    per_step_s = max(2.0, min(20.0, 120.0 / max(1, args.steps + args.warmup)))
+    vals = []
+    desc = ""
+    for i in range(args.warmup + args.steps):
+        v, desc, spent = run_cpu_sample(w, target_s=per_step_s)
+        if i >= args.warmup:
+            vals.append(v)
+    value = statistics.mean(vals)
+    res = {"metric": METRIC, "value": round(value, 5), "unit": "windows/s", "n_gpus": world, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": round(1000.0 / value * w["attn"][0].batch, 2) if value else None,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "impl": "reference", "config": {**workload_config(w), "parallelism": "cpu"},
+           "cpu_baseline": {"value": round(value, 5), "unit": "windows/s", "cores": cores, "kind": "oracle",
+                            "sample": desc},
+           "e2e": {"value": round(value, 5), "unit": "windows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    return res
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["gpu", "reference"], default="gpu")
+    ap.add_argument("--workload", default="serving128",
+                    choices=["serving128", "tiny", "batch8", "varlen64", "long32k"])
+    ap.add_argument("--layers", type=int, default=None, help="layer count of the serving workload (default 24)")
+    ap.add_argument("--batch", type=int, default=None, help="sequences of the serving workload (default 128; "
+                    "smaller values are for profiling captures, not bench lines)")
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        print(json.dumps(run_reference(args, rank, world)), flush=True)
+        return
+    if world > 1:
+        torch.distributed.init_process_group("nccl")
+    res = run_gpu(args, rank, world)
+    if rank == 0:
+        print(json.dumps(res), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,890 @@
+// Window attention of an MBE editing pass (Eq. 5; Sec. 2.2; Sec. 4.3) on sm_103a.
+//
+// Three launches on the caller's stream, all sized from host-known bounds so
+// the sequence can be captured in a CUDA graph (shapes are device data):
+//
+//  1. attn_schedule_kernel (1 CTA): reads prefix_len/window_len/mask_mode,
+//     cuts every (sequence, KV head, 256-row query slab) into work units of
+//     key tiles, splits long units so that there are a few units per SM, and
+//     orders them by descending cost (counting sort) for longest-first
+//     dynamic scheduling.
+//  2. attn_kernel (persistent, one CTA per SM, 12 warps):
+//       warp 0      TMA producer: Q slab once per unit, then K/V tiles of 128
+//                   keys into a 2-stage ring (paged prefix via a 4-D tensor
+//                   map with the page id as a coordinate; window via 3-D)
+//       warp 1      MMA issuer: S_i = Q_i K^T (SS form) and O_i += P_i V
+//                   (TS form, P read from TMEM), tcgen05, accumulators in TMEM
+//       warps 4-11  two softmax warpgroups, one per 128-row query tile: TMEM
+//                   load of S, row max, exp2, P written back to TMEM as bf16,
+//                   lazy rescaling of O, epilogue
+//     GQA: the G query heads sharing a KV head are packed into the rows of a
+//     tile (row = token * G + head), so every K/V tile feeds 256 query rows.
+//     The mask is applied per row as a visible-column count: every prefix key
+//     is visible; window keys are visible up to W (bidirectional) or up to
+//     the end of the query's own block (block-causal), and tiles past the
+//     unit's last visible key are never loaded.
+//  3. attn_merge_kernel: combines split-KV partial results by their
+//     log-sum-exp.
+#include <cmath>
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <algorithm>
+#include <mutex>
+#include "common.cuh"
+#include "ptx_sm103.cuh"
+
+namespace mbe {
+
+MBE_DEFINE_ERROR_WORD(attention_take_error)
+
+namespace attn {
+
+constexpr int kTileKeys = 128;      // keys per K/V tile
+constexpr int kTileRows = 128;      // packed query rows per tile (= TMEM lanes)
+constexpr int kUnitRows = 256;      // packed query rows per work unit (two tiles)
+constexpr int kThreads = 384;       // 12 warps
+constexpr int kMinChunk = 8;        // fewest key tiles in a split piece
+constexpr int kSplitFactor = 4;     // target pieces per SM when splitting
+constexpr int kBuckets = 1024;      // counting-sort buckets for unit cost
+constexpr float kRescaleLog2 = 8.0f;  // rescale O only when the max grows by > 2^8
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kTmemS = 256;    // S/P of tile i at columns 256 + 128 i; O_i at i * D
+
+struct WorkUnit {
+  int32_t seq, kv_head, row0, tile_begin, tile_end, slot, prefix, window_mode;  // window_mode = W | mode << 30
+};
+struct MergeGroup {
+  int32_t seq, kv_head, row0, n_splits, slot_base, window, pad0, pad1;
+};
+struct Header {
+  int32_t counter, n_units, n_groups, pad[61];
+};
+static_assert(sizeof(Header) == 256, "header size");
+
+struct Layout {
+  size_t units_tmp, units, groups, part_o, part_lse, total;
+  int64_t max_units, max_groups, max_slots;
+};
+
+inline Layout make_layout(int batch, int Hq, int Hkv, int D, int max_window, int max_prefix, int num_sms) {
+  const int64_t G = Hq / Hkv;
+  const int64_t slabs = (static_cast<int64_t>(max_window) * G + kUnitRows - 1) / kUnitRows;
+  const int64_t n_groups_all = static_cast<int64_t>(batch) * Hkv * slabs;
+  const int64_t t_max = (max_prefix + kTileKeys - 1) / kTileKeys + (max_window + kTileKeys - 1) / kTileKeys;
+  const int64_t total_max = std::max<int64_t>(n_groups_all * t_max, 1);
+  Layout L;
+  L.max_units = std::min<int64_t>(n_groups_all + static_cast<int64_t>(kSplitFactor) * num_sms, total_max) + 1;
+  L.max_groups = std::min<int64_t>(static_cast<int64_t>(kSplitFactor) * num_sms, total_max / kMinChunk) + 1;
+  L.max_slots = std::min<int64_t>(2ll * kSplitFactor * num_sms, 2 * total_max / kMinChunk) + 1;
+  auto up = [](size_t x) { return (x + 255) & ~size_t(255); };
+  size_t off = up(sizeof(Header));
+  L.units_tmp = off; off = up(off + sizeof(WorkUnit) * L.max_units);
+  L.units = off;     off = up(off + sizeof(WorkUnit) * L.max_units);
+  L.groups = off;    off = up(off + sizeof(MergeGroup) * L.max_groups);
+  L.part_o = off;    off = up(off + sizeof(float) * L.max_slots * kUnitRows * D);
+  L.part_lse = off;  off = up(off + sizeof(float) * L.max_slots * kUnitRows);
+  L.total = off;
+  return L;
+}
+
+// ------------------------------------------------------------------ scheduler
+struct SchedParams {
+  const int32_t* prefix_len;
+  const int32_t* window_len;
+  const uint8_t* mask_mode;
+  const int32_t* cu_window;
+  int batch, G, Hkv, block_size, max_window, max_prefix, num_sms, total_tokens;
+  Header* hdr;
+  WorkUnit* units_tmp;
+  WorkUnit* units;
+  MergeGroup* groups;
+  int64_t max_units, max_groups, max_slots;
+};
+
+// Key tiles (prefix, then window) that packed query rows [row0, row0 + 256) need.
+__device__ __forceinline__ int slab_tiles(int P, int W, int mode, int row0, int G, int B) {
+  const int nP = (P + kTileKeys - 1) / kTileKeys;
+  int lim = W;
+  if (mode == MBE_BLOCK_CAUSAL) {
+    const int qmax = min(W, (row0 + kUnitRows) / G) - 1;
+    lim = min(W, (qmax / B + 1) * B);
+  }
+  return nP + (lim + kTileKeys - 1) / kTileKeys;
+}
+
+// A sequence is scheduled only if its lengths are within the declared bounds
+// and its window rows [cu, cu + W) lie inside the q/out tensors.
+__device__ __forceinline__ bool seq_ok(const SchedParams& p, int s, int P, int W, int mode) {
+  if (W < 0 || W > p.max_window || P < 0 || P > p.max_prefix || mode > 1) return false;
+  const int cu = p.cu_window[s];
+  return cu >= 0 && static_cast<int64_t>(cu) + W <= p.total_tokens;
+}
+
+__device__ __forceinline__ int cost_bucket(int cost, int chunk) {
+  const int b = static_cast<int>((static_cast<int64_t>(cost - 1) * kBuckets) / chunk);
+  return min(max(b, 0), kBuckets - 1);
+}
+
+__global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p) {
+  __shared__ int s_total, s_nunits, s_ngroups, s_nslots, s_bad;
+  __shared__ int hist[kBuckets];
+  __shared__ int warp_sums[32];
+  const int tid = threadIdx.x;
+  if (tid == 0) { s_total = 0; s_nunits = 0; s_ngroups = 0; s_nslots = 0; s_bad = 0; }
+  for (int b = tid; b < kBuckets; b += blockDim.x) hist[b] = 0;
+  __syncthreads();
+  // pass 1: validate and count key tiles
+  int local = 0, bad = 0;
+  for (int s = tid; s < p.batch; s += blockDim.x) {
+    const int P = p.prefix_len[s], W = p.window_len[s], mode = p.mask_mode[s];
+    if (!seq_ok(p, s, P, W, mode)) { bad = 1; continue; }
+    const int slabs = (W * p.G + kUnitRows - 1) / kUnitRows;
+    for (int sl = 0; sl < slabs; ++sl) local += slab_tiles(P, W, mode, sl * kUnitRows, p.G, p.block_size) * p.Hkv;
+  }
+  atomicAdd(&s_total, local);
+  if (bad) atomicOr(&s_bad, 1);
+  __syncthreads();
+  const int64_t target = static_cast<int64_t>(kSplitFactor) * p.num_sms;
+  const int chunk = max(kMinChunk, static_cast<int>((s_total + target - 1) / target));
+  // pass 2: emit units (unsorted) and merge groups
+  bool overflow = false;
+  for (int s = tid; s < p.batch; s += blockDim.x) {
+    const int P = p.prefix_len[s], W = p.window_len[s], mode = p.mask_mode[s];
+    if (!seq_ok(p, s, P, W, mode)) continue;
+    const int slabs = (W * p.G + kUnitRows - 1) / kUnitRows;
+    for (int sl = 0; sl < slabs; ++sl) {
+      const int T = slab_tiles(P, W, mode, sl * kUnitRows, p.G, p.block_size);
+      const int n = (T + chunk - 1) / chunk;
+      for (int g = 0; g < p.Hkv; ++g) {
+        const int base = atomicAdd(&s_nunits, n);
+        int slot0 = -1;
+        if (n > 1) {
+          const int gi = atomicAdd(&s_ngroups, 1);
+          slot0 = atomicAdd(&s_nslots, n);
+          if (gi < p.max_groups && slot0 + n <= p.max_slots) {
+            p.groups[gi] = MergeGroup{s, g, sl * kUnitRows, n, slot0, W, 0, 0};
+          } else {
+            overflow = true;
+          }
+        }
+        for (int k = 0; k < n; ++k) {
+          const int tb = static_cast<int>((static_cast<int64_t>(k) * T) / n);
+          const int te = static_cast<int>((static_cast<int64_t>(k + 1) * T) / n);
+          if (base + k < p.max_units) {
+            p.units_tmp[base + k] =
+                WorkUnit{s, g, sl * kUnitRows, tb, te, n > 1 ? slot0 + k : -1, P, W | (mode << 30)};
+            atomicAdd(&hist[cost_bucket(te - tb, chunk)], 1);
+          } else {
+            overflow = true;
+          }
+        }
+      }
+    }
+  }
+  if (overflow) atomicOr(&s_bad, 2);
+  __syncthreads();
+  // exclusive scan of the histogram in descending-cost order
+  {
+    const int lane = tid & 31, warp = tid >> 5;
+    const int b = kBuckets - 1 - tid;  // blockDim.x == kBuckets
+    int v = hist[b];
+    int x = v;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, x, off);
+      if (lane >= off) x += y;
+    }
+    if (lane == 31) warp_sums[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+      int w = warp_sums[lane];
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, w, off);
+        if (lane >= off) w += y;
+      }
+      warp_sums[lane] = w;
+    }
+    __syncthreads();
+    const int excl = x - v + (warp > 0 ? warp_sums[warp - 1] : 0);
+    __syncthreads();
+    hist[b] = excl;
+  }
+  __syncthreads();
+  const bool ok = (s_bad & 2) == 0;
+  const int n_units = ok ? s_nunits : 0;
+  for (int u = tid; u < n_units; u += blockDim.x) {
+    const WorkUnit wu = p.units_tmp[u];
+    const int pos = atomicAdd(&hist[cost_bucket(wu.tile_end - wu.tile_begin, chunk)], 1);
+    p.units[pos] = wu;
+  }
+  if (tid == 0) {
+    p.hdr->counter = 0;
+    p.hdr->n_units = n_units;
+    p.hdr->n_groups = ok ? s_ngroups : 0;
+    if (s_bad & 1) atomicOr(&g_error_word, MBE_DEVERR_LENGTH);
+    if (s_bad & 2) atomicOr(&g_error_word, MBE_DEVERR_CAPACITY);
+  }
+}
+
+// ------------------------------------------------------------------ main kernel
+struct AttnParams {
+  const int32_t* block_table;
+  const int32_t* cu_window;
+  __nv_bfloat16* out;
+  float* lse;
+  Header* hdr;
+  const WorkUnit* units;
+  float* part_o;
+  float* part_lse;
+  int max_pages, num_pages, Hq, G, block_size, page_size, box_rows, loads_per_tile;
+  float scale_log2;
+};
+
+template <int D>
+struct Smem {
+  static constexpr int kHalves = D / 64;
+  static constexpr int kHalfBytes = 128 * 128;             // 128 rows x 128 B
+  static constexpr int kQTile = kTileRows * D * 2;
+  static constexpr int kKVTile = kTileKeys * D * 2;
+  static constexpr int kQ = 0;
+  static constexpr int kK = 2 * kQTile;
+  static constexpr int kV = kK + 2 * kKVTile;
+  static constexpr int kUsed = kV + 2 * kKVTile;
+  // at least 114 KB so that one CTA (and its 512 TMEM columns) owns the SM
+  static constexpr int kBytes = (kUsed > 120 * 1024 ? kUsed : 120 * 1024) + 1024;
+};
+
+__device__ __forceinline__ float ex2f(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float neg_inf() { return __int_as_float(0xff800000u); }
+
+struct Bars {
+  uint64_t q_full, q_empty, mma_done;
+  uint64_t k_full[2], v_full[2], kv_empty[2];
+  uint64_t s_full[2], p_full[2], o_full[2], o_empty[2];
+  uint64_t u_full[2], u_empty[2];
+};
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kw,
+                const __grid_constant__ CUtensorMap tm_vw, const __grid_constant__ CUtensorMap tm_kc,
+                const __grid_constant__ CUtensorMap tm_vc, const AttnParams p) {
+  using S = Smem<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  __shared__ __align__(8) Bars bars;
+  __shared__ WorkUnit unit_ring[2];
+  __shared__ uint32_t tmem_base_s;
+  __shared__ int abort_s;
+  volatile int* abort_flag = &abort_s;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t sbase = smem_u32(smem);
+  auto bar = [](uint64_t& b) { return smem_u32(&b); };
+
+  if (tid == 0) {
+    abort_s = 0;
+    mbar_init(bar(bars.q_full), 1);
+    mbar_init(bar(bars.q_empty), 1);
+    mbar_init(bar(bars.mma_done), 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(bar(bars.k_full[i]), 1);
+      mbar_init(bar(bars.v_full[i]), 1);
+      mbar_init(bar(bars.kv_empty[i]), 1);
+      mbar_init(bar(bars.s_full[i]), 1);
+      mbar_init(bar(bars.p_full[i]), 4);
+      mbar_init(bar(bars.o_full[i]), 1);
+      mbar_init(bar(bars.o_empty[i]), 4);
+      mbar_init(bar(bars.u_full[i]), 1);
+      mbar_init(bar(bars.u_empty[i]), 9);
+    }
+    mbar_fence_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&tmem_base_s), kTmemCols);
+    tmem_relinquish();
+  }
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_s;
+  const int n_units = p.hdr->n_units;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_q);
+      tma_prefetch_desc(&tm_kw);
+      tma_prefetch_desc(&tm_vw);
+      tma_prefetch_desc(&tm_kc);
+      tma_prefetch_desc(&tm_vc);
+      uint32_t kv_it = 0, u_it = 0, q_loads = 0;
+      bool ok = true;
+      for (;;) {
+        const int uidx = atomicAdd(&p.hdr->counter, 1);
+        const bool done = uidx >= n_units;
+        const int slot = u_it & 1;
+        if (u_it >= 2 && !mbar_wait(bar(bars.u_empty[slot]), ((u_it >> 1) - 1) & 1, abort_flag)) { ok = false; break; }
+        WorkUnit wu;
+        if (done) {
+          wu.seq = -1;
+        } else {
+          wu = p.units[uidx];
+        }
+        unit_ring[slot] = wu;
+        mbar_arrive(bar(bars.u_full[slot]));
+        ++u_it;
+        if (done) break;
+        const int W = wu.window_mode & 0x3FFFFFFF;
+        const int n_qt = (W * p.G - wu.row0) > kTileRows ? 2 : 1;
+        const int cu = p.cu_window[wu.seq];
+        if (q_loads >= 1 && !mbar_wait(bar(bars.q_empty), (q_loads - 1) & 1, abort_flag)) { ok = false; break; }
+        mbar_arrive_expect_tx(bar(bars.q_full), n_qt * S::kQTile);
+        for (int qt = 0; qt < n_qt; ++qt)
+          for (int h = 0; h < S::kHalves; ++h)
+            tma_load_3d(sbase + S::kQ + qt * S::kQTile + h * S::kHalfBytes, &tm_q, bar(bars.q_full), h * 64,
+                        wu.kv_head * p.G, cu + (wu.row0 + qt * kTileRows) / p.G);
+        ++q_loads;
+        const int P = wu.prefix;
+        const int nP = (P + kTileKeys - 1) / kTileKeys;
+        for (int t = wu.tile_begin; t < wu.tile_end; ++t, ++kv_it) {
+          const int st = kv_it & 1;
+          if (kv_it >= 2 && !mbar_wait(bar(bars.kv_empty[st]), ((kv_it >> 1) - 1) & 1, abort_flag)) { ok = false; break; }
+          const uint32_t kdst = sbase + S::kK + st * S::kKVTile;
+          const uint32_t vdst = sbase + S::kV + st * S::kKVTile;
+          mbar_arrive_expect_tx(bar(bars.k_full[st]), S::kKVTile);
+          if (t < nP) {
+            int pages[16], offs[16];  // page_size >= 8: at most 16 loads per tile
+            for (int l = 0; l < p.loads_per_tile; ++l) {
+              const int key0 = t * kTileKeys + l * p.box_rows;
+              int page = p.num_pages;  // out of range: TMA fills zeros
+              if (key0 < P) {
+                page = p.block_table[static_cast<int64_t>(wu.seq) * p.max_pages + key0 / p.page_size];
+                if (page < 0 || page >= p.num_pages) {
+                  atomicOr(&g_error_word, MBE_DEVERR_PAGE);
+                  page = p.num_pages;
+                }
+              }
+              pages[l] = page;
+              offs[l] = key0 % p.page_size;
+              for (int h = 0; h < S::kHalves; ++h)
+                tma_load_4d(kdst + h * S::kHalfBytes + l * p.box_rows * 128, &tm_kc, bar(bars.k_full[st]), h * 64,
+                            offs[l], wu.kv_head, page);
+            }
+            mbar_arrive_expect_tx(bar(bars.v_full[st]), S::kKVTile);
+            for (int l = 0; l < p.loads_per_tile; ++l)
+              for (int h = 0; h < S::kHalves; ++h)
+                tma_load_4d(vdst + h * S::kHalfBytes + l * p.box_rows * 128, &tm_vc, bar(bars.v_full[st]), h * 64,
+                            offs[l], wu.kv_head, pages[l]);
+          } else {
+            const int tok = cu + (t - nP) * kTileKeys;
+            for (int h = 0; h < S::kHalves; ++h)
+              tma_load_3d(kdst + h * S::kHalfBytes, &tm_kw, bar(bars.k_full[st]), h * 64, wu.kv_head, tok);
+            mbar_arrive_expect_tx(bar(bars.v_full[st]), S::kKVTile);
+            for (int h = 0; h < S::kHalves; ++h)
+              tma_load_3d(vdst + h * S::kHalfBytes, &tm_vw, bar(bars.v_full[st]), h * 64, wu.kv_head, tok);
+          }
+        }
+        if (!ok) break;
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        atomicOr(&g_error_word, MBE_DEVERR_TIMEOUT);
+        // let the copies already issued land before the CTA can exit
+        const int zero = 0;
+        for (uint32_t k = (kv_it >= 2 ? kv_it - 2 : 0); k < kv_it; ++k) {
+          mbar_wait(bar(bars.k_full[k & 1]), (k >> 1) & 1, &zero);
+          mbar_wait(bar(bars.v_full[k & 1]), (k >> 1) & 1, &zero);
+        }
+        if (q_loads >= 1) mbar_wait(bar(bars.q_full), (q_loads - 1) & 1, &zero);
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc_qk = idesc_bf16_f32(128, 128, false, false);
+      constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, false, true);
+      uint32_t kv_it = 0, u_it = 0, q_it = 0;
+      uint32_t p_cnt[2] = {0, 0}, o_cnt[2] = {0, 0};
+      bool ok = true;
+      auto issue_qk = [&](int i, int st) {
+        const uint32_t qa = sbase + S::kQ + i * S::kQTile;
+        const uint32_t ka = sbase + S::kK + st * S::kKVTile;
+#pragma unroll
+        for (int h = 0; h < S::kHalves; ++h)
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            umma_ss(tmem + kTmemS + 128 * i, sdesc_sw128(qa + h * S::kHalfBytes + k * 32, 16, 1024),
+                    sdesc_sw128(ka + h * S::kHalfBytes + k * 32, 16, 1024), idesc_qk, (h | k) ? 1u : 0u);
+      };
+      auto issue_pv = [&](int i, int st, bool acc) {
+        const uint32_t va = sbase + S::kV + st * S::kKVTile;
+#pragma unroll
+        for (int kk = 0; kk < kTileKeys / 16; ++kk)
+          umma_ts(tmem + i * D, tmem + kTmemS + 128 * i + kk * 8, sdesc_sw128(va + kk * 16 * 128, S::kHalfBytes, 1024),
+                  idesc_pv, (acc || kk > 0) ? 1u : 0u);
+      };
+      for (;;) {
+        const int slot = u_it & 1;
+        if (!mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag)) { ok = false; break; }
+        const WorkUnit wu = unit_ring[slot];
+        mbar_arrive(bar(bars.u_empty[slot]));
+        ++u_it;
+        if (wu.seq < 0) break;
+        const int W = wu.window_mode & 0x3FFFFFFF;
+        const int n_qt = (W * p.G - wu.row0) > kTileRows ? 2 : 1;
+        const int n_t = wu.tile_end - wu.tile_begin;
+        if (!mbar_wait(bar(bars.q_full), q_it & 1, abort_flag)) { ok = false; break; }
+        ++q_it;
+        if (!mbar_wait(bar(bars.k_full[kv_it & 1]), (kv_it >> 1) & 1, abort_flag)) { ok = false; break; }
+        tc_fence_after();
+        for (int i = 0; i < n_qt; ++i) {
+          issue_qk(i, kv_it & 1);
+          umma_commit(bar(bars.s_full[i]));
+        }
+        if (n_t == 1) umma_commit(bar(bars.q_empty));
+        for (int j = 0; j < n_t && ok; ++j) {
+          const uint32_t ki = kv_it + j;
+          const int st = ki & 1;
+          if (!mbar_wait(bar(bars.v_full[st]), (ki >> 1) & 1, abort_flag)) { ok = false; break; }
+          for (int i = 0; i < n_qt; ++i) {
+            if (!mbar_wait(bar(bars.p_full[i]), p_cnt[i] & 1, abort_flag)) { ok = false; break; }
+            ++p_cnt[i];
+            if (j == 0 && o_cnt[i] > 0 && !mbar_wait(bar(bars.o_empty[i]), (o_cnt[i] - 1) & 1, abort_flag)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            issue_pv(i, st, j > 0);
+            if (j == n_t - 1) umma_commit(bar(bars.o_full[i]));
+            if (i == n_qt - 1) umma_commit(bar(bars.kv_empty[st]));
+            if (j + 1 < n_t) {
+              const uint32_t kn = ki + 1;
+              if (i == 0) {
+                if (!mbar_wait(bar(bars.k_full[kn & 1]), (kn >> 1) & 1, abort_flag)) { ok = false; break; }
+                tc_fence_after();
+              }
+              issue_qk(i, kn & 1);
+              umma_commit(bar(bars.s_full[i]));
+              if (j + 2 == n_t && i == n_qt - 1) umma_commit(bar(bars.q_empty));
+            }
+          }
+        }
+        if (!ok) break;
+        kv_it += n_t;
+        for (int i = 0; i < n_qt; ++i) ++o_cnt[i];
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        atomicOr(&g_error_word, MBE_DEVERR_TIMEOUT);
+      }
+      // every MMA this thread issued must finish before TMEM is released
+      const int zero = 0;
+      umma_commit(bar(bars.mma_done));
+      mbar_wait(bar(bars.mma_done), 0, &zero);
+    }
+  } else if (warp >= 4) {
+    // ---------------------------------------------------------------- softmax + epilogue
+    const int wg = (warp - 4) >> 2;           // query tile 0 or 1
+    const int quad = warp & 3;                // TMEM lane quadrant of this warp
+    const int r = quad * 32 + lane;           // row within the tile
+    const uint32_t t_lane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+    const uint32_t tS = t_lane + kTmemS + 128 * wg;
+    const uint32_t tO = t_lane + wg * D;
+    uint32_t u_it = 0, s_cnt = 0, o_cnt = 0, kv_it = 0;
+    bool ok = true;
+    for (;;) {
+      const int slot = u_it & 1;
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag));
+      if (!ok) break;
+      const WorkUnit wu = unit_ring[slot];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar(bars.u_empty[slot]));
+      ++u_it;
+      if (wu.seq < 0) break;
+      const int W = wu.window_mode & 0x3FFFFFFF;
+      const int mode = wu.window_mode >> 30;
+      const int n_qt = (W * p.G - wu.row0) > kTileRows ? 2 : 1;
+      const int n_t = wu.tile_end - wu.tile_begin;
+      const int P = wu.prefix;
+      const int nP = (P + kTileKeys - 1) / kTileKeys;
+      if (wg >= n_qt) {
+        kv_it += n_t;
+        continue;
+      }
+      const int R = wu.row0 + kTileRows * wg + r;
+      const int qi = R / p.G, hh = R - qi * p.G;
+      const bool valid = qi < W;
+      const int lim = (mode == MBE_MULTI_BLOCK_BIDIRECTIONAL) ? W : min(W, (qi / p.block_size + 1) * p.block_size);
+      float m = neg_inf(), l = 0.f;
+      for (int j = 0; j < n_t; ++j) {
+        const int t = wu.tile_begin + j;
+        const uint32_t ki = kv_it + j;
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.s_full[wg]), s_cnt & 1, abort_flag));
+        if (!ok) break;
+        ++s_cnt;
+        tc_fence_after();
+        const int n_vis = t < nP ? min(kTileKeys, P - t * kTileKeys) : max(0, min(kTileKeys, lim - (t - nP) * kTileKeys));
+        uint32_t sr[128];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) tmem_ld32(tS + 32 * c, *reinterpret_cast<uint32_t(*)[32]>(&sr[32 * c]));
+        float mx = neg_inf();
+#pragma unroll
+        for (int c = 0; c < 128; ++c)
+          if (c < n_vis) mx = fmaxf(mx, __uint_as_float(sr[c]));
+        const float m_new = fmaxf(m, mx * p.scale_log2);
+        const bool need = m_new > m + kRescaleLog2;
+        if (__any_sync(0xffffffffu, need)) {
+          const float alpha = (m_new == neg_inf()) ? 1.f : ex2f(m - m_new);
+          l *= alpha;
+          if (j > 0) {
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+              uint32_t o[32];
+              tmem_ld32(tO + 32 * c, o);
+#pragma unroll
+              for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * alpha);
+              tmem_st32(tO + 32 * c, o);
+            }
+          }
+          m = m_new;
+        }
+        const float mu = (m == neg_inf()) ? 0.f : m;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          uint32_t pk[32];
+#pragma unroll
+          for (int k = 0; k < 32; ++k) {
+            const int c = 64 * h + 2 * k;
+            const float p0 = c < n_vis ? ex2f(fmaf(__uint_as_float(sr[c]), p.scale_log2, -mu)) : 0.f;
+            const float p1 = c + 1 < n_vis ? ex2f(fmaf(__uint_as_float(sr[c + 1]), p.scale_log2, -mu)) : 0.f;
+            l += p0 + p1;
+            pk[k] = pack_bf16x2(p0, p1);
+          }
+          tmem_st32(tS + 32 * h, pk);
+        }
+        tmem_st_wait();
+        if (wg == 0 && t == nP - 1 && (P % kTileKeys) != 0) {
+          // stale cache rows past the prefix end: zero them in V so that 0 * V stays 0
+          ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.v_full[ki & 1]), (ki >> 1) & 1, abort_flag));
+          if (!ok) break;
+          const int v0 = P % kTileKeys;
+          uint8_t* vt = smem + S::kV + (ki & 1) * S::kKVTile;
+          const int per_row = S::kHalves * 8;  // 16-byte chunks per key row
+          for (int idx = r; idx < (kTileKeys - v0) * per_row; idx += kTileRows) {
+            const int row = v0 + idx / per_row, rem = idx % per_row;
+            *reinterpret_cast<uint4*>(vt + (rem / 8) * S::kHalfBytes + row * 128 + (rem % 8) * 16) =
+                make_uint4(0u, 0u, 0u, 0u);
+          }
+          fence_proxy_async_smem();
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(bars.p_full[wg]));
+      }
+      if (!ok) break;
+      kv_it += n_t;
+      // epilogue: O_i is complete once o_full fires
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.o_full[wg]), o_cnt & 1, abort_flag));
+      if (!ok) break;
+      ++o_cnt;
+      tc_fence_after();
+      const float inv_l = l > 0.f ? 1.f / l : 0.f;
+      const float lse2 = l > 0.f ? m + __log2f(l) : neg_inf();
+      if (wu.slot < 0) {
+        const int cu = p.cu_window[wu.seq];
+        __nv_bfloat16* orow =
+            p.out + (static_cast<int64_t>(cu + qi) * p.Hq + wu.kv_head * p.G + hh) * D;
+#pragma unroll
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t o[32];
+          tmem_ld32(tO + 32 * c, o);
+          if (valid) {
+            uint4* dst = reinterpret_cast<uint4*>(orow + 32 * c);
+#pragma unroll
+            for (int v = 0; v < 4; ++v) {
+              uint4 w;
+              w.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv_l, __uint_as_float(o[8 * v + 1]) * inv_l);
+              w.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv_l, __uint_as_float(o[8 * v + 3]) * inv_l);
+              w.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv_l, __uint_as_float(o[8 * v + 5]) * inv_l);
+              w.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv_l, __uint_as_float(o[8 * v + 7]) * inv_l);
+              dst[v] = w;
+            }
+          }
+        }
+        if (valid && p.lse) p.lse[static_cast<int64_t>(cu + qi) * p.Hq + wu.kv_head * p.G + hh] = lse2 * 0.6931471805599453f;
+      } else {
+        const int prow = kTileRows * wg + r;
+        float* po = p.part_o + (static_cast<int64_t>(wu.slot) * kUnitRows + prow) * D;
+#pragma unroll
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t o[32];
+          tmem_ld32(tO + 32 * c, o);
+          if (valid) {
+            float4* dst = reinterpret_cast<float4*>(po + 32 * c);
+#pragma unroll
+            for (int v = 0; v < 8; ++v)
+              dst[v] = make_float4(__uint_as_float(o[4 * v]) * inv_l, __uint_as_float(o[4 * v + 1]) * inv_l,
+                                   __uint_as_float(o[4 * v + 2]) * inv_l, __uint_as_float(o[4 * v + 3]) * inv_l);
+          }
+        }
+        if (valid) p.part_lse[static_cast<int64_t>(wu.slot) * kUnitRows + prow] = lse2;
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar(bars.o_empty[wg]));
+    }
+    if (!ok && lane == 0) {
+      *abort_flag = 1;
+      atomicOr(&g_error_word, MBE_DEVERR_TIMEOUT);
+    }
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------ split merge
+struct MergeParams {
+  const Header* hdr;
+  const MergeGroup* groups;
+  const float* part_o;
+  const float* part_lse;
+  const int32_t* cu_window;
+  __nv_bfloat16* out;
+  float* lse;
+  int Hq, G, D;
+};
+
+__global__ void __launch_bounds__(kUnitRows) attn_merge_kernel(const MergeParams p) {
+  const int gi = blockIdx.x;
+  if (gi >= p.hdr->n_groups) return;
+  const MergeGroup grp = p.groups[gi];
+  const int r = threadIdx.x;
+  const int R = grp.row0 + r;
+  const int qi = R / p.G, hh = R - qi * p.G;
+  if (qi >= grp.window) return;
+  float M = neg_inf();
+  for (int k = 0; k < grp.n_splits; ++k)
+    M = fmaxf(M, p.part_lse[static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r]);
+  float wsum = 0.f;
+  float acc[128];
+  for (int d = 0; d < p.D; ++d) acc[d] = 0.f;
+  for (int k = 0; k < grp.n_splits; ++k) {
+    const float lk = p.part_lse[static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r];
+    const float w = (lk == neg_inf()) ? 0.f : ex2f(lk - M);
+    if (w == 0.f) continue;
+    wsum += w;
+    const float4* src = reinterpret_cast<const float4*>(p.part_o + (static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r) * p.D);
+    for (int d4 = 0; d4 < p.D / 4; ++d4) {
+      const float4 v = src[d4];
+      acc[4 * d4] += w * v.x;
+      acc[4 * d4 + 1] += w * v.y;
+      acc[4 * d4 + 2] += w * v.z;
+      acc[4 * d4 + 3] += w * v.w;
+    }
+  }
+  const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
+  const int cu = p.cu_window[grp.seq];
+  const int64_t orow = static_cast<int64_t>(cu + qi) * p.Hq + grp.kv_head * p.G + hh;
+  uint32_t* dst = reinterpret_cast<uint32_t*>(p.out + orow * p.D);
+  for (int d = 0; d < p.D; d += 2) dst[d / 2] = pack_bf16x2(acc[d] * inv, acc[d + 1] * inv);
+  if (p.lse) p.lse[orow] = (wsum > 0.f ? M + __log2f(wsum) : neg_inf()) * 0.6931471805599453f;
+}
+
+// ------------------------------------------------------------------ host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  });
+  return fn;
+}
+
+bool encode(CUtensorMap* tm, const void* base, int rank, const cuuint64_t* dims, const cuuint64_t* strides,
+            const cuuint32_t* box) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+struct DeviceInfo {
+  int num_sms = 0;
+  bool attr_set[2] = {false, false};
+};
+
+DeviceInfo* device_info(int dev) {
+  static DeviceInfo info[64];
+  static std::mutex mu;
+  if (dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lock(mu);
+  DeviceInfo& d = info[dev];
+  if (d.num_sms == 0) {
+    if (cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) d.num_sms = 0;
+  }
+  return &d;
+}
+
+template <int D>
+bool ensure_smem_attr(DeviceInfo* di) {
+  const int idx = D == 128 ? 1 : 0;
+  if (!di->attr_set[idx]) {
+    if (cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<D>::kBytes) !=
+        cudaSuccess)
+      return false;
+    di->attr_set[idx] = true;
+  }
+  return true;
+}
+
+inline bool pow2(int x) { return x > 0 && (x & (x - 1)) == 0; }
+
+mbe_status check_shapes(int32_t batch, int32_t Hq, int32_t Hkv, int32_t D, int32_t max_window, int32_t max_prefix) {
+  if (batch < 0 || Hq < 1 || Hkv < 1 || max_window < 0 || max_prefix < 0) return MBE_ERR_INVALID_ARG;
+  if (Hq % Hkv != 0) return MBE_ERR_INVALID_ARG;
+  if (D != 64 && D != 128) return MBE_ERR_UNSUPPORTED;
+  const int G = Hq / Hkv;
+  if (!pow2(G) || G > kTileRows) return MBE_ERR_UNSUPPORTED;
+  if (max_window > (1 << 20) || max_prefix > (1 << 28)) return MBE_ERR_UNSUPPORTED;
+  return MBE_OK;
+}
+
+template <int D>
+mbe_status run(const void* q, const void* k_win, const void* v_win, const void* k_cache, const void* v_cache,
+               int32_t num_pages, const int32_t* block_table, int32_t max_pages, const int32_t* prefix_len,
+               const int32_t* window_len, const int32_t* cu_window, const uint8_t* mask_mode, int32_t batch,
+               int32_t total_q_tokens, int32_t Hq, int32_t Hkv, int32_t block_size, int32_t page_size,
+               int32_t max_window, int32_t max_prefix, float scale, void* out, float* lse, void* workspace,
+               const Layout& L, DeviceInfo* di, cudaStream_t stream) {
+  const int G = Hq / Hkv;
+  CUtensorMap tq, tkw, tvw, tkc, tvc;
+  {
+    const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)Hq, (cuuint64_t)total_q_tokens};
+    const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)Hq * D * 2};
+    const cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)(kTileRows / G)};
+    if (!encode(&tq, q, 3, dims, strides, box)) return MBE_ERR_CUDA;
+  }
+  {
+    const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)Hkv, (cuuint64_t)total_q_tokens};
+    const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)Hkv * D * 2};
+    const cuuint32_t box[3] = {64, 1, (cuuint32_t)kTileKeys};
+    if (!encode(&tkw, k_win, 3, dims, strides, box) || !encode(&tvw, v_win, 3, dims, strides, box))
+      return MBE_ERR_CUDA;
+  }
+  const int box_rows = std::min(page_size, kTileKeys);
+  {
+    const cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)page_size, (cuuint64_t)Hkv, (cuuint64_t)num_pages};
+    const cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)page_size * D * 2,
+                                   (cuuint64_t)Hkv * page_size * D * 2};
+    const cuuint32_t box[4] = {64, (cuuint32_t)box_rows, 1, 1};
+    if (!encode(&tkc, k_cache, 4, dims, strides, box) || !encode(&tvc, v_cache, 4, dims, strides, box))
+      return MBE_ERR_CUDA;
+  }
+  if (!ensure_smem_attr<D>(di)) return MBE_ERR_CUDA;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  Header* hdr = reinterpret_cast<Header*>(ws);
+  SchedParams sp{prefix_len, window_len, mask_mode, cu_window, batch, G, Hkv, block_size, max_window, max_prefix,
+                 di->num_sms, total_q_tokens, hdr, reinterpret_cast<WorkUnit*>(ws + L.units_tmp), reinterpret_cast<WorkUnit*>(ws + L.units),
+                 reinterpret_cast<MergeGroup*>(ws + L.groups), L.max_units, L.max_groups, L.max_slots};
+  attn_schedule_kernel<<<1, kBuckets, 0, stream>>>(sp);
+  if (cudaGetLastError() != cudaSuccess) return MBE_ERR_CUDA;
+  AttnParams ap;
+  ap.block_table = block_table;
+  ap.cu_window = cu_window;
+  ap.out = static_cast<__nv_bfloat16*>(out);
+  ap.lse = lse;
+  ap.hdr = hdr;
+  ap.units = reinterpret_cast<const WorkUnit*>(ws + L.units);
+  ap.part_o = reinterpret_cast<float*>(ws + L.part_o);
+  ap.part_lse = reinterpret_cast<float*>(ws + L.part_lse);
+  ap.max_pages = max_pages;
+  ap.num_pages = num_pages;
+  ap.Hq = Hq;
+  ap.G = G;
+  ap.block_size = block_size;
+  ap.page_size = page_size;
+  ap.box_rows = box_rows;
+  ap.loads_per_tile = kTileKeys / box_rows;
+  ap.scale_log2 = scale * 1.4426950408889634f;
+  attn_kernel<D><<<di->num_sms, kThreads, Smem<D>::kBytes, stream>>>(tq, tkw, tvw, tkc, tvc, ap);
+  if (cudaGetLastError() != cudaSuccess) return MBE_ERR_CUDA;
+  MergeParams mp{hdr, reinterpret_cast<const MergeGroup*>(ws + L.groups), ap.part_o, ap.part_lse, cu_window,
+                 ap.out, lse, Hq, G, D};
+  attn_merge_kernel<<<static_cast<unsigned>(L.max_groups), kUnitRows, 0, stream>>>(mp);
+  if (cudaGetLastError() != cudaSuccess) return MBE_ERR_CUDA;
+  return MBE_OK;
+}
+
+}  // namespace attn
+}  // namespace mbe
+
+using namespace mbe;
+using namespace mbe::attn;
+
+extern "C" size_t mbe_window_attention_workspace_size(int32_t batch, int32_t num_q_heads, int32_t num_kv_heads,
+                                                      int32_t head_dim, int32_t max_window, int32_t max_prefix) {
+  if (check_shapes(batch, num_q_heads, num_kv_heads, head_dim, max_window, max_prefix) != MBE_OK) return 0;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  DeviceInfo* di = device_info(dev);
+  if (!di || di->num_sms <= 0) return 0;
+  return make_layout(batch, num_q_heads, num_kv_heads, head_dim, max_window, max_prefix, di->num_sms).total;
+}
+
+extern "C" mbe_status mbe_window_attention(const void* q, const void* k_win, const void* v_win, const void* k_cache,
+                                           const void* v_cache, int32_t num_pages, const int32_t* block_table,
+                                           int32_t max_pages_per_seq, const int32_t* prefix_len,
+                                           const int32_t* window_len, const int32_t* cu_window,
+                                           const uint8_t* mask_mode, int32_t batch, int32_t total_q_tokens,
+                                           int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim,
+                                           int32_t block_size, int32_t page_size, int32_t max_window,
+                                           int32_t max_prefix, float softmax_scale, void* out, float* lse_or_null,
+                                           void* workspace, size_t workspace_bytes, cudaStream_t stream) {
+  mbe_status st = check_shapes(batch, num_q_heads, num_kv_heads, head_dim, max_window, max_prefix);
+  if (st != MBE_OK) return st;
+  if (block_size < 1 || total_q_tokens < 0 || num_pages < 1 || max_pages_per_seq < 1) return MBE_ERR_INVALID_ARG;
+  if (!pow2(page_size) || page_size < 8) return MBE_ERR_UNSUPPORTED;
+  if (static_cast<int64_t>(max_pages_per_seq) * page_size < max_prefix) return MBE_ERR_INVALID_ARG;
+  if (!(softmax_scale >= 0.f) || std::isinf(softmax_scale)) return MBE_ERR_INVALID_ARG;
+  if (batch == 0 || total_q_tokens == 0 || max_window == 0) return MBE_OK;
+  if (!q || !k_win || !v_win || !k_cache || !v_cache || !block_table || !prefix_len || !window_len || !cu_window ||
+      !mask_mode || !out)
+    return MBE_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k_win) || !aligned16(v_win) || !aligned16(k_cache) || !aligned16(v_cache) ||
+      !aligned16(out))
+    return MBE_ERR_INVALID_ARG;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return MBE_ERR_CUDA;
+  DeviceInfo* di = device_info(dev);
+  if (!di || di->num_sms <= 0) return MBE_ERR_CUDA;
+  const Layout L = make_layout(batch, num_q_heads, num_kv_heads, head_dim, max_window, max_prefix, di->num_sms);
+  if (!workspace || workspace_bytes < L.total || !aligned16(workspace)) return MBE_ERR_WORKSPACE;
+  if (L.max_groups > 0x7FFFFFFF) return MBE_ERR_UNSUPPORTED;
+  const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(head_dim));
+  if (head_dim == 128)
+    return run<128>(q, k_win, v_win, k_cache, v_cache, num_pages, block_table, max_pages_per_seq, prefix_len,
+                    window_len, cu_window, mask_mode, batch, total_q_tokens, num_q_heads, num_kv_heads, block_size,
+                    page_size, max_window, max_prefix, scale, out, lse_or_null, workspace, L, di, stream);
+  return run<64>(q, k_win, v_win, k_cache, v_cache, num_pages, block_table, max_pages_per_seq, prefix_len, window_len,
+                 cu_window, mask_mode, batch, total_q_tokens, num_q_heads, num_kv_heads, block_size, page_size,
+                 max_window, max_prefix, scale, out, lse_or_null, workspace, L, di, stream);
+}

@@ -1,0 +1,31 @@
+// Internal helpers shared by the translation units of libmbe.
+#pragma once
+#include <cstdint>
+#include <cuda_runtime.h>
+#include "mbe.h"
+
+namespace mbe {
+
+// Each translation unit owns one device error word (no relocatable device
+// code is needed); mbe_get_device_error() reads and clears all of them.
+#define MBE_DEFINE_ERROR_WORD(accessor)                                                     \
+  static __device__ unsigned int g_error_word;                                              \
+  uint32_t accessor() {                                                                     \
+    unsigned int v = 0, z = 0;                                                              \
+    if (cudaMemcpyFromSymbol(&v, g_error_word, sizeof(v)) != cudaSuccess) return 0xFFFFFFFFu; \
+    cudaMemcpyToSymbol(g_error_word, &z, sizeof(z));                                        \
+    return v;                                                                               \
+  }
+
+uint32_t edit_decide_take_error();
+uint32_t kv_write_take_error();
+uint32_t attention_take_error();
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+inline mbe_status launch_status() {
+  cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? MBE_OK : MBE_ERR_CUDA;
+}
+
+}  // namespace mbe

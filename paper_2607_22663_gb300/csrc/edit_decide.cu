@@ -1,0 +1,217 @@
+// Edit-decide: the T2T update of Eq. 2 fused into one pass over the logits.
+//
+// One CTA owns one row. Each thread streams 16-byte vectors of the row and keeps
+// an online (max, sum of exp(l - max), argmax) triple; triples are merged with
+// warp shuffles and then across warps through shared memory. Thread 0 turns the
+// row's triple into the confidence c = 1 / sum_v exp(l_v - l_max) and applies
+// the threshold-and-replace rule. The logits are read exactly once, so the
+// kernel is bound by HBM bandwidth.
+#include <cuda_bf16.h>
+#include "common.cuh"
+
+namespace mbe {
+
+MBE_DEFINE_ERROR_WORD(edit_decide_take_error)
+
+namespace {
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+struct Triple {
+  float m;  // running maximum
+  float s;  // sum of exp(l - m)
+  int idx;  // lowest index attaining m
+};
+
+// Adds one element (or a vector's maximum first) to the triple.
+__device__ __forceinline__ void absorb_max(Triple& t, float lm, int li) {
+  if (lm > t.m) {
+    t.s *= ex2((t.m - lm) * kLog2e);  // m = -inf gives ex2(-inf) = 0
+    t.m = lm;
+    t.idx = li;
+  }
+}
+
+__device__ __forceinline__ void merge(Triple& a, const Triple& b) {
+  if (b.idx < 0) return;  // b saw no element
+  if (a.idx < 0) {
+    a = b;
+    return;
+  }
+  if (b.m > a.m) {
+    a.s = a.s * ex2((a.m - b.m) * kLog2e) + b.s;
+    a.m = b.m;
+    a.idx = b.idx;
+  } else if (b.m < a.m) {
+    a.s += b.s * ex2((b.m - a.m) * kLog2e);
+  } else {
+    a.s += b.s;
+    a.idx = min(a.idx, b.idx);
+  }
+}
+
+__device__ __forceinline__ Triple shfl_xor(const Triple& t, int mask) {
+  Triple o;
+  o.m = __shfl_xor_sync(0xffffffffu, t.m, mask);
+  o.s = __shfl_xor_sync(0xffffffffu, t.s, mask);
+  o.idx = __shfl_xor_sync(0xffffffffu, t.idx, mask);
+  return o;
+}
+
+template <typename T>
+__device__ __forceinline__ float to_f32(T x);
+template <>
+__device__ __forceinline__ float to_f32<float>(float x) { return x; }
+template <>
+__device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 x) { return __bfloat162float(x); }
+
+// Unpacks one 16-byte vector into floats.
+template <typename T>
+struct Vec;
+template <>
+struct Vec<float> {
+  static constexpr int N = 4;
+  __device__ __forceinline__ static void unpack(const uint4& v, float (&x)[4]) {
+    x[0] = __uint_as_float(v.x); x[1] = __uint_as_float(v.y);
+    x[2] = __uint_as_float(v.z); x[3] = __uint_as_float(v.w);
+  }
+};
+template <>
+struct Vec<__nv_bfloat16> {
+  static constexpr int N = 8;
+  __device__ __forceinline__ static void unpack(const uint4& v, float (&x)[8]) {
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      x[2 * k] = __uint_as_float(w[k] << 16);
+      x[2 * k + 1] = __uint_as_float(w[k] & 0xFFFF0000u);
+    }
+  }
+};
+
+template <typename T>
+__device__ __forceinline__ void absorb_vector(Triple& t, const uint4& v, int col0) {
+  constexpr int N = Vec<T>::N;
+  float x[N];
+  Vec<T>::unpack(v, x);
+  float lm = x[0];
+  int li = 0;
+#pragma unroll
+  for (int k = 1; k < N; ++k)
+    if (x[k] > lm) { lm = x[k]; li = k; }
+  absorb_max(t, lm, col0 + li);
+  float acc = 0.f;
+#pragma unroll
+  for (int k = 0; k < N; ++k) acc += ex2((x[k] - t.m) * kLog2e);
+  t.s += acc;
+}
+
+template <typename T, int kThreads>
+__global__ void __launch_bounds__(kThreads) edit_decide_kernel(const T* __restrict__ logits, int64_t row_stride,
+                                                               int vocab, bool vec_ok,
+                                                               const int32_t* __restrict__ committed,
+                                                               const float* __restrict__ tau_per_row, float tau,
+                                                               const uint8_t* __restrict__ editable,
+                                                               int32_t* new_tokens, uint8_t* __restrict__ edit_mask,
+                                                               float* __restrict__ confidence,
+                                                               int32_t* __restrict__ argmax_out) {
+  constexpr int N = Vec<T>::N;
+  constexpr int kUnroll = 4;
+  const int row = blockIdx.x;
+  const T* rp = logits + static_cast<int64_t>(row) * row_stride;
+  Triple t{__int_as_float(0xff800000u), 0.f, -1};  // empty: m = -inf
+  int scalar_from = 0;
+  if (vec_ok) {
+    const uint4* vp = reinterpret_cast<const uint4*>(rp);
+    const int nvec = vocab / N;
+    int v = threadIdx.x;
+    for (; v + (kUnroll - 1) * kThreads < nvec; v += kUnroll * kThreads) {
+      uint4 buf[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) buf[u] = __ldcs(vp + v + u * kThreads);
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) absorb_vector<T>(t, buf[u], (v + u * kThreads) * N);
+    }
+    for (; v < nvec; v += kThreads) absorb_vector<T>(t, __ldcs(vp + v), v * N);
+    scalar_from = nvec * N;
+  }
+  for (int c = scalar_from + threadIdx.x; c < vocab; c += kThreads) {
+    const float x = to_f32<T>(rp[c]);
+    absorb_max(t, x, c);
+    t.s += ex2((x - t.m) * kLog2e);
+  }
+  // warp merge
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    Triple o = shfl_xor(t, off);
+    merge(t, o);
+  }
+  __shared__ Triple warp_part[kThreads / 32];
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  if (lane == 0) warp_part[warp] = t;
+  __syncthreads();
+  if (warp == 0) {
+    Triple a = lane < kThreads / 32 ? warp_part[lane] : Triple{__int_as_float(0xff800000u), 0.f, -1};
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      Triple o = shfl_xor(a, off);
+      merge(a, o);
+    }
+    if (lane == 0) {
+      const float c = 1.0f / a.s;
+      const int32_t x = committed[row];
+      const float tr = tau_per_row ? tau_per_row[row] : tau;
+      const bool can = editable ? (editable[row] != 0) : true;
+      const bool ed = can && (a.idx != x) && (c > tr);
+      new_tokens[row] = ed ? a.idx : x;
+      edit_mask[row] = ed ? 1 : 0;
+      confidence[row] = c;
+      if (argmax_out) argmax_out[row] = a.idx;
+    }
+  }
+}
+
+template <typename T>
+mbe_status launch(const void* logits, int64_t row_stride, int32_t rows, int32_t vocab, const int32_t* committed,
+                  const float* tpr, float tau, const uint8_t* editable, int32_t* new_tokens, uint8_t* edit_mask,
+                  float* confidence, int32_t* argmax_out, cudaStream_t stream) {
+  const T* lp = static_cast<const T*>(logits);
+  const bool vec_ok = aligned16(logits) && ((row_stride * static_cast<int64_t>(sizeof(T))) % 16 == 0);
+  const int64_t row_bytes = static_cast<int64_t>(vocab) * sizeof(T);
+  if (row_bytes >= 64 * 1024) {
+    edit_decide_kernel<T, 512><<<rows, 512, 0, stream>>>(lp, row_stride, vocab, vec_ok, committed, tpr, tau, editable,
+                                                         new_tokens, edit_mask, confidence, argmax_out);
+  } else if (row_bytes >= 8 * 1024) {
+    edit_decide_kernel<T, 256><<<rows, 256, 0, stream>>>(lp, row_stride, vocab, vec_ok, committed, tpr, tau, editable,
+                                                         new_tokens, edit_mask, confidence, argmax_out);
+  } else {
+    edit_decide_kernel<T, 64><<<rows, 64, 0, stream>>>(lp, row_stride, vocab, vec_ok, committed, tpr, tau, editable,
+                                                       new_tokens, edit_mask, confidence, argmax_out);
+  }
+  return launch_status();
+}
+
+}  // namespace
+}  // namespace mbe
+
+extern "C" mbe_status mbe_edit_decide(const void* logits, mbe_dtype dtype, int64_t row_stride, int32_t rows,
+                                      int32_t vocab, const int32_t* committed, const float* tau_per_row_or_null,
+                                      float tau, const uint8_t* editable_or_null, int32_t* new_tokens,
+                                      uint8_t* edit_mask, float* confidence, int32_t* argmax_or_null,
+                                      cudaStream_t stream) {
+  if (rows < 0 || vocab < 1 || row_stride < vocab) return MBE_ERR_INVALID_ARG;
+  if (dtype != MBE_F32 && dtype != MBE_BF16) return MBE_ERR_INVALID_ARG;
+  if (rows == 0) return MBE_OK;
+  if (!logits || !committed || !new_tokens || !edit_mask || !confidence) return MBE_ERR_INVALID_ARG;
+  if (dtype == MBE_F32)
+    return mbe::launch<float>(logits, row_stride, rows, vocab, committed, tau_per_row_or_null, tau, editable_or_null,
+                              new_tokens, edit_mask, confidence, argmax_or_null, stream);
+  return mbe::launch<__nv_bfloat16>(logits, row_stride, rows, vocab, committed, tau_per_row_or_null, tau,
+                                    editable_or_null, new_tokens, edit_mask, confidence, argmax_or_null, stream);
+}

@@ -1,0 +1,197 @@
+"""Python binding of libmbe (argument marshalling only).
+
+Each function takes torch tensors, checks their dtype/device/layout, and calls
+the C entry point of the same name in ``libmbe.so`` on the current CUDA stream.
+All arithmetic runs in the library's CUDA kernels; there is no fallback: if the
+library is missing or the call fails, an exception is raised.
+"""
+from __future__ import annotations
+
+import ctypes
+import re
+from pathlib import Path
+from typing import Optional
+
+import torch
+
+from . import build as _build
+
+MBE_OK = 0
+STATUS_NAMES = {0: "MBE_OK", 1: "MBE_ERR_INVALID_ARG", 2: "MBE_ERR_UNSUPPORTED", 3: "MBE_ERR_CUDA",
+                4: "MBE_ERR_TIMEOUT", 5: "MBE_ERR_WORKSPACE", 6: "MBE_ERR_DEVICE_CHECK"}
+DEVERR_TIMEOUT, DEVERR_LENGTH, DEVERR_PAGE, DEVERR_CAPACITY = 0x1, 0x2, 0x4, 0x8
+BLOCK_CAUSAL, MULTI_BLOCK_BIDIRECTIONAL = 0, 1
+HEADER = _build.INCLUDE / "mbe.h"
+
+_lib = None
+
+
+class MbeError(RuntimeError):
+    def __init__(self, fn, status):
+        self.status = status
+        super().__init__(f"{fn} failed: {STATUS_NAMES.get(status, status)} ({_status_string(status)})")
+
+
+def _status_string(status):
+    try:
+        return lib().mbe_status_string(status).decode()
+    except Exception:
+        return "?"
+
+
+def lib(build_if_missing: bool = True):
+    """The loaded libmbe (ctypes.CDLL), building it in-tree if needed."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.LIB
+    if build_if_missing:
+        path = _build.build()
+    if not Path(path).exists():
+        raise RuntimeError(f"libmbe.so not found at {path}; run paper_2607_22663_gb300.build.build()")
+    L = ctypes.CDLL(str(path))
+    P, i32, i64, f32, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
+    L.mbe_window_attention.restype = ctypes.c_int
+    L.mbe_window_attention.argtypes = [P, P, P, P, P, i32, P, i32, P, P, P, P, i32, i32, i32, i32, i32, i32, i32, i32,
+                                       i32, f32, P, P, P, sz, P]
+    L.mbe_window_attention_workspace_size.restype = sz
+    L.mbe_window_attention_workspace_size.argtypes = [i32, i32, i32, i32, i32, i32]
+    L.mbe_edit_decide.restype = ctypes.c_int
+    L.mbe_edit_decide.argtypes = [P, ctypes.c_int, i64, i32, i32, P, P, f32, P, P, P, P, P, P]
+    L.mbe_kv_window_write.restype = ctypes.c_int
+    L.mbe_kv_window_write.argtypes = [P, P, P, P, i32, P, i32, P, P, P, P, i32, i32, i32, i32, i32, i32, i32, P]
+    L.mbe_get_device_error.restype = ctypes.c_int
+    L.mbe_get_device_error.argtypes = [P, ctypes.POINTER(ctypes.c_uint32)]
+    L.mbe_status_string.restype = ctypes.c_char_p
+    L.mbe_status_string.argtypes = [ctypes.c_int]
+    L.mbe_version.restype = i32
+    L.mbe_version.argtypes = []
+    _lib = L
+    return L
+
+
+def declared_symbols():
+    """Function names declared in include/mbe.h."""
+    text = HEADER.read_text()
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\s*\*?\s*(mbe_\w+)\s*\(", text, flags=re.M)))
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _need(t, name, dtype=None, cuda=True):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if cuda and not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
+def _check(fn, st):
+    if st != MBE_OK:
+        raise MbeError(fn, st)
+
+
+def window_attention_workspace_size(batch, num_q_heads, num_kv_heads, head_dim, max_window, max_prefix):
+    return int(lib().mbe_window_attention_workspace_size(batch, num_q_heads, num_kv_heads, head_dim, max_window,
+                                                         max_prefix))
+
+
+def window_attention(q, k_win, v_win, k_cache, v_cache, block_table, prefix_len, window_len, cu_window, mask_mode, *,
+                     block_size, max_window, max_prefix, softmax_scale=0.0, out=None, lse=None, return_lse=False,
+                     workspace=None, stream=None):
+    """mbe_window_attention: see include/mbe.h. Returns out (and lse if requested)."""
+    for t, n in ((q, "q"), (k_win, "k_win"), (v_win, "v_win"), (k_cache, "k_cache"), (v_cache, "v_cache")):
+        _need(t, n, torch.bfloat16)
+    for t, n in ((block_table, "block_table"), (prefix_len, "prefix_len"), (window_len, "window_len"),
+                 (cu_window, "cu_window")):
+        _need(t, n, torch.int32)
+    _need(mask_mode, "mask_mode", torch.uint8)
+    T, Hq, D = q.shape
+    num_pages, Hkv, page_size, D2 = k_cache.shape
+    if D2 != D or tuple(k_win.shape) != (T, Hkv, D) or tuple(v_win.shape) != (T, Hkv, D) or v_cache.shape != k_cache.shape:
+        raise ValueError("inconsistent q/k/v shapes")
+    batch, max_pages = block_table.shape
+    if out is None:
+        out = torch.empty_like(q)
+    _need(out, "out", torch.bfloat16)
+    if return_lse and lse is None:
+        lse = torch.empty((T, Hq), dtype=torch.float32, device=q.device)
+    if lse is not None:
+        _need(lse, "lse", torch.float32)
+    need = window_attention_workspace_size(batch, Hq, Hkv, D, max_window, max_prefix)
+    if workspace is None or workspace.numel() < need:
+        workspace = torch.empty(max(need, 1), dtype=torch.uint8, device=q.device)
+    st = lib().mbe_window_attention(_ptr(q), _ptr(k_win), _ptr(v_win), _ptr(k_cache), _ptr(v_cache), num_pages,
+                                    _ptr(block_table), max_pages, _ptr(prefix_len), _ptr(window_len), _ptr(cu_window),
+                                    _ptr(mask_mode), batch, T, Hq, Hkv, D, block_size, page_size, max_window,
+                                    max_prefix, float(softmax_scale), _ptr(out), _ptr(lse), _ptr(workspace),
+                                    workspace.numel(), _stream(stream))
+    _check("mbe_window_attention", st)
+    return (out, lse) if return_lse else out
+
+
+def edit_decide(logits, committed, tau=0.0, tau_per_row=None, editable=None, *, new_tokens=None, edit_mask=None,
+                confidence=None, argmax=None, want_argmax=True, stream=None):
+    """mbe_edit_decide: see include/mbe.h. Returns (new_tokens, edit_mask, confidence, argmax)."""
+    if logits.dim() != 2 or logits.stride(1) != 1:
+        raise ValueError("logits must be [rows, vocab] with unit stride along the vocabulary")
+    if not logits.is_cuda:
+        raise ValueError("logits must be a CUDA tensor")
+    dt = {torch.float32: 0, torch.bfloat16: 1}.get(logits.dtype)
+    if dt is None:
+        raise TypeError("logits must be float32 or bfloat16")
+    R, V = logits.shape
+    _need(committed, "committed", torch.int32)
+    dev = logits.device
+    new_tokens = torch.empty(R, dtype=torch.int32, device=dev) if new_tokens is None else new_tokens
+    edit_mask = torch.empty(R, dtype=torch.uint8, device=dev) if edit_mask is None else edit_mask
+    confidence = torch.empty(R, dtype=torch.float32, device=dev) if confidence is None else confidence
+    if want_argmax and argmax is None:
+        argmax = torch.empty(R, dtype=torch.int32, device=dev)
+    if tau_per_row is not None:
+        _need(tau_per_row, "tau_per_row", torch.float32)
+    if editable is not None:
+        _need(editable, "editable", torch.uint8)
+    st = lib().mbe_edit_decide(_ptr(logits), dt, logits.stride(0), R, V, _ptr(committed), _ptr(tau_per_row),
+                               float(tau), _ptr(editable), _ptr(new_tokens), _ptr(edit_mask), _ptr(confidence),
+                               _ptr(argmax), _stream(stream))
+    _check("mbe_edit_decide", st)
+    return new_tokens, edit_mask, confidence, argmax
+
+
+def kv_window_write(k_win, v_win, k_cache, v_cache, block_table, prefix_len, window_len, cu_window, *, block_size,
+                    max_window, block_write_mask=None, stream=None):
+    """mbe_kv_window_write: see include/mbe.h. Writes k_cache/v_cache in place."""
+    for t, n in ((k_win, "k_win"), (v_win, "v_win"), (k_cache, "k_cache"), (v_cache, "v_cache")):
+        _need(t, n, torch.bfloat16)
+    for t, n in ((block_table, "block_table"), (prefix_len, "prefix_len"), (window_len, "window_len"),
+                 (cu_window, "cu_window")):
+        _need(t, n, torch.int32)
+    num_pages, Hkv, page_size, D = k_cache.shape
+    batch, max_pages = block_table.shape
+    max_blocks = 0
+    if block_write_mask is not None:
+        _need(block_write_mask, "block_write_mask", torch.uint8)
+        max_blocks = block_write_mask.shape[1]
+    st = lib().mbe_kv_window_write(_ptr(k_win), _ptr(v_win), _ptr(k_cache), _ptr(v_cache), num_pages,
+                                   _ptr(block_table), max_pages, _ptr(prefix_len), _ptr(window_len), _ptr(cu_window),
+                                   _ptr(block_write_mask), max_blocks, batch, max_window, Hkv, D, block_size,
+                                   page_size, _stream(stream))
+    _check("mbe_kv_window_write", st)
+
+
+def get_device_error(stream=None):
+    """(status, flag bits) of the device error word; clears it."""
+    flags = ctypes.c_uint32(0)
+    st = lib().mbe_get_device_error(_stream(stream), ctypes.byref(flags))
+    return st, flags.value

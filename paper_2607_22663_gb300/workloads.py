@@ -281,6 +281,42 @@ def serving128(device="cpu", layers=24, vocab=131072, batch=128):
 WORKLOADS = {"tiny": tiny, "batch8": batch8, "varlen64": varlen64, "long32k": long32k, "serving128": serving128}
 
 
+def extract_sequences(prob: AttnProblem, seqs):
+    """The given sequences of `prob` as a standalone CPU problem (their pages
+    copied into a compact cache, block table renumbered)."""
+    ps = prob.page_size
+    bt_all = prob.block_table.cpu()
+    cu_all = prob.cu_window.cpu()
+    pages, bts, qs, kws, vws = [], [], [], [], []
+    prefix, window, modes, cu = [], [], [], [0]
+    for s in seqs:
+        P, W = prob.prefix_host[s], prob.window_host[s]
+        n = (P + ps - 1) // ps
+        ids = bt_all[s, :n].long()
+        bts.append(list(range(len(pages), len(pages) + n)))
+        pages += ids.tolist()
+        t0 = int(cu_all[s])
+        qs.append(prob.q[t0:t0 + W].cpu())
+        kws.append(prob.k_win[t0:t0 + W].cpu())
+        vws.append(prob.v_win[t0:t0 + W].cpu())
+        prefix.append(P)
+        window.append(W)
+        modes.append(prob.mode_host[s])
+        cu.append(cu[-1] + W)
+    idx = torch.tensor(pages if pages else [0], dtype=torch.long, device=prob.k_cache.device)
+    kc = prob.k_cache.index_select(0, idx).cpu()
+    vc = prob.v_cache.index_select(0, idx).cpu()
+    maxp = max(1, max(len(b) for b in bts))
+    bt = torch.full((len(seqs), maxp), -1, dtype=torch.int32)
+    for i, b in enumerate(bts):
+        bt[i, :len(b)] = torch.tensor(b, dtype=torch.int32)
+    t32 = lambda x: torch.tensor(x, dtype=torch.int32)
+    return AttnProblem(q=torch.cat(qs), k_win=torch.cat(kws), v_win=torch.cat(vws), k_cache=kc, v_cache=vc,
+                       block_table=bt, prefix_len=t32(prefix), window_len=t32(window), cu_window=t32(cu),
+                       mask_mode=torch.tensor(modes, dtype=torch.uint8), block_size=prob.block_size,
+                       page_size=ps, prefix_host=prefix, window_host=window, mode_host=modes)
+
+
 def bf16_bits(t: torch.Tensor):
     """uint16 numpy view of a bf16 tensor (for the oracle's C interface)."""
     return t.detach().cpu().contiguous().view(torch.int16).numpy().view("uint16")
