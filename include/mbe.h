@@ -118,6 +118,41 @@ mbe_status mbe_window_attention(const void* q, const void* k_win, const void* v_
                                 float softmax_scale, void* out, float* lse_or_null, void* workspace,
                                 size_t workspace_bytes, cudaStream_t stream);
 
+/*
+ * mbe_window_attention_noalloc -- mbe_window_attention for callers that cannot
+ * allocate device memory. The paper has no counterpart: this is an interface
+ * convenience of this library, not a step of the method.
+ *
+ * Some callers cannot call cudaMalloc: code that runs inside a host framework
+ * which owns every byte of device memory through its own pool and only hands
+ * out input and output buffers, and code on a latency-critical path that must
+ * not risk the device-wide synchronisation cudaMalloc/cudaFree may cause. This
+ * entry point takes the same arguments as mbe_window_attention except the
+ * workspace, and uses instead a static device array of 64 MiB that lives in
+ * the library (every GPU that loads libmbe holds those 64 MiB until the
+ * process exits). It allocates nothing.
+ *
+ *   - Shapes whose workspace (mbe_window_attention_workspace_size) exceeds
+ *     64 MiB are rejected with MBE_ERR_WORKSPACE before anything is launched.
+ *   - The first call on a device, with that device current, looks up the
+ *     array's device address (cudaGetSymbolAddress); make that first call
+ *     before any stream capture on that device.
+ *   - All calls on a device share the one array and each call overwrites what
+ *     the previous call left there. Calls whose kernels overlap on the GPU
+ *     (for example on two streams without ordering between them) race and give
+ *     wrong results: order them on one stream or with events.
+ * Errors: as mbe_window_attention, plus MBE_ERR_CUDA if the address lookup fails.
+ */
+mbe_status mbe_window_attention_noalloc(const void* q, const void* k_win, const void* v_win, const void* k_cache,
+                                        const void* v_cache, int32_t num_pages, const int32_t* block_table,
+                                        int32_t max_pages_per_seq, const int32_t* prefix_len,
+                                        const int32_t* window_len, const int32_t* cu_window,
+                                        const uint8_t* mask_mode, int32_t batch, int32_t total_q_tokens,
+                                        int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim,
+                                        int32_t block_size, int32_t page_size, int32_t max_window,
+                                        int32_t max_prefix, float softmax_scale, void* out, float* lse_or_null,
+                                        cudaStream_t stream);
+
 /* Bytes of device workspace mbe_window_attention needs for these bounds on the
  * current device (depends on its SM count). Returns 0 for invalid arguments. */
 size_t mbe_window_attention_workspace_size(int32_t batch, int32_t num_q_heads, int32_t num_kv_heads,

@@ -888,3 +888,56 @@ extern "C" mbe_status mbe_window_attention(const void* q, const void* k_win, con
                  cu_window, mask_mode, batch, total_q_tokens, num_q_heads, num_kv_heads, block_size, page_size,
                  max_window, max_prefix, scale, out, lse_or_null, workspace, L, di, stream);
 }
+
+// ------------------------------------------------------------------ no-allocation variant
+// Scratch for mbe_window_attention_noalloc: a fixed device array that every
+// GPU loading this library holds until the process exits. Host code must not
+// pass the symbol itself to a kernel (on the host it is only a stand-in); the
+// device address is looked up once per device with cudaGetSymbolAddress.
+namespace mbe {
+namespace attn {
+constexpr size_t kNoAllocScratchBytes = size_t(64) << 20;  // 64 MiB
+}  // namespace attn
+}  // namespace mbe
+
+static __device__ __align__(256) uint8_t g_noalloc_scratch[mbe::attn::kNoAllocScratchBytes];
+
+namespace {
+
+// Device address of g_noalloc_scratch on device `dev` (looked up on the first
+// call made with that device current), or nullptr if the lookup failed.
+void* noalloc_scratch(int dev) {
+  static void* addr[64] = {};
+  static std::mutex mu;
+  if (dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lock(mu);
+  if (addr[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) return nullptr;
+    addr[dev] = p;
+  }
+  return addr[dev];
+}
+
+}  // namespace
+
+extern "C" mbe_status mbe_window_attention_noalloc(const void* q, const void* k_win, const void* v_win,
+                                                   const void* k_cache, const void* v_cache, int32_t num_pages,
+                                                   const int32_t* block_table, int32_t max_pages_per_seq,
+                                                   const int32_t* prefix_len, const int32_t* window_len,
+                                                   const int32_t* cu_window, const uint8_t* mask_mode, int32_t batch,
+                                                   int32_t total_q_tokens, int32_t num_q_heads, int32_t num_kv_heads,
+                                                   int32_t head_dim, int32_t block_size, int32_t page_size,
+                                                   int32_t max_window, int32_t max_prefix, float softmax_scale,
+                                                   void* out, float* lse_or_null, cudaStream_t stream) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return MBE_ERR_CUDA;
+  void* scratch = noalloc_scratch(dev);
+  if (scratch == nullptr) return MBE_ERR_CUDA;
+  // The regular entry point checks the bounds against the scratch size and
+  // returns MBE_ERR_WORKSPACE, launching nothing, when they need more.
+  return mbe_window_attention(q, k_win, v_win, k_cache, v_cache, num_pages, block_table, max_pages_per_seq,
+                              prefix_len, window_len, cu_window, mask_mode, batch, total_q_tokens, num_q_heads,
+                              num_kv_heads, head_dim, block_size, page_size, max_window, max_prefix, softmax_scale,
+                              out, lse_or_null, scratch, mbe::attn::kNoAllocScratchBytes, stream);
+}

@@ -54,6 +54,9 @@ def lib(build_if_missing: bool = True):
     L.mbe_window_attention.restype = ctypes.c_int
     L.mbe_window_attention.argtypes = [P, P, P, P, P, i32, P, i32, P, P, P, P, i32, i32, i32, i32, i32, i32, i32, i32,
                                        i32, f32, P, P, P, sz, P]
+    L.mbe_window_attention_noalloc.restype = ctypes.c_int
+    L.mbe_window_attention_noalloc.argtypes = [P, P, P, P, P, i32, P, i32, P, P, P, P, i32, i32, i32, i32, i32, i32,
+                                               i32, i32, i32, f32, P, P, P]
     L.mbe_window_attention_workspace_size.restype = sz
     L.mbe_window_attention_workspace_size.argtypes = [i32, i32, i32, i32, i32, i32]
     L.mbe_edit_decide.restype = ctypes.c_int
@@ -138,6 +141,24 @@ def window_attention(q, k_win, v_win, k_cache, v_cache, block_table, prefix_len,
                                     workspace.numel(), _stream(stream))
     _check("mbe_window_attention", st)
     return (out, lse) if return_lse else out
+
+
+def window_attention_noalloc(q, k_win, v_win, k_cache, v_cache, block_table, prefix_len, window_len, cu_window,
+                             mask_mode, *, block_size, max_window, max_prefix, softmax_scale=0.0, out, lse=None,
+                             stream=None):
+    """mbe_window_attention_noalloc: the attention with the library's static
+    64 MiB scratch instead of a workspace, for callers that must not allocate.
+    `out` (and `lse`, if wanted) must be given: this call allocates nothing."""
+    T, Hq, D = q.shape
+    num_pages, Hkv, page_size, _ = k_cache.shape
+    batch, max_pages = block_table.shape
+    st = lib().mbe_window_attention_noalloc(_ptr(q), _ptr(k_win), _ptr(v_win), _ptr(k_cache), _ptr(v_cache),
+                                            num_pages, _ptr(block_table), max_pages, _ptr(prefix_len),
+                                            _ptr(window_len), _ptr(cu_window), _ptr(mask_mode), batch, T, Hq, Hkv,
+                                            D, block_size, page_size, max_window, max_prefix, float(softmax_scale),
+                                            _ptr(out), _ptr(lse), _stream(stream))
+    _check("mbe_window_attention_noalloc", st)
+    return out
 
 
 def edit_decide(logits, committed, tau=0.0, tau_per_row=None, editable=None, *, new_tokens=None, edit_mask=None,
