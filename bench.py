@@ -68,6 +68,23 @@ def edit_bytes(rows, vocab, elem):
     return rows * vocab * elem + rows * (4 + 4 + 1 + 4)
 
 
+# ------------------------------------------------------------------ ranks
+def max_over_ranks(x: float, device="cpu") -> float:
+    """Maximum of a per-rank scalar over all ranks (identity on one rank)."""
+    if not torch.distributed.is_available() or not torch.distributed.is_initialized():
+        return x
+    if torch.distributed.get_world_size() == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: int, world: int, seconds_max: float) -> float:
+    """Units processed by all ranks per second of the slowest rank."""
+    return units_per_rank * world / seconds_max
+
+
 # ------------------------------------------------------------------ clocks
 class ClockSampler:
     def __init__(self, index):
@@ -217,11 +234,7 @@ def run_gpu(args, rank, world):
         t1.record(stream)
         barrier()
     clocks = clk.summary()
-    ms_total = t0.elapsed_time(t1)
-    if world > 1:
-        tt = torch.tensor([ms_total], device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        ms_total = float(tt.item())
+    ms_total = max_over_ranks(t0.elapsed_time(t1), dev)
     ms_step = ms_total / K
     attn_ms = [statistics.mean(ev_attn[k][i][0].elapsed_time(ev_attn[k][i][1]) for k in range(K))
                for i in range(len(attn))]
@@ -236,8 +249,7 @@ def run_gpu(args, rank, world):
     attn_time = sum(attn_ms)
     attn_tflops = sum(flops) / (attn_time * 1e-3) / 1e12
     attn_gbs = sum(abytes) / (attn_time * 1e-3) / 1e9
-    windows = a0.batch * world
-    value = windows / (ms_step * 1e-3)
+    value = whole_job_rate(a0.batch, world, ms_step * 1e-3)
     res = {"metric": METRIC, "value": round(value, 3), "unit": "windows/s", "n_gpus": world, "steps": K,
            "warmup": args.warmup, "ms_per_step": round(ms_step, 4), "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
@@ -330,13 +342,8 @@ def run_e2e(args, w, attention_call, edit_call, dev, stream, world, new_t, mask_
     for _ in range(K):
         step()
     torch.cuda.synchronize()
-    el = time.perf_counter() - t0
-    if world > 1:
-        tt = torch.tensor([el], device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        el = float(tt.item())
-    windows = attn[0].batch * world
-    return {"value": round(windows * K / el, 3), "unit": "windows/s", "h2d_bytes_per_step": int(h2d),
+    el = max_over_ranks(time.perf_counter() - t0, dev)
+    return {"value": round(whole_job_rate(attn[0].batch * K, world, el), 3), "unit": "windows/s", "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h), "steps": K,
             "resident_state": "paged KV caches of every layer (written by earlier passes)"}
 

@@ -241,19 +241,24 @@ struct AttnParams {
   float scale_log2;
 };
 
+// Shared memory: two Q tiles, then a ring of kSlots K-or-V tiles. Items are
+// loaded in the order K(0), V(0), K(1), V(1), ...; K(t) is released once the
+// QK products of tile t are done and V(t) once its PV products are done, so up
+// to kSlots tile loads can be in flight.
 template <int D>
 struct Smem {
   static constexpr int kHalves = D / 64;
   static constexpr int kHalfBytes = 128 * 128;             // 128 rows x 128 B
   static constexpr int kQTile = kTileRows * D * 2;
-  static constexpr int kKVTile = kTileKeys * D * 2;
+  static constexpr int kItem = kTileKeys * D * 2;          // one K or one V tile
+  static constexpr int kSlots = D == 128 ? 5 : 8;
   static constexpr int kQ = 0;
-  static constexpr int kK = 2 * kQTile;
-  static constexpr int kV = kK + 2 * kKVTile;
-  static constexpr int kUsed = kV + 2 * kKVTile;
+  static constexpr int kRing = 2 * kQTile;
+  static constexpr int kUsed = kRing + kSlots * kItem;
   // at least 114 KB so that one CTA (and its 512 TMEM columns) owns the SM
   static constexpr int kBytes = (kUsed > 120 * 1024 ? kUsed : 120 * 1024) + 1024;
 };
+constexpr int kMaxSlots = 8;
 
 __device__ __forceinline__ float ex2f(float x) {
   float y;
@@ -264,7 +269,7 @@ __device__ __forceinline__ float neg_inf() { return __int_as_float(0xff800000u);
 
 struct Bars {
   uint64_t q_full, q_empty, mma_done;
-  uint64_t k_full[2], v_full[2], kv_empty[2];
+  uint64_t full[kMaxSlots], empty[kMaxSlots];
   uint64_t s_full[2], p_full[2], o_full[2], o_empty[2];
   uint64_t u_full[2], u_empty[2];
 };
@@ -292,10 +297,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(bar(bars.q_full), 1);
     mbar_init(bar(bars.q_empty), 1);
     mbar_init(bar(bars.mma_done), 1);
+    for (int i = 0; i < S::kSlots; ++i) {
+      mbar_init(bar(bars.full[i]), 1);
+      mbar_init(bar(bars.empty[i]), 1);
+    }
     for (int i = 0; i < 2; ++i) {
-      mbar_init(bar(bars.k_full[i]), 1);
-      mbar_init(bar(bars.v_full[i]), 1);
-      mbar_init(bar(bars.kv_empty[i]), 1);
       mbar_init(bar(bars.s_full[i]), 1);
       mbar_init(bar(bars.p_full[i]), 4);
       mbar_init(bar(bars.o_full[i]), 1);
@@ -316,92 +322,127 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // ---------------------------------------------------------------- producer
+    // The whole warp runs the loop (lane 0 issues the copies and barrier ops);
+    // the lanes fetch 32 block-table entries at a time for the page lookups.
     if (lane == 0) {
       tma_prefetch_desc(&tm_q);
       tma_prefetch_desc(&tm_kw);
       tma_prefetch_desc(&tm_vw);
       tma_prefetch_desc(&tm_kc);
       tma_prefetch_desc(&tm_vc);
-      uint32_t kv_it = 0, u_it = 0, q_loads = 0;
-      bool ok = true;
-      for (;;) {
-        const int uidx = atomicAdd(&p.hdr->counter, 1);
-        const bool done = uidx >= n_units;
-        const int slot = u_it & 1;
-        if (u_it >= 2 && !mbar_wait(bar(bars.u_empty[slot]), ((u_it >> 1) - 1) & 1, abort_flag)) { ok = false; break; }
-        WorkUnit wu;
-        if (done) {
-          wu.seq = -1;
-        } else {
-          wu = p.units[uidx];
-        }
-        unit_ring[slot] = wu;
-        mbar_arrive(bar(bars.u_full[slot]));
-        ++u_it;
-        if (done) break;
-        const int W = wu.window_mode & 0x3FFFFFFF;
-        const int n_qt = (W * p.G - wu.row0) > kTileRows ? 2 : 1;
-        const int cu = p.cu_window[wu.seq];
-        if (q_loads >= 1 && !mbar_wait(bar(bars.q_empty), (q_loads - 1) & 1, abort_flag)) { ok = false; break; }
+    }
+    constexpr unsigned kAll = 0xffffffffu;
+    uint32_t item = 0, u_it = 0, q_loads = 0;
+    bool ok = true;
+    auto slot_of = [](uint32_t n) { return n % S::kSlots; };
+    for (;;) {
+      int uidx = 0;
+      if (lane == 0) uidx = atomicAdd(&p.hdr->counter, 1);
+      uidx = __shfl_sync(kAll, uidx, 0);
+      const bool done = uidx >= n_units;
+      const int uslot = u_it & 1;
+      if (u_it >= 2) {
+        ok = __all_sync(kAll, mbar_wait(bar(bars.u_empty[uslot]), ((u_it >> 1) - 1) & 1, abort_flag));
+        if (!ok) break;
+      }
+      WorkUnit wu;
+      if (done) {
+        wu.seq = -1;
+      } else {
+        wu = p.units[uidx];
+      }
+      if (lane == 0) {
+        unit_ring[uslot] = wu;
+        mbar_arrive(bar(bars.u_full[uslot]));
+      }
+      __syncwarp();
+      ++u_it;
+      if (done) break;
+      const int W = wu.window_mode & 0x3FFFFFFF;
+      const int n_qt = (W * p.G - wu.row0) > kTileRows ? 2 : 1;
+      const int cu = p.cu_window[wu.seq];
+      if (q_loads >= 1) {
+        ok = __all_sync(kAll, mbar_wait(bar(bars.q_empty), (q_loads - 1) & 1, abort_flag));
+        if (!ok) break;
+      }
+      if (lane == 0) {
         mbar_arrive_expect_tx(bar(bars.q_full), n_qt * S::kQTile);
         for (int qt = 0; qt < n_qt; ++qt)
           for (int h = 0; h < S::kHalves; ++h)
             tma_load_3d(sbase + S::kQ + qt * S::kQTile + h * S::kHalfBytes, &tm_q, bar(bars.q_full), h * 64,
                         wu.kv_head * p.G, cu + (wu.row0 + qt * kTileRows) / p.G);
-        ++q_loads;
-        const int P = wu.prefix;
-        const int nP = (P + kTileKeys - 1) / kTileKeys;
-        for (int t = wu.tile_begin; t < wu.tile_end; ++t, ++kv_it) {
-          const int st = kv_it & 1;
-          if (kv_it >= 2 && !mbar_wait(bar(bars.kv_empty[st]), ((kv_it >> 1) - 1) & 1, abort_flag)) { ok = false; break; }
-          const uint32_t kdst = sbase + S::kK + st * S::kKVTile;
-          const uint32_t vdst = sbase + S::kV + st * S::kKVTile;
-          mbar_arrive_expect_tx(bar(bars.k_full[st]), S::kKVTile);
-          if (t < nP) {
-            int pages[16], offs[16];  // page_size >= 8: at most 16 loads per tile
-            for (int l = 0; l < p.loads_per_tile; ++l) {
-              const int key0 = t * kTileKeys + l * p.box_rows;
-              int page = p.num_pages;  // out of range: TMA fills zeros
-              if (key0 < P) {
-                page = p.block_table[static_cast<int64_t>(wu.seq) * p.max_pages + key0 / p.page_size];
-                if (page < 0 || page >= p.num_pages) {
-                  atomicOr(&g_error_word, MBE_DEVERR_PAGE);
-                  page = p.num_pages;
-                }
-              }
-              pages[l] = page;
-              offs[l] = key0 % p.page_size;
-              for (int h = 0; h < S::kHalves; ++h)
-                tma_load_4d(kdst + h * S::kHalfBytes + l * p.box_rows * 128, &tm_kc, bar(bars.k_full[st]), h * 64,
-                            offs[l], wu.kv_head, page);
-            }
-            mbar_arrive_expect_tx(bar(bars.v_full[st]), S::kKVTile);
-            for (int l = 0; l < p.loads_per_tile; ++l)
-              for (int h = 0; h < S::kHalves; ++h)
-                tma_load_4d(vdst + h * S::kHalfBytes + l * p.box_rows * 128, &tm_vc, bar(bars.v_full[st]), h * 64,
-                            offs[l], wu.kv_head, pages[l]);
-          } else {
-            const int tok = cu + (t - nP) * kTileKeys;
-            for (int h = 0; h < S::kHalves; ++h)
-              tma_load_3d(kdst + h * S::kHalfBytes, &tm_kw, bar(bars.k_full[st]), h * 64, wu.kv_head, tok);
-            mbar_arrive_expect_tx(bar(bars.v_full[st]), S::kKVTile);
-            for (int h = 0; h < S::kHalves; ++h)
-              tma_load_3d(vdst + h * S::kHalfBytes, &tm_vw, bar(bars.v_full[st]), h * 64, wu.kv_head, tok);
+      }
+      ++q_loads;
+      const int P = wu.prefix;
+      const int nP = (P + kTileKeys - 1) / kTileKeys;
+      const int64_t bt_row = static_cast<int64_t>(wu.seq) * p.max_pages;
+      // Page ids: lane L holds the physical page of logical pages pg_base + L
+      // (pg_lo) and pg_base + 32 + L (pg_hi); one coalesced block-table read
+      // serves 32 pages.
+      auto fetch_page = [&](int lpage) {
+        int pg = p.num_pages;  // out of range: TMA fills zeros
+        if (lpage >= 0 && static_cast<int64_t>(lpage) * p.page_size < P) {
+          pg = p.block_table[bt_row + lpage];
+          if (pg < 0 || pg >= p.num_pages) {
+            atomicOr(&g_error_word, MBE_DEVERR_PAGE);
+            pg = p.num_pages;
           }
         }
-        if (!ok) break;
-      }
-      if (!ok) {
-        *abort_flag = 1;
-        atomicOr(&g_error_word, MBE_DEVERR_TIMEOUT);
-        // let the copies already issued land before the CTA can exit
-        const int zero = 0;
-        for (uint32_t k = (kv_it >= 2 ? kv_it - 2 : 0); k < kv_it; ++k) {
-          mbar_wait(bar(bars.k_full[k & 1]), (k >> 1) & 1, &zero);
-          mbar_wait(bar(bars.v_full[k & 1]), (k >> 1) & 1, &zero);
+        return pg;
+      };
+      int pg_base = -(1 << 30), pg_lo = 0, pg_hi = 0;
+      auto page_of = [&](int lp) {  // warp-uniform lp >= pg_base
+        return __shfl_sync(kAll, lp < pg_base + 32 ? pg_lo : pg_hi, (lp - pg_base) & 31);
+      };
+      auto ensure_window = [&](int lp) {  // makes lp the current page window's anchor if needed
+        if (lp < pg_base || lp >= pg_base + 64) {
+          pg_base = lp;
+          pg_lo = fetch_page(pg_base + lane);
+          pg_hi = fetch_page(pg_base + 32 + lane);
+        } else if (lp >= pg_base + 32) {
+          pg_base += 32;
+          pg_lo = pg_hi;
+          pg_hi = fetch_page(pg_base + 32 + lane);
         }
-        if (q_loads >= 1) mbar_wait(bar(bars.q_full), (q_loads - 1) & 1, &zero);
+      };
+      for (int t = wu.tile_begin; t < wu.tile_end && ok; ++t) {
+        if (t < nP) ensure_window((t * kTileKeys) / p.page_size);
+        for (int kv = 0; kv < 2; ++kv, ++item) {
+          const uint32_t sl = slot_of(item), use = item / S::kSlots;
+          if (use >= 1) {
+            ok = __all_sync(kAll, mbar_wait(bar(bars.empty[sl]), (use - 1) & 1, abort_flag));
+            if (!ok) break;
+          }
+          const uint32_t dst = sbase + S::kRing + sl * S::kItem;
+          const uint32_t fb = bar(bars.full[sl]);
+          if (lane == 0) mbar_arrive_expect_tx(fb, S::kItem);
+          if (t < nP) {
+            const CUtensorMap* tm = kv ? &tm_vc : &tm_kc;
+            for (int l = 0; l < p.loads_per_tile; ++l) {
+              const int key0 = t * kTileKeys + l * p.box_rows;
+              const int page = page_of(key0 / p.page_size);
+              if (lane == 0)
+                for (int h = 0; h < S::kHalves; ++h)
+                  tma_load_4d(dst + h * S::kHalfBytes + l * p.box_rows * 128, tm, fb, h * 64, key0 % p.page_size,
+                              wu.kv_head, page);
+            }
+          } else if (lane == 0) {
+            const int tok = cu + (t - nP) * kTileKeys;
+            for (int h = 0; h < S::kHalves; ++h)
+              tma_load_3d(dst + h * S::kHalfBytes, kv ? &tm_vw : &tm_kw, fb, h * 64, wu.kv_head, tok);
+          }
+        }
       }
+      if (!ok) break;
+    }
+    if (!ok && lane == 0) {
+      *abort_flag = 1;
+      atomicOr(&g_error_word, MBE_DEVERR_TIMEOUT);
+      // let the copies already issued land before the CTA can exit
+      const int zero = 0;
+      for (uint32_t n = (item >= S::kSlots ? item - S::kSlots : 0); n < item; ++n)
+        mbar_wait(bar(bars.full[slot_of(n)]), (n / S::kSlots) & 1, &zero);
+      if (q_loads >= 1) mbar_wait(bar(bars.q_full), (q_loads - 1) & 1, &zero);
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
@@ -411,9 +452,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t kv_it = 0, u_it = 0, q_it = 0;
       uint32_t p_cnt[2] = {0, 0}, o_cnt[2] = {0, 0};
       bool ok = true;
-      auto issue_qk = [&](int i, int st) {
+      auto item_addr = [&](uint32_t n) { return sbase + S::kRing + (n % S::kSlots) * S::kItem; };
+      auto wait_item = [&](uint32_t n) { return mbar_wait(bar(bars.full[n % S::kSlots]), (n / S::kSlots) & 1, abort_flag); };
+      auto release_item = [&](uint32_t n) { umma_commit(bar(bars.empty[n % S::kSlots])); };
+      auto issue_qk = [&](int i, uint32_t ka) {
         const uint32_t qa = sbase + S::kQ + i * S::kQTile;
-        const uint32_t ka = sbase + S::kK + st * S::kKVTile;
 #pragma unroll
         for (int h = 0; h < S::kHalves; ++h)
 #pragma unroll
@@ -421,8 +464,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             umma_ss(tmem + kTmemS + 128 * i, sdesc_sw128(qa + h * S::kHalfBytes + k * 32, 16, 1024),
                     sdesc_sw128(ka + h * S::kHalfBytes + k * 32, 16, 1024), idesc_qk, (h | k) ? 1u : 0u);
       };
-      auto issue_pv = [&](int i, int st, bool acc) {
-        const uint32_t va = sbase + S::kV + st * S::kKVTile;
+      auto issue_pv = [&](int i, uint32_t va, bool acc) {
 #pragma unroll
         for (int kk = 0; kk < kTileKeys / 16; ++kk)
           umma_ts(tmem + i * D, tmem + kTmemS + 128 * i + kk * 8, sdesc_sw128(va + kk * 16 * 128, S::kHalfBytes, 1024),
@@ -440,17 +482,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int n_t = wu.tile_end - wu.tile_begin;
         if (!mbar_wait(bar(bars.q_full), q_it & 1, abort_flag)) { ok = false; break; }
         ++q_it;
-        if (!mbar_wait(bar(bars.k_full[kv_it & 1]), (kv_it >> 1) & 1, abort_flag)) { ok = false; break; }
+        // items of tile ki: K = 2 ki, V = 2 ki + 1
+        if (!wait_item(2 * kv_it)) { ok = false; break; }
         tc_fence_after();
         for (int i = 0; i < n_qt; ++i) {
-          issue_qk(i, kv_it & 1);
+          issue_qk(i, item_addr(2 * kv_it));
           umma_commit(bar(bars.s_full[i]));
         }
+        release_item(2 * kv_it);
         if (n_t == 1) umma_commit(bar(bars.q_empty));
         for (int j = 0; j < n_t && ok; ++j) {
           const uint32_t ki = kv_it + j;
-          const int st = ki & 1;
-          if (!mbar_wait(bar(bars.v_full[st]), (ki >> 1) & 1, abort_flag)) { ok = false; break; }
+          if (!wait_item(2 * ki + 1)) { ok = false; break; }
           for (int i = 0; i < n_qt; ++i) {
             if (!mbar_wait(bar(bars.p_full[i]), p_cnt[i] & 1, abort_flag)) { ok = false; break; }
             ++p_cnt[i];
@@ -459,18 +502,21 @@ __global__ void __launch_bounds__(kThreads, 1)
               break;
             }
             tc_fence_after();
-            issue_pv(i, st, j > 0);
+            issue_pv(i, item_addr(2 * ki + 1), j > 0);
             if (j == n_t - 1) umma_commit(bar(bars.o_full[i]));
-            if (i == n_qt - 1) umma_commit(bar(bars.kv_empty[st]));
+            if (i == n_qt - 1) release_item(2 * ki + 1);
             if (j + 1 < n_t) {
-              const uint32_t kn = ki + 1;
+              const uint32_t kn = 2 * (ki + 1);
               if (i == 0) {
-                if (!mbar_wait(bar(bars.k_full[kn & 1]), (kn >> 1) & 1, abort_flag)) { ok = false; break; }
+                if (!wait_item(kn)) { ok = false; break; }
                 tc_fence_after();
               }
-              issue_qk(i, kn & 1);
+              issue_qk(i, item_addr(kn));
               umma_commit(bar(bars.s_full[i]));
-              if (j + 2 == n_t && i == n_qt - 1) umma_commit(bar(bars.q_empty));
+              if (i == n_qt - 1) {
+                release_item(kn);
+                if (j + 2 == n_t) umma_commit(bar(bars.q_empty));
+              }
             }
           }
         }
@@ -529,51 +575,81 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++s_cnt;
         tc_fence_after();
         const int n_vis = t < nP ? min(kTileKeys, P - t * kTileKeys) : max(0, min(kTileKeys, lim - (t - nP) * kTileKeys));
-        uint32_t sr[128];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) tmem_ld32(tS + 32 * c, *reinterpret_cast<uint32_t(*)[32]>(&sr[32 * c]));
+        // The whole S row (128 fp32) comes from TMEM in one load; P is packed to
+        // bf16 in place (entry k <- columns 2k, 2k+1) and stored as 64 columns
+        // over the start of the same TMEM region.
+        const bool full = __all_sync(0xffffffffu, n_vis == kTileKeys);
+        uint32_t v[128];
+        tmem_ld128(tS, v);
         float mx = neg_inf();
+        if (full) {
+          float a0 = neg_inf(), a1 = neg_inf();
 #pragma unroll
-        for (int c = 0; c < 128; ++c)
-          if (c < n_vis) mx = fmaxf(mx, __uint_as_float(sr[c]));
-        const float m_new = fmaxf(m, mx * p.scale_log2);
-        const bool need = m_new > m + kRescaleLog2;
-        if (__any_sync(0xffffffffu, need)) {
-          const float alpha = (m_new == neg_inf()) ? 1.f : ex2f(m - m_new);
-          l *= alpha;
-          if (j > 0) {
-#pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
-              uint32_t o[32];
-              tmem_ld32(tO + 32 * c, o);
-#pragma unroll
-              for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * alpha);
-              tmem_st32(tO + 32 * c, o);
-            }
+          for (int k = 0; k < 128; k += 4) {
+            a0 = fmax3(a0, __uint_as_float(v[k]), __uint_as_float(v[k + 1]));
+            a1 = fmax3(a1, __uint_as_float(v[k + 2]), __uint_as_float(v[k + 3]));
           }
+          mx = fmaxf(a0, a1);
+        } else {
+#pragma unroll
+          for (int k = 0; k < 128; ++k)
+            if (k < n_vis) mx = fmaxf(mx, __uint_as_float(v[k]));
+        }
+        // Lazy rescaling: the reference max m only moves when the tile's max
+        // exceeds it by more than 2^8; P, l and O then all use the new m.
+        const float m_new = fmaxf(m, mx * p.scale_log2);
+        const bool rescale = __any_sync(0xffffffffu, m_new > m + kRescaleLog2);
+        float alpha = 1.f;
+        if (rescale) {
+          alpha = (m_new == neg_inf()) ? 1.f : ex2f(m - m_new);
           m = m_new;
         }
-        const float mu = (m == neg_inf()) ? 0.f : m;
+        const float neg_mu = (m == neg_inf()) ? 0.f : -m;
+        float l0 = 0.f, l1 = 0.f;
+        if (full) {
+          const float2 sl2 = make_float2(p.scale_log2, p.scale_log2), nm2 = make_float2(neg_mu, neg_mu);
+          float2 la = make_float2(0.f, 0.f), lb = make_float2(0.f, 0.f);
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          uint32_t pk[32];
-#pragma unroll
-          for (int k = 0; k < 32; ++k) {
-            const int c = 64 * h + 2 * k;
-            const float p0 = c < n_vis ? ex2f(fmaf(__uint_as_float(sr[c]), p.scale_log2, -mu)) : 0.f;
-            const float p1 = c + 1 < n_vis ? ex2f(fmaf(__uint_as_float(sr[c + 1]), p.scale_log2, -mu)) : 0.f;
-            l += p0 + p1;
-            pk[k] = pack_bf16x2(p0, p1);
+          for (int k = 0; k < 64; ++k) {
+            const float2 x = ffma2(make_float2(__uint_as_float(v[2 * k]), __uint_as_float(v[2 * k + 1])), sl2, nm2);
+            const float2 e = make_float2(ex2f(x.x), ex2f(x.y));
+            if (k & 1) lb = fadd2(lb, e); else la = fadd2(la, e);
+            v[k] = pack_bf16x2(e.x, e.y);
           }
-          tmem_st32(tS + 32 * h, pk);
+          const float2 ls = fadd2(la, lb);
+          l0 = ls.x;
+          l1 = ls.y;
+        } else {
+#pragma unroll
+          for (int k = 0; k < 64; ++k) {
+            const float p0 = 2 * k < n_vis ? ex2f(fmaf(__uint_as_float(v[2 * k]), p.scale_log2, neg_mu)) : 0.f;
+            const float p1 = 2 * k + 1 < n_vis ? ex2f(fmaf(__uint_as_float(v[2 * k + 1]), p.scale_log2, neg_mu)) : 0.f;
+            l0 += p0;
+            l1 += p1;
+            v[k] = pack_bf16x2(p0, p1);
+          }
+        }
+        tmem_st64(tS, v);
+        l = l * alpha + (l0 + l1);
+        if (rescale && j > 0) {
+          // O holds PV of tiles < j (complete: s_full(j) was committed after them)
+#pragma unroll 1
+          for (int c = 0; c < D / 32; ++c) {
+            uint32_t o[32];
+            tmem_ld32(tO + 32 * c, o);
+#pragma unroll
+            for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * alpha);
+            tmem_st32(tO + 32 * c, o);
+          }
         }
         tmem_st_wait();
         if (wg == 0 && t == nP - 1 && (P % kTileKeys) != 0) {
           // stale cache rows past the prefix end: zero them in V so that 0 * V stays 0
-          ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.v_full[ki & 1]), (ki >> 1) & 1, abort_flag));
+          const uint32_t nv = 2 * ki + 1;  // the V item of this tile
+          ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.full[nv % S::kSlots]), (nv / S::kSlots) & 1, abort_flag));
           if (!ok) break;
           const int v0 = P % kTileKeys;
-          uint8_t* vt = smem + S::kV + (ki & 1) * S::kKVTile;
+          uint8_t* vt = smem + S::kRing + (nv % S::kSlots) * S::kItem;
           const int per_row = S::kHalves * 8;  // 16-byte chunks per key row
           for (int idx = r; idx < (kTileKeys - v0) * per_row; idx += kTileRows) {
             const int row = v0 + idx / per_row, rem = idx % per_row;
@@ -659,9 +735,10 @@ struct MergeParams {
   const int32_t* cu_window;
   __nv_bfloat16* out;
   float* lse;
-  int Hq, G, D;
+  int Hq, G;
 };
 
+template <int D>
 __global__ void __launch_bounds__(kUnitRows) attn_merge_kernel(const MergeParams p) {
   const int gi = blockIdx.x;
   if (gi >= p.hdr->n_groups) return;
@@ -674,15 +751,17 @@ __global__ void __launch_bounds__(kUnitRows) attn_merge_kernel(const MergeParams
   for (int k = 0; k < grp.n_splits; ++k)
     M = fmaxf(M, p.part_lse[static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r]);
   float wsum = 0.f;
-  float acc[128];
-  for (int d = 0; d < p.D; ++d) acc[d] = 0.f;
+  float acc[D];
+#pragma unroll
+  for (int d = 0; d < D; ++d) acc[d] = 0.f;
   for (int k = 0; k < grp.n_splits; ++k) {
     const float lk = p.part_lse[static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r];
     const float w = (lk == neg_inf()) ? 0.f : ex2f(lk - M);
     if (w == 0.f) continue;
     wsum += w;
-    const float4* src = reinterpret_cast<const float4*>(p.part_o + (static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r) * p.D);
-    for (int d4 = 0; d4 < p.D / 4; ++d4) {
+    const float4* src = reinterpret_cast<const float4*>(p.part_o + (static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r) * D);
+#pragma unroll
+    for (int d4 = 0; d4 < D / 4; ++d4) {
       const float4 v = src[d4];
       acc[4 * d4] += w * v.x;
       acc[4 * d4 + 1] += w * v.y;
@@ -693,8 +772,11 @@ __global__ void __launch_bounds__(kUnitRows) attn_merge_kernel(const MergeParams
   const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
   const int cu = p.cu_window[grp.seq];
   const int64_t orow = static_cast<int64_t>(cu + qi) * p.Hq + grp.kv_head * p.G + hh;
-  uint32_t* dst = reinterpret_cast<uint32_t*>(p.out + orow * p.D);
-  for (int d = 0; d < p.D; d += 2) dst[d / 2] = pack_bf16x2(acc[d] * inv, acc[d + 1] * inv);
+  uint4* dst = reinterpret_cast<uint4*>(p.out + orow * D);
+#pragma unroll
+  for (int d = 0; d < D; d += 8)
+    dst[d / 8] = make_uint4(pack_bf16x2(acc[d] * inv, acc[d + 1] * inv), pack_bf16x2(acc[d + 2] * inv, acc[d + 3] * inv),
+                            pack_bf16x2(acc[d + 4] * inv, acc[d + 5] * inv), pack_bf16x2(acc[d + 6] * inv, acc[d + 7] * inv));
   if (p.lse) p.lse[orow] = (wsum > 0.f ? M + __log2f(wsum) : neg_inf()) * 0.6931471805599453f;
 }
 
@@ -828,8 +910,8 @@ mbe_status run(const void* q, const void* k_win, const void* v_win, const void* 
   attn_kernel<D><<<di->num_sms, kThreads, Smem<D>::kBytes, stream>>>(tq, tkw, tvw, tkc, tvc, ap);
   if (cudaGetLastError() != cudaSuccess) return MBE_ERR_CUDA;
   MergeParams mp{hdr, reinterpret_cast<const MergeGroup*>(ws + L.groups), ap.part_o, ap.part_lse, cu_window,
-                 ap.out, lse, Hq, G, D};
-  attn_merge_kernel<<<static_cast<unsigned>(L.max_groups), kUnitRows, 0, stream>>>(mp);
+                 ap.out, lse, Hq, G};
+  attn_merge_kernel<D><<<static_cast<unsigned>(L.max_groups), kUnitRows, 0, stream>>>(mp);
   if (cudaGetLastError() != cudaSuccess) return MBE_ERR_CUDA;
   return MBE_OK;
 }

@@ -20,7 +20,8 @@ The shapes follow the five workloads the library is measured on:
                 32/8 heads, page 64 with a random page permutation; KV write of
                 each window; seed 4.
 * ``serving128`` 128 sequences, prefix U[512,16384] (not rounded), window 64,
-                32/8 heads, page 32, 24 layers with independent Q/K/V and
+                32/8 heads, page 64 (not stated by the workload; 64 tokens make one
+                8 KB TMA box per page, head and half of D), 24 layers with independent Q/K/V and
                 caches; bf16 logits [8192 x 131072] N(0, sd 2) with peaks
                 U(0,12) on every row, committed = the row argmax on 80% of
                 rows; tau 0.9; seed 5.
@@ -258,12 +259,12 @@ def long32k(device="cpu", windows=(64, 128, 256)):
     return {"name": "long32k", "attn": calls, "edit": None, "layers": 1}
 
 
-def serving128(device="cpu", layers=24, vocab=131072, batch=128):
+def serving128(device="cpu", layers=24, vocab=131072, batch=128, page_size=64):
     g = _gen(5, "cpu")
     prefix = torch.randint(512, 16385, (batch,), generator=g).tolist()
     window = [64] * batch
     gd = _gen(5, device)
-    first = attention_problem(prefix, window, [BIDIRECTIONAL] * batch, 32, 8, 128, 32, 32, 5, device, g=gd)
+    first = attention_problem(prefix, window, [BIDIRECTIONAL] * batch, 32, 8, 128, 32, page_size, 5, device, g=gd)
     attn = [first]
     for _ in range(1, layers):
         attn.append(AttnProblem(q=_randn_bf16(first.q.shape, gd, device), k_win=_randn_bf16(first.k_win.shape, gd, device),
@@ -271,7 +272,8 @@ def serving128(device="cpu", layers=24, vocab=131072, batch=128):
                                 k_cache=_randn_bf16(first.k_cache.shape, gd, device),
                                 v_cache=_randn_bf16(first.v_cache.shape, gd, device), block_table=first.block_table,
                                 prefix_len=first.prefix_len, window_len=first.window_len, cu_window=first.cu_window,
-                                mask_mode=first.mask_mode, block_size=32, page_size=32, prefix_host=first.prefix_host,
+                                mask_mode=first.mask_mode, block_size=32, page_size=page_size,
+                                prefix_host=first.prefix_host,
                                 window_host=first.window_host, mode_host=first.mode_host))
     edit = edit_problem(batch * 64, vocab, torch.bfloat16, 5, device, sd=2.0, peak_frac=1.0, peak_lo=0.0,
                         peak_hi=12.0, tau=0.9, committed_argmax_frac=0.8, g=gd)
