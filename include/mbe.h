@@ -214,6 +214,10 @@ mbe_status mbe_kv_window_write(const void* k_win, const void* v_win, void* k_cac
  * MBE_DEVERR_* bits. */
 mbe_status mbe_get_device_error(cudaStream_t stream, uint32_t* flags_or_null);
 
+/* Host-thread-local description of the last CUDA runtime failure the library
+ * saw (the call site, the error name and message); useful after MBE_ERR_CUDA. */
+const char* mbe_last_error_string(void);
+
 /* Static description of a status code. */
 const char* mbe_status_string(mbe_status status);
 

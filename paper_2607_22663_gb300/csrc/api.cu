@@ -1,5 +1,17 @@
-// Status strings, version and the device error word query of libmbe.
+// Status strings, version, the last CUDA error and the device error word query of libmbe.
+#include <cstdio>
 #include "common.cuh"
+
+namespace mbe {
+namespace {
+thread_local char g_last_error[256] = "no CUDA error recorded";
+}
+void record_cuda_error(cudaError_t e, const char* where) {
+  snprintf(g_last_error, sizeof(g_last_error), "%s: %s (%s)", where, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+}  // namespace mbe
+
+extern "C" const char* mbe_last_error_string(void) { return mbe::g_last_error; }
 
 extern "C" mbe_status mbe_get_device_error(cudaStream_t stream, uint32_t* flags_or_null) {
   if (cudaStreamSynchronize(stream) != cudaSuccess) return MBE_ERR_CUDA;

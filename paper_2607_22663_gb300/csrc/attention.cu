@@ -881,14 +881,17 @@ mbe_status run(const void* q, const void* k_win, const void* v_win, const void* 
     if (!encode(&tkc, k_cache, 4, dims, strides, box) || !encode(&tvc, v_cache, 4, dims, strides, box))
       return MBE_ERR_CUDA;
   }
-  if (!ensure_smem_attr<D>(di)) return MBE_ERR_CUDA;
+  if (!ensure_smem_attr<D>(di)) {
+    record_cuda_error(cudaGetLastError(), "cudaFuncSetAttribute(attn_kernel)");
+    return MBE_ERR_CUDA;
+  }
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   Header* hdr = reinterpret_cast<Header*>(ws);
   SchedParams sp{prefix_len, window_len, mask_mode, cu_window, batch, G, Hkv, block_size, max_window, max_prefix,
                  di->num_sms, total_q_tokens, hdr, reinterpret_cast<WorkUnit*>(ws + L.units_tmp), reinterpret_cast<WorkUnit*>(ws + L.units),
                  reinterpret_cast<MergeGroup*>(ws + L.groups), L.max_units, L.max_groups, L.max_slots};
   attn_schedule_kernel<<<1, kBuckets, 0, stream>>>(sp);
-  if (cudaGetLastError() != cudaSuccess) return MBE_ERR_CUDA;
+  if (launch_status("attn_schedule_kernel launch") != MBE_OK) return MBE_ERR_CUDA;
   AttnParams ap;
   ap.block_table = block_table;
   ap.cu_window = cu_window;
@@ -908,11 +911,11 @@ mbe_status run(const void* q, const void* k_win, const void* v_win, const void* 
   ap.loads_per_tile = kTileKeys / box_rows;
   ap.scale_log2 = scale * 1.4426950408889634f;
   attn_kernel<D><<<di->num_sms, kThreads, Smem<D>::kBytes, stream>>>(tq, tkw, tvw, tkc, tvc, ap);
-  if (cudaGetLastError() != cudaSuccess) return MBE_ERR_CUDA;
+  if (launch_status("attn_kernel launch") != MBE_OK) return MBE_ERR_CUDA;
   MergeParams mp{hdr, reinterpret_cast<const MergeGroup*>(ws + L.groups), ap.part_o, ap.part_lse, cu_window,
                  ap.out, lse, Hq, G};
   attn_merge_kernel<D><<<static_cast<unsigned>(L.max_groups), kUnitRows, 0, stream>>>(mp);
-  if (cudaGetLastError() != cudaSuccess) return MBE_ERR_CUDA;
+  if (launch_status("attn_merge_kernel launch") != MBE_OK) return MBE_ERR_CUDA;
   return MBE_OK;
 }
 

@@ -23,9 +23,14 @@ uint32_t attention_take_error();
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-inline mbe_status launch_status() {
+// Remembers (per host thread) the last CUDA failure seen by the library.
+void record_cuda_error(cudaError_t e, const char* where);
+
+inline mbe_status launch_status(const char* where = "kernel launch") {
   cudaError_t e = cudaGetLastError();
-  return e == cudaSuccess ? MBE_OK : MBE_ERR_CUDA;
+  if (e == cudaSuccess) return MBE_OK;
+  record_cuda_error(e, where);
+  return MBE_ERR_CUDA;
 }
 
 }  // namespace mbe

@@ -29,7 +29,13 @@ _lib = None
 class MbeError(RuntimeError):
     def __init__(self, fn, status):
         self.status = status
-        super().__init__(f"{fn} failed: {STATUS_NAMES.get(status, status)} ({_status_string(status)})")
+        detail = ""
+        if status == 3:
+            try:
+                detail = "; " + lib().mbe_last_error_string().decode()
+            except Exception:
+                pass
+        super().__init__(f"{fn} failed: {STATUS_NAMES.get(status, status)} ({_status_string(status)}{detail})")
 
 
 def _status_string(status):
@@ -67,6 +73,8 @@ def lib(build_if_missing: bool = True):
     L.mbe_get_device_error.argtypes = [P, ctypes.POINTER(ctypes.c_uint32)]
     L.mbe_status_string.restype = ctypes.c_char_p
     L.mbe_status_string.argtypes = [ctypes.c_int]
+    L.mbe_last_error_string.restype = ctypes.c_char_p
+    L.mbe_last_error_string.argtypes = []
     L.mbe_version.restype = i32
     L.mbe_version.argtypes = []
     _lib = L
