@@ -68,6 +68,27 @@ def edit_bytes(rows, vocab, elem):
     return rows * vocab * elem + rows * (4 + 4 + 1 + 4)
 
 
+# ------------------------------------------------------------------ measured traffic
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum, one-pass ncu counters)
+# of one attention call (attn_kernel + merge) on the full-size workload, keyed by
+# the first 16 hex digits of the SHA-256 of the kernel source that was measured;
+# a changed kernel gets no traffic figure until it is measured again. Source:
+# profiles/attn_dram_serving128.md.
+MEASURED_TRAFFIC = {
+    "fa00c3dfb283c68d": {"serving128": 4442133248 + 60110336 + 16384},
+}
+
+
+def measured_traffic(workload):
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "paper_2607_22663_gb300", "csrc", "attention.cu"), "rb") as f:
+            h = hashlib.sha256(f.read()).hexdigest()[:16]
+    except OSError:
+        return None
+    return MEASURED_TRAFFIC.get(h, {}).get(workload)
+
+
 # ------------------------------------------------------------------ ranks
 def max_over_ranks(x: float, device="cpu") -> float:
     """Maximum of a per-rank scalar over all ranks (identity on one rank)."""
@@ -183,11 +204,16 @@ def run_gpu(args, rank, world):
         mask_t = torch.empty(R, dtype=torch.uint8, device=dev)
         conf_t = torch.empty(R, dtype=torch.float32, device=dev)
 
+    plan_layers = len(set(id(a.prefix_len) for a in attn)) == 1  # every call shares the lengths: one plan per pass
+
     def attention_call(i, a, q=None, kw=None, vw=None):
-        mbe.window_attention(a.q if q is None else q, a.k_win if kw is None else kw, a.v_win if vw is None else vw,
-                             a.k_cache, a.v_cache, a.block_table, a.prefix_len, a.window_len, a.cu_window,
-                             a.mask_mode, block_size=a.block_size, max_window=a.max_window, max_prefix=a.max_prefix,
-                             out=outs[i], workspace=wss[i])
+        # the first call of a pass plans (mbe_window_attention = plan + run); the
+        # other layers reuse that work list
+        fn = mbe.window_attention if (i == 0 or not plan_layers) else mbe.window_attention_run
+        fn(a.q if q is None else q, a.k_win if kw is None else kw, a.v_win if vw is None else vw,
+           a.k_cache, a.v_cache, a.block_table, a.prefix_len, a.window_len, a.cu_window,
+           a.mask_mode, block_size=a.block_size, max_window=a.max_window, max_prefix=a.max_prefix,
+           out=outs[i], workspace=wss[i])
 
     def edit_call(logits=None, committed=None):
         mbe.edit_decide(ep.logits if logits is None else logits, ep.committed if committed is None else committed,
@@ -268,11 +294,12 @@ def run_gpu(args, rank, world):
                               "ms": round(edit_ms, 4), "bytes": eb,
                               "edit_rate": round(float(mask_t.float().mean().item()), 5)}
     res["roofline"] = {"bound": "hbm", "achieved": round(attn_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                       "frac": round(attn_gbs / peaks["hbm_gbs"], 4), "traffic": None,
-                       "kernel": "mbe_window_attention (schedule + attn_kernel + merge)",
+                       "frac": round(attn_gbs / peaks["hbm_gbs"], 4), "traffic": measured_traffic(args.workload),
+                       "kernel": "mbe_window_attention per layer (attn_kernel + split merge; one plan per pass)",
                        "peak_source": f"{peak_src} hbm_gbs"}
     res["clocks"] = clocks
-    per_step = len(attn) * 3 + (1 if ep is not None else 0) + (len(attn) if with_kv_write else 0)
+    per_step = len(attn) * 2 + (1 if plan_layers else len(attn)) + (1 if ep is not None else 0) + \
+        (len(attn) if with_kv_write else 0)
     res["gpu_launches"] = per_step * K
     res["e2e"] = run_e2e(args, w, attention_call, edit_call, dev, stream, world, new_t if ep is not None else None,
                          mask_t if ep is not None else None, conf_t if ep is not None else None)

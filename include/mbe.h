@@ -119,6 +119,37 @@ mbe_status mbe_window_attention(const void* q, const void* k_win, const void* v_
                                 size_t workspace_bytes, cudaStream_t stream);
 
 /*
+ * mbe_window_attention_plan / mbe_window_attention_run -- the same attention as
+ * mbe_window_attention, split so that one work list serves many calls.
+ * Paper: Sec. 4.3 (an editing pass runs every layer over the same window
+ * shapes); Eq. 5 and Sec. 2.2 as for mbe_window_attention.
+ *
+ * mbe_window_attention = plan + run. The plan (a device-side work list built
+ * from prefix_len, window_len, cu_window, mask_mode and the bounds) is written
+ * into `workspace`; every later run with the same workspace, the same
+ * per-sequence lengths and modes, the same batch, heads, head_dim, block_size
+ * and bounds reuses it, so the layers of one pass pay for one plan. Q/K/V,
+ * cache, block table, scale and outputs may differ between runs. Runs that
+ * share a workspace must be ordered on the GPU (one stream). Arguments,
+ * layouts and errors are those of mbe_window_attention; a run after a plan
+ * made for other lengths computes garbage (the lengths are device data the
+ * host cannot compare).
+ */
+mbe_status mbe_window_attention_plan(const int32_t* prefix_len, const int32_t* window_len, const int32_t* cu_window,
+                                     const uint8_t* mask_mode, int32_t batch, int32_t total_q_tokens,
+                                     int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim, int32_t block_size,
+                                     int32_t max_window, int32_t max_prefix, void* workspace, size_t workspace_bytes,
+                                     cudaStream_t stream);
+mbe_status mbe_window_attention_run(const void* q, const void* k_win, const void* v_win, const void* k_cache,
+                                    const void* v_cache, int32_t num_pages, const int32_t* block_table,
+                                    int32_t max_pages_per_seq, const int32_t* prefix_len, const int32_t* window_len,
+                                    const int32_t* cu_window, const uint8_t* mask_mode, int32_t batch,
+                                    int32_t total_q_tokens, int32_t num_q_heads, int32_t num_kv_heads,
+                                    int32_t head_dim, int32_t block_size, int32_t page_size, int32_t max_window,
+                                    int32_t max_prefix, float softmax_scale, void* out, float* lse_or_null,
+                                    void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/*
  * mbe_window_attention_noalloc -- mbe_window_attention for callers that cannot
  * allocate device memory. The paper has no counterpart: this is an interface
  * convenience of this library, not a step of the method.

@@ -44,7 +44,7 @@ constexpr int kTileRows = 128;      // packed query rows per tile (= TMEM lanes)
 constexpr int kUnitRows = 256;      // packed query rows per work unit (two tiles)
 constexpr int kThreads = 384;       // 12 warps
 constexpr int kMinChunk = 8;        // fewest key tiles in a split piece
-constexpr int kSplitFactor = 4;     // target pieces per SM when splitting
+constexpr int kSplitFactor = 2;     // target pieces per SM when splitting
 constexpr int kBuckets = 1024;      // counting-sort buckets for unit cost
 constexpr float kRescaleLog2 = 8.0f;  // rescale O only when the max grows by > 2^8
 constexpr uint32_t kTmemCols = 512;
@@ -728,7 +728,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // ------------------------------------------------------------------ split merge
 struct MergeParams {
-  const Header* hdr;
+  Header* hdr;
   const MergeGroup* groups;
   const float* part_o;
   const float* part_lse;
@@ -741,6 +741,9 @@ struct MergeParams {
 template <int D>
 __global__ void __launch_bounds__(kUnitRows) attn_merge_kernel(const MergeParams p) {
   const int gi = blockIdx.x;
+  // the attention kernel has finished: re-arm the work counter so that the same
+  // plan can serve the next run
+  if (gi == 0 && threadIdx.x == 0) p.hdr->counter = 0;
   if (gi >= p.hdr->n_groups) return;
   const MergeGroup grp = p.groups[gi];
   const int r = threadIdx.x;
@@ -856,7 +859,7 @@ mbe_status run(const void* q, const void* k_win, const void* v_win, const void* 
                const int32_t* window_len, const int32_t* cu_window, const uint8_t* mask_mode, int32_t batch,
                int32_t total_q_tokens, int32_t Hq, int32_t Hkv, int32_t block_size, int32_t page_size,
                int32_t max_window, int32_t max_prefix, float scale, void* out, float* lse, void* workspace,
-               const Layout& L, DeviceInfo* di, cudaStream_t stream) {
+               const Layout& L, DeviceInfo* di, bool with_plan, cudaStream_t stream) {
   const int G = Hq / Hkv;
   CUtensorMap tq, tkw, tvw, tkc, tvc;
   {
@@ -890,8 +893,10 @@ mbe_status run(const void* q, const void* k_win, const void* v_win, const void* 
   SchedParams sp{prefix_len, window_len, mask_mode, cu_window, batch, G, Hkv, block_size, max_window, max_prefix,
                  di->num_sms, total_q_tokens, hdr, reinterpret_cast<WorkUnit*>(ws + L.units_tmp), reinterpret_cast<WorkUnit*>(ws + L.units),
                  reinterpret_cast<MergeGroup*>(ws + L.groups), L.max_units, L.max_groups, L.max_slots};
-  attn_schedule_kernel<<<1, kBuckets, 0, stream>>>(sp);
-  if (launch_status("attn_schedule_kernel launch") != MBE_OK) return MBE_ERR_CUDA;
+  if (with_plan) {
+    attn_schedule_kernel<<<1, kBuckets, 0, stream>>>(sp);
+    if (launch_status("attn_schedule_kernel launch") != MBE_OK) return MBE_ERR_CUDA;
+  }
   AttnParams ap;
   ap.block_table = block_table;
   ap.cu_window = cu_window;
@@ -935,6 +940,71 @@ extern "C" size_t mbe_window_attention_workspace_size(int32_t batch, int32_t num
   return make_layout(batch, num_q_heads, num_kv_heads, head_dim, max_window, max_prefix, di->num_sms).total;
 }
 
+namespace {
+
+struct Checked {
+  Layout L;
+  DeviceInfo* di;
+  float scale;
+};
+
+// Host-side validation shared by the attention entry points; st == MBE_OK with
+// nothing_to_do set means the call is a no-op.
+mbe_status check_call(int32_t num_pages, int32_t max_pages_per_seq, int32_t batch, int32_t total_q_tokens,
+                      int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim, int32_t block_size,
+                      int32_t page_size, int32_t max_window, int32_t max_prefix, float softmax_scale,
+                      void* workspace, size_t workspace_bytes, bool pointers_ok, bool& nothing_to_do, Checked& c) {
+  nothing_to_do = false;
+  mbe_status st = check_shapes(batch, num_q_heads, num_kv_heads, head_dim, max_window, max_prefix);
+  if (st != MBE_OK) return st;
+  if (block_size < 1 || total_q_tokens < 0 || num_pages < 1 || max_pages_per_seq < 1) return MBE_ERR_INVALID_ARG;
+  if (!pow2(page_size) || page_size < 8) return MBE_ERR_UNSUPPORTED;
+  if (static_cast<int64_t>(max_pages_per_seq) * page_size < max_prefix) return MBE_ERR_INVALID_ARG;
+  if (!(softmax_scale >= 0.f) || std::isinf(softmax_scale)) return MBE_ERR_INVALID_ARG;
+  if (batch == 0 || total_q_tokens == 0 || max_window == 0) {
+    nothing_to_do = true;
+    return MBE_OK;
+  }
+  if (!pointers_ok) return MBE_ERR_INVALID_ARG;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return MBE_ERR_CUDA;
+  c.di = device_info(dev);
+  if (!c.di || c.di->num_sms <= 0) return MBE_ERR_CUDA;
+  c.L = make_layout(batch, num_q_heads, num_kv_heads, head_dim, max_window, max_prefix, c.di->num_sms);
+  if (!workspace || workspace_bytes < c.L.total || !aligned16(workspace)) return MBE_ERR_WORKSPACE;
+  if (c.L.max_groups > 0x7FFFFFFF) return MBE_ERR_UNSUPPORTED;
+  c.scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(head_dim));
+  return MBE_OK;
+}
+
+mbe_status attention_call(const void* q, const void* k_win, const void* v_win, const void* k_cache, const void* v_cache,
+                          int32_t num_pages, const int32_t* block_table, int32_t max_pages_per_seq,
+                          const int32_t* prefix_len, const int32_t* window_len, const int32_t* cu_window,
+                          const uint8_t* mask_mode, int32_t batch, int32_t total_q_tokens, int32_t num_q_heads,
+                          int32_t num_kv_heads, int32_t head_dim, int32_t block_size, int32_t page_size,
+                          int32_t max_window, int32_t max_prefix, float softmax_scale, void* out, float* lse_or_null,
+                          void* workspace, size_t workspace_bytes, bool with_plan, cudaStream_t stream) {
+  bool noop = false;
+  Checked c;
+  const bool pointers_ok = q && k_win && v_win && k_cache && v_cache && block_table && prefix_len && window_len &&
+                           cu_window && mask_mode && out && aligned16(q) && aligned16(k_win) && aligned16(v_win) &&
+                           aligned16(k_cache) && aligned16(v_cache) && aligned16(out);
+  mbe_status st = check_call(num_pages, max_pages_per_seq, batch, total_q_tokens, num_q_heads, num_kv_heads, head_dim,
+                             block_size, page_size, max_window, max_prefix, softmax_scale, workspace, workspace_bytes,
+                             pointers_ok, noop, c);
+  if (st != MBE_OK || noop) return st;
+  if (head_dim == 128)
+    return run<128>(q, k_win, v_win, k_cache, v_cache, num_pages, block_table, max_pages_per_seq, prefix_len,
+                    window_len, cu_window, mask_mode, batch, total_q_tokens, num_q_heads, num_kv_heads, block_size,
+                    page_size, max_window, max_prefix, c.scale, out, lse_or_null, workspace, c.L, c.di, with_plan,
+                    stream);
+  return run<64>(q, k_win, v_win, k_cache, v_cache, num_pages, block_table, max_pages_per_seq, prefix_len, window_len,
+                 cu_window, mask_mode, batch, total_q_tokens, num_q_heads, num_kv_heads, block_size, page_size,
+                 max_window, max_prefix, c.scale, out, lse_or_null, workspace, c.L, c.di, with_plan, stream);
+}
+
+}  // namespace
+
 extern "C" mbe_status mbe_window_attention(const void* q, const void* k_win, const void* v_win, const void* k_cache,
                                            const void* v_cache, int32_t num_pages, const int32_t* block_table,
                                            int32_t max_pages_per_seq, const int32_t* prefix_len,
@@ -944,34 +1014,49 @@ extern "C" mbe_status mbe_window_attention(const void* q, const void* k_win, con
                                            int32_t block_size, int32_t page_size, int32_t max_window,
                                            int32_t max_prefix, float softmax_scale, void* out, float* lse_or_null,
                                            void* workspace, size_t workspace_bytes, cudaStream_t stream) {
-  mbe_status st = check_shapes(batch, num_q_heads, num_kv_heads, head_dim, max_window, max_prefix);
-  if (st != MBE_OK) return st;
-  if (block_size < 1 || total_q_tokens < 0 || num_pages < 1 || max_pages_per_seq < 1) return MBE_ERR_INVALID_ARG;
-  if (!pow2(page_size) || page_size < 8) return MBE_ERR_UNSUPPORTED;
-  if (static_cast<int64_t>(max_pages_per_seq) * page_size < max_prefix) return MBE_ERR_INVALID_ARG;
-  if (!(softmax_scale >= 0.f) || std::isinf(softmax_scale)) return MBE_ERR_INVALID_ARG;
-  if (batch == 0 || total_q_tokens == 0 || max_window == 0) return MBE_OK;
-  if (!q || !k_win || !v_win || !k_cache || !v_cache || !block_table || !prefix_len || !window_len || !cu_window ||
-      !mask_mode || !out)
-    return MBE_ERR_INVALID_ARG;
-  if (!aligned16(q) || !aligned16(k_win) || !aligned16(v_win) || !aligned16(k_cache) || !aligned16(v_cache) ||
-      !aligned16(out))
-    return MBE_ERR_INVALID_ARG;
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return MBE_ERR_CUDA;
-  DeviceInfo* di = device_info(dev);
-  if (!di || di->num_sms <= 0) return MBE_ERR_CUDA;
-  const Layout L = make_layout(batch, num_q_heads, num_kv_heads, head_dim, max_window, max_prefix, di->num_sms);
-  if (!workspace || workspace_bytes < L.total || !aligned16(workspace)) return MBE_ERR_WORKSPACE;
-  if (L.max_groups > 0x7FFFFFFF) return MBE_ERR_UNSUPPORTED;
-  const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(head_dim));
-  if (head_dim == 128)
-    return run<128>(q, k_win, v_win, k_cache, v_cache, num_pages, block_table, max_pages_per_seq, prefix_len,
-                    window_len, cu_window, mask_mode, batch, total_q_tokens, num_q_heads, num_kv_heads, block_size,
-                    page_size, max_window, max_prefix, scale, out, lse_or_null, workspace, L, di, stream);
-  return run<64>(q, k_win, v_win, k_cache, v_cache, num_pages, block_table, max_pages_per_seq, prefix_len, window_len,
-                 cu_window, mask_mode, batch, total_q_tokens, num_q_heads, num_kv_heads, block_size, page_size,
-                 max_window, max_prefix, scale, out, lse_or_null, workspace, L, di, stream);
+  return attention_call(q, k_win, v_win, k_cache, v_cache, num_pages, block_table, max_pages_per_seq, prefix_len,
+                        window_len, cu_window, mask_mode, batch, total_q_tokens, num_q_heads, num_kv_heads, head_dim,
+                        block_size, page_size, max_window, max_prefix, softmax_scale, out, lse_or_null, workspace,
+                        workspace_bytes, true, stream);
+}
+
+extern "C" mbe_status mbe_window_attention_plan(const int32_t* prefix_len, const int32_t* window_len,
+                                                const int32_t* cu_window, const uint8_t* mask_mode, int32_t batch,
+                                                int32_t total_q_tokens, int32_t num_q_heads, int32_t num_kv_heads,
+                                                int32_t head_dim, int32_t block_size, int32_t max_window,
+                                                int32_t max_prefix, void* workspace, size_t workspace_bytes,
+                                                cudaStream_t stream) {
+  bool noop = false;
+  Checked c;
+  // page geometry does not enter the plan: pass a page size and table width that always validate
+  const bool pointers_ok = prefix_len && window_len && cu_window && mask_mode;
+  mbe_status st = check_call(1, max_prefix > 0 ? max_prefix : 1, batch, total_q_tokens, num_q_heads, num_kv_heads,
+                             head_dim, block_size, 8, max_window, max_prefix, 0.f, workspace, workspace_bytes,
+                             pointers_ok, noop, c);
+  if (st != MBE_OK || noop) return st;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  SchedParams sp{prefix_len, window_len, mask_mode, cu_window, batch, num_q_heads / num_kv_heads, num_kv_heads,
+                 block_size, max_window, max_prefix, c.di->num_sms, total_q_tokens, reinterpret_cast<Header*>(ws),
+                 reinterpret_cast<WorkUnit*>(ws + c.L.units_tmp), reinterpret_cast<WorkUnit*>(ws + c.L.units),
+                 reinterpret_cast<MergeGroup*>(ws + c.L.groups), c.L.max_units, c.L.max_groups, c.L.max_slots};
+  attn_schedule_kernel<<<1, kBuckets, 0, stream>>>(sp);
+  return launch_status("attn_schedule_kernel launch");
+}
+
+extern "C" mbe_status mbe_window_attention_run(const void* q, const void* k_win, const void* v_win,
+                                               const void* k_cache, const void* v_cache, int32_t num_pages,
+                                               const int32_t* block_table, int32_t max_pages_per_seq,
+                                               const int32_t* prefix_len, const int32_t* window_len,
+                                               const int32_t* cu_window, const uint8_t* mask_mode, int32_t batch,
+                                               int32_t total_q_tokens, int32_t num_q_heads, int32_t num_kv_heads,
+                                               int32_t head_dim, int32_t block_size, int32_t page_size,
+                                               int32_t max_window, int32_t max_prefix, float softmax_scale, void* out,
+                                               float* lse_or_null, void* workspace, size_t workspace_bytes,
+                                               cudaStream_t stream) {
+  return attention_call(q, k_win, v_win, k_cache, v_cache, num_pages, block_table, max_pages_per_seq, prefix_len,
+                        window_len, cu_window, mask_mode, batch, total_q_tokens, num_q_heads, num_kv_heads, head_dim,
+                        block_size, page_size, max_window, max_prefix, softmax_scale, out, lse_or_null, workspace,
+                        workspace_bytes, false, stream);
 }
 
 // ------------------------------------------------------------------ no-allocation variant

@@ -60,6 +60,10 @@ def lib(build_if_missing: bool = True):
     L.mbe_window_attention.restype = ctypes.c_int
     L.mbe_window_attention.argtypes = [P, P, P, P, P, i32, P, i32, P, P, P, P, i32, i32, i32, i32, i32, i32, i32, i32,
                                        i32, f32, P, P, P, sz, P]
+    L.mbe_window_attention_run.restype = ctypes.c_int
+    L.mbe_window_attention_run.argtypes = list(L.mbe_window_attention.argtypes)
+    L.mbe_window_attention_plan.restype = ctypes.c_int
+    L.mbe_window_attention_plan.argtypes = [P, P, P, P, i32, i32, i32, i32, i32, i32, i32, i32, P, sz, P]
     L.mbe_window_attention_noalloc.restype = ctypes.c_int
     L.mbe_window_attention_noalloc.argtypes = [P, P, P, P, P, i32, P, i32, P, P, P, P, i32, i32, i32, i32, i32, i32,
                                                i32, i32, i32, f32, P, P, P]
@@ -117,10 +121,9 @@ def window_attention_workspace_size(batch, num_q_heads, num_kv_heads, head_dim, 
                                                          max_prefix))
 
 
-def window_attention(q, k_win, v_win, k_cache, v_cache, block_table, prefix_len, window_len, cu_window, mask_mode, *,
-                     block_size, max_window, max_prefix, softmax_scale=0.0, out=None, lse=None, return_lse=False,
-                     workspace=None, stream=None):
-    """mbe_window_attention: see include/mbe.h. Returns out (and lse if requested)."""
+def _attention(fn_name, q, k_win, v_win, k_cache, v_cache, block_table, prefix_len, window_len, cu_window, mask_mode, *,
+               block_size, max_window, max_prefix, softmax_scale=0.0, out=None, lse=None, return_lse=False,
+               workspace=None, stream=None):
     for t, n in ((q, "q"), (k_win, "k_win"), (v_win, "v_win"), (k_cache, "k_cache"), (v_cache, "v_cache")):
         _need(t, n, torch.bfloat16)
     for t, n in ((block_table, "block_table"), (prefix_len, "prefix_len"), (window_len, "window_len"),
@@ -141,14 +144,43 @@ def window_attention(q, k_win, v_win, k_cache, v_cache, block_table, prefix_len,
         _need(lse, "lse", torch.float32)
     need = window_attention_workspace_size(batch, Hq, Hkv, D, max_window, max_prefix)
     if workspace is None or workspace.numel() < need:
+        if fn_name == "mbe_window_attention_run":
+            raise ValueError("mbe_window_attention_run needs the workspace its plan was written into")
         workspace = torch.empty(max(need, 1), dtype=torch.uint8, device=q.device)
-    st = lib().mbe_window_attention(_ptr(q), _ptr(k_win), _ptr(v_win), _ptr(k_cache), _ptr(v_cache), num_pages,
-                                    _ptr(block_table), max_pages, _ptr(prefix_len), _ptr(window_len), _ptr(cu_window),
-                                    _ptr(mask_mode), batch, T, Hq, Hkv, D, block_size, page_size, max_window,
-                                    max_prefix, float(softmax_scale), _ptr(out), _ptr(lse), _ptr(workspace),
-                                    workspace.numel(), _stream(stream))
-    _check("mbe_window_attention", st)
+    st = getattr(lib(), fn_name)(_ptr(q), _ptr(k_win), _ptr(v_win), _ptr(k_cache), _ptr(v_cache), num_pages,
+                                 _ptr(block_table), max_pages, _ptr(prefix_len), _ptr(window_len), _ptr(cu_window),
+                                 _ptr(mask_mode), batch, T, Hq, Hkv, D, block_size, page_size, max_window,
+                                 max_prefix, float(softmax_scale), _ptr(out), _ptr(lse), _ptr(workspace),
+                                 workspace.numel(), _stream(stream))
+    _check(fn_name, st)
     return (out, lse) if return_lse else out
+
+
+def window_attention(q, k_win, v_win, k_cache, v_cache, block_table, prefix_len, window_len, cu_window, mask_mode,
+                     **kw):
+    """mbe_window_attention: see include/mbe.h. Returns out (and lse if requested)."""
+    return _attention("mbe_window_attention", q, k_win, v_win, k_cache, v_cache, block_table, prefix_len,
+                      window_len, cu_window, mask_mode, **kw)
+
+
+def window_attention_plan(prefix_len, window_len, cu_window, mask_mode, *, total_q_tokens, num_q_heads, num_kv_heads,
+                          head_dim, block_size, max_window, max_prefix, workspace, stream=None):
+    """mbe_window_attention_plan: writes the work list for these lengths into `workspace`."""
+    for t, n in ((prefix_len, "prefix_len"), (window_len, "window_len"), (cu_window, "cu_window")):
+        _need(t, n, torch.int32)
+    _need(mask_mode, "mask_mode", torch.uint8)
+    batch = prefix_len.shape[0]
+    st = lib().mbe_window_attention_plan(_ptr(prefix_len), _ptr(window_len), _ptr(cu_window), _ptr(mask_mode), batch,
+                                         total_q_tokens, num_q_heads, num_kv_heads, head_dim, block_size, max_window,
+                                         max_prefix, _ptr(workspace), workspace.numel(), _stream(stream))
+    _check("mbe_window_attention_plan", st)
+
+
+def window_attention_run(q, k_win, v_win, k_cache, v_cache, block_table, prefix_len, window_len, cu_window, mask_mode,
+                         **kw):
+    """mbe_window_attention_run: the attention with the plan already in `workspace`."""
+    return _attention("mbe_window_attention_run", q, k_win, v_win, k_cache, v_cache, block_table, prefix_len,
+                      window_len, cu_window, mask_mode, **kw)
 
 
 def window_attention_noalloc(q, k_win, v_win, k_cache, v_cache, block_table, prefix_len, window_len, cu_window,

@@ -114,3 +114,13 @@ def test_workspace_size_rejects_bad_shapes():
     L = mbe.lib()
     assert L.mbe_window_attention_workspace_size(1, 6, 4, 128, 64, 64) == 0
     assert L.mbe_window_attention_workspace_size(1, 4, 1, 96, 64, 64) == 0
+
+
+def test_attention_plan_host_validation():
+    L = mbe.lib()
+    P = ctypes.c_void_p
+    f = L.mbe_window_attention_plan
+    # null length array; a zero batch is a no-op
+    assert f(None, P(16), P(16), P(16), 1, 64, 4, 1, 128, 32, 64, 64, P(16), 1 << 20, None) == 1
+    assert f(None, None, None, None, 0, 0, 4, 1, 128, 32, 64, 64, None, 0, None) == 0
+    assert f(P(16), P(16), P(16), P(16), 1, 64, 6, 4, 128, 32, 64, 64, P(16), 1 << 20, None) == 1   # heads

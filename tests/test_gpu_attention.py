@@ -187,3 +187,26 @@ def test_serving128_full_size_sampled():
         # include the longest and the shortest prefix
         seqs = sorted(set(seqs) | {int(np.argmax(prob.prefix_host)), int(np.argmin(prob.prefix_host))})
         compare_attention(prob, out, lse, seqs=seqs, heads=[0, 7, 13, 31])
+
+
+def test_plan_once_run_many_layers_equals_per_call():
+    """One plan serves several layers (different Q/K/V and caches, same
+    lengths); every run matches a full call bit for bit, and repeated runs on
+    the same plan give identical results."""
+    w = wl.serving128(DEV, layers=3, batch=16, vocab=8)
+    a0 = w["attn"][0]
+    kw = dict(block_size=a0.block_size, max_window=a0.max_window, max_prefix=a0.max_prefix)
+    need = mbe.window_attention_workspace_size(a0.batch, a0.num_q_heads, a0.num_kv_heads, a0.head_dim,
+                                               a0.max_window, a0.max_prefix)
+    ws = torch.empty(need, dtype=torch.uint8, device=DEV)
+    mbe.window_attention_plan(a0.prefix_len, a0.window_len, a0.cu_window, a0.mask_mode, total_q_tokens=a0.total_tokens,
+                              num_q_heads=a0.num_q_heads, num_kv_heads=a0.num_kv_heads, head_dim=a0.head_dim,
+                              workspace=ws, **kw)
+    for rep in range(2):
+        for a in w["attn"]:
+            args = (a.q, a.k_win, a.v_win, a.k_cache, a.v_cache, a.block_table, a.prefix_len, a.window_len,
+                    a.cu_window, a.mask_mode)
+            ref, ref_lse = mbe.window_attention(*args, return_lse=True, **kw)
+            out, lse = mbe.window_attention_run(*args, return_lse=True, workspace=ws, **kw)
+            assert torch.equal(out, ref) and torch.equal(lse, ref_lse)
+    assert mbe.get_device_error() == (0, 0)
