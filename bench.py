@@ -75,7 +75,7 @@ def edit_bytes(rows, vocab, elem):
 # a changed kernel gets no traffic figure until it is measured again. Source:
 # profiles/attn_dram_serving128.md.
 MEASURED_TRAFFIC = {
-    "fa00c3dfb283c68d": {"serving128": 4442133248 + 60110336 + 16384},
+    "2c6da1740a420c42": {"serving128": 4442437120 + 59812864 + 16896},
 }
 
 
@@ -204,7 +204,9 @@ def run_gpu(args, rank, world):
         mask_t = torch.empty(R, dtype=torch.uint8, device=dev)
         conf_t = torch.empty(R, dtype=torch.float32, device=dev)
 
-    plan_layers = len(set(id(a.prefix_len) for a in attn)) == 1  # every call shares the lengths: one plan per pass
+    # one plan per pass when every call shares the lengths, modes and bounds
+    plan_layers = len({(id(a.prefix_len), id(a.window_len), id(a.cu_window), id(a.mask_mode), a.max_window,
+                        a.max_prefix, a.total_tokens) for a in attn}) == 1
 
     def attention_call(i, a, q=None, kw=None, vw=None):
         # the first call of a pass plans (mbe_window_attention = plan + run); the

@@ -66,6 +66,7 @@ typedef enum { MBE_F32 = 0, MBE_BF16 = 1 } mbe_dtype;
 #define MBE_DEVERR_LENGTH 0x2u        /* prefix_len/window_len/mask_mode outside the declared range */
 #define MBE_DEVERR_PAGE 0x4u          /* a block_table entry outside [0, num_pages) */
 #define MBE_DEVERR_CAPACITY 0x8u      /* work list larger than the workspace was sized for */
+#define MBE_DEVERR_PLAN 0x10u         /* mbe_window_attention_run found no plan for its parameters in the workspace */
 
 /*
  * mbe_window_attention -- attention of one editing (or standard) pass.
@@ -131,9 +132,13 @@ mbe_status mbe_window_attention(const void* q, const void* k_win, const void* v_
  * and bounds reuses it, so the layers of one pass pay for one plan. Q/K/V,
  * cache, block table, scale and outputs may differ between runs. Runs that
  * share a workspace must be ordered on the GPU (one stream). Arguments,
- * layouts and errors are those of mbe_window_attention; a run after a plan
- * made for other lengths computes garbage (the lengths are device data the
- * host cannot compare).
+ * layouts and errors are those of mbe_window_attention. The plan records the
+ * parameters that fix its layout (batch, total_q_tokens, heads, head_dim,
+ * block_size, max_window, max_prefix); a run whose parameters differ, or a
+ * workspace holding no plan, computes nothing and sets MBE_DEVERR_PLAN. A run
+ * whose cu_window places a planned window outside q/out skips it and sets
+ * MBE_DEVERR_LENGTH. Changing the device-side lengths or modes without a new
+ * plan is not detected and gives wrong (but in-bounds) results.
  */
 mbe_status mbe_window_attention_plan(const int32_t* prefix_len, const int32_t* window_len, const int32_t* cu_window,
                                      const uint8_t* mask_mode, int32_t batch, int32_t total_q_tokens,

@@ -44,7 +44,9 @@ constexpr int kTileRows = 128;      // packed query rows per tile (= TMEM lanes)
 constexpr int kUnitRows = 256;      // packed query rows per work unit (two tiles)
 constexpr int kThreads = 384;       // 12 warps
 constexpr int kMinChunk = 8;        // fewest key tiles in a split piece
-constexpr int kSplitFactor = 2;     // target pieces per SM when splitting
+constexpr int kSplitFactor = 4;     // most pieces per SM when splitting (bounds the workspace)
+constexpr int kMaxGroupedSlabs = 8; // slabs of one (sequence, KV head) kept adjacent in the work list
+constexpr float kUnitStartTiles = 2.f;  // start-up cost of a work unit, in key tiles (scheduler estimate)
 constexpr int kBuckets = 1024;      // counting-sort buckets for unit cost
 constexpr float kRescaleLog2 = 8.0f;  // rescale O only when the max grows by > 2^8
 constexpr uint32_t kTmemCols = 512;
@@ -56,8 +58,28 @@ struct WorkUnit {
 struct MergeGroup {
   int32_t seq, kv_head, row0, n_splits, slot_base, window, pad0, pad1;
 };
+// Plan signature: the call parameters that fix the workspace layout and the
+// meaning of the work list. A run compares it with its own before using units.
+constexpr int kSigWords = 9;
+constexpr int32_t kPlanMagic = 0x4D424531;  // "MBE1"
+struct PlanSig {
+  int32_t w[kSigWords];
+};
+__host__ __device__ inline PlanSig make_sig(int batch, int total_tokens, int G, int Hkv, int D, int block_size,
+                                            int max_window, int max_prefix) {
+  return PlanSig{{kPlanMagic, batch, total_tokens, G, Hkv, D, block_size, max_window, max_prefix}};
+}
+__device__ inline bool sig_equal(const volatile int32_t* a, const PlanSig& b) {
+  bool eq = true;
+#pragma unroll
+  for (int i = 0; i < kSigWords; ++i) eq &= (a[i] == b.w[i]);
+  return eq;
+}
+
 struct Header {
-  int32_t counter, n_units, n_groups, pad[61];
+  int32_t counter, n_units, n_groups;
+  int32_t sig[kSigWords];
+  int32_t pad[64 - 3 - kSigWords];
 };
 static_assert(sizeof(Header) == 256, "header size");
 
@@ -94,6 +116,7 @@ struct SchedParams {
   const uint8_t* mask_mode;
   const int32_t* cu_window;
   int batch, G, Hkv, block_size, max_window, max_prefix, num_sms, total_tokens;
+  PlanSig sig;
   Header* hdr;
   WorkUnit* units_tmp;
   WorkUnit* units;
@@ -133,7 +156,7 @@ __global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p
   if (tid == 0) { s_total = 0; s_nunits = 0; s_ngroups = 0; s_nslots = 0; s_bad = 0; }
   for (int b = tid; b < kBuckets; b += blockDim.x) hist[b] = 0;
   __syncthreads();
-  // pass 1: validate and count key tiles
+  // pass 1: validate and count key tiles and (sequence, KV head) pairs
   int local = 0, bad = 0;
   for (int s = tid; s < p.batch; s += blockDim.x) {
     const int P = p.prefix_len[s], W = p.window_len[s], mode = p.mask_mode[s];
@@ -144,39 +167,106 @@ __global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p
   atomicAdd(&s_total, local);
   if (bad) atomicOr(&s_bad, 1);
   __syncthreads();
-  const int64_t target = static_cast<int64_t>(kSplitFactor) * p.num_sms;
-  const int chunk = max(kMinChunk, static_cast<int>((s_total + target - 1) / target));
-  // pass 2: emit units (unsorted) and merge groups
+  // Piece length: for each candidate (about 1..kSplitFactor pieces per SM)
+  // count the units it makes and estimate the makespan as
+  //   ceil(units / SMs) * (mean piece length + per-unit start-up cost),
+  // keeping the longest pieces among equal estimates (fewer split-KV partials).
+  __shared__ int s_units[kSplitFactor];
+  if (tid < kSplitFactor) s_units[tid] = 0;
+  __syncthreads();
+  int cand[kSplitFactor];
+#pragma unroll
+  for (int k = 0; k < kSplitFactor; ++k) {
+    const int64_t target = static_cast<int64_t>(k + 1) * p.num_sms;
+    cand[k] = max(kMinChunk, static_cast<int>((s_total + target - 1) / target));
+  }
+  {
+    int cnt[kSplitFactor] = {};
+    for (int s = tid; s < p.batch; s += blockDim.x) {
+      const int P = p.prefix_len[s], W = p.window_len[s], mode = p.mask_mode[s];
+      if (!seq_ok(p, s, P, W, mode)) continue;
+      const int slabs = (W * p.G + kUnitRows - 1) / kUnitRows;
+      for (int sl = 0; sl < slabs; ++sl) {
+        const int T = slab_tiles(P, W, mode, sl * kUnitRows, p.G, p.block_size);
+#pragma unroll
+        for (int k = 0; k < kSplitFactor; ++k) cnt[k] += p.Hkv * ((T + cand[k] - 1) / cand[k]);
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < kSplitFactor; ++k) atomicAdd(&s_units[k], cnt[k]);
+  }
+  __syncthreads();
+  int chunk = cand[0];
+  {
+    float best = 3.4e38f;
+#pragma unroll
+    for (int k = 0; k < kSplitFactor; ++k) {
+      const int U = max(1, s_units[k]);
+      const int waves = (U + p.num_sms - 1) / p.num_sms;
+      const float est = waves * (static_cast<float>(s_total) / U + kUnitStartTiles);
+      if (est < best * 0.98f) {  // a finer split must win clearly
+        best = est;
+        chunk = cand[k];
+      }
+    }
+  }
+  // pass 2: emit units (unsorted) and merge groups. The units of piece k of all
+  // slabs of one (sequence, KV head) are emitted together (a "piece"): they
+  // read the same K/V tiles, and the sort keeps them adjacent so that they run
+  // at the same time and share those tiles in L2. The first unit of a piece
+  // carries the piece's unit count and cost bucket in kv_head bits 16-19 / 20-29.
   bool overflow = false;
+  auto emit_piece = [&](const WorkUnit* u, int count, int cost) {
+    const int base = atomicAdd(&s_nunits, count);
+    if (base + count > p.max_units) {
+      overflow = true;
+      return;
+    }
+    const int b = cost_bucket(cost, chunk);
+    for (int i = 0; i < count; ++i) {
+      WorkUnit w = u[i];
+      if (i == 0) w.kv_head |= (count << 16) | (b << 20);
+      p.units_tmp[base + i] = w;
+    }
+    atomicAdd(&hist[b], count);
+  };
   for (int s = tid; s < p.batch; s += blockDim.x) {
     const int P = p.prefix_len[s], W = p.window_len[s], mode = p.mask_mode[s];
     if (!seq_ok(p, s, P, W, mode)) continue;
     const int slabs = (W * p.G + kUnitRows - 1) / kUnitRows;
-    for (int sl = 0; sl < slabs; ++sl) {
-      const int T = slab_tiles(P, W, mode, sl * kUnitRows, p.G, p.block_size);
-      const int n = (T + chunk - 1) / chunk;
-      for (int g = 0; g < p.Hkv; ++g) {
-        const int base = atomicAdd(&s_nunits, n);
-        int slot0 = -1;
-        if (n > 1) {
-          const int gi = atomicAdd(&s_ngroups, 1);
-          slot0 = atomicAdd(&s_nslots, n);
-          if (gi < p.max_groups && slot0 + n <= p.max_slots) {
-            p.groups[gi] = MergeGroup{s, g, sl * kUnitRows, n, slot0, W, 0, 0};
-          } else {
-            overflow = true;
+    const int ng = slabs <= kMaxGroupedSlabs ? slabs : 1;  // slabs per piece
+    for (int g = 0; g < p.Hkv; ++g) {
+      for (int s0 = 0; s0 < slabs; s0 += ng) {
+        const int cnt = min(ng, slabs - s0);
+        int T[kMaxGroupedSlabs], n[kMaxGroupedSlabs], slot0[kMaxGroupedSlabs];
+        int nmax = 0;
+        for (int i = 0; i < cnt; ++i) {
+          const int sl = s0 + i;
+          T[i] = slab_tiles(P, W, mode, sl * kUnitRows, p.G, p.block_size);
+          n[i] = (T[i] + chunk - 1) / chunk;
+          nmax = max(nmax, n[i]);
+          slot0[i] = -1;
+          if (n[i] > 1) {
+            const int gi = atomicAdd(&s_ngroups, 1);
+            slot0[i] = atomicAdd(&s_nslots, n[i]);
+            if (gi < p.max_groups && slot0[i] + n[i] <= p.max_slots) {
+              p.groups[gi] = MergeGroup{s, g, sl * kUnitRows, n[i], slot0[i], W, 0, 0};
+            } else {
+              overflow = true;
+            }
           }
         }
-        for (int k = 0; k < n; ++k) {
-          const int tb = static_cast<int>((static_cast<int64_t>(k) * T) / n);
-          const int te = static_cast<int>((static_cast<int64_t>(k + 1) * T) / n);
-          if (base + k < p.max_units) {
-            p.units_tmp[base + k] =
-                WorkUnit{s, g, sl * kUnitRows, tb, te, n > 1 ? slot0 + k : -1, P, W | (mode << 30)};
-            atomicAdd(&hist[cost_bucket(te - tb, chunk)], 1);
-          } else {
-            overflow = true;
+        for (int k = 0; k < nmax; ++k) {
+          WorkUnit u[kMaxGroupedSlabs];
+          int c = 0, cost = 1;
+          for (int i = 0; i < cnt; ++i) {
+            if (k >= n[i]) continue;
+            const int tb = static_cast<int>((static_cast<int64_t>(k) * T[i]) / n[i]);
+            const int te = static_cast<int>((static_cast<int64_t>(k + 1) * T[i]) / n[i]);
+            u[c++] = WorkUnit{s, g, (s0 + i) * kUnitRows, tb, te, n[i] > 1 ? slot0[i] + k : -1, P, W | (mode << 30)};
+            cost = max(cost, te - tb);
           }
+          if (c > 0) emit_piece(u, c, cost);
         }
       }
     }
@@ -214,13 +304,21 @@ __global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p
   const bool ok = (s_bad & 2) == 0;
   const int n_units = ok ? s_nunits : 0;
   for (int u = tid; u < n_units; u += blockDim.x) {
-    const WorkUnit wu = p.units_tmp[u];
-    const int pos = atomicAdd(&hist[cost_bucket(wu.tile_end - wu.tile_begin, chunk)], 1);
-    p.units[pos] = wu;
+    const WorkUnit head = p.units_tmp[u];
+    const int c = (head.kv_head >> 16) & 0xF;
+    if (c == 0) continue;  // not the first unit of a piece
+    const int pos = atomicAdd(&hist[(head.kv_head >> 20) & (kBuckets - 1)], c);
+    for (int i = 0; i < c; ++i) {
+      WorkUnit w = p.units_tmp[u + i];
+      w.kv_head &= 0xFFFF;
+      p.units[pos + i] = w;
+    }
   }
+  __syncthreads();
   if (tid == 0) {
     p.hdr->counter = 0;
     p.hdr->n_units = n_units;
+    for (int i = 0; i < kSigWords; ++i) p.hdr->sig[i] = p.sig.w[i];
     p.hdr->n_groups = ok ? s_ngroups : 0;
     if (s_bad & 1) atomicOr(&g_error_word, MBE_DEVERR_LENGTH);
     if (s_bad & 2) atomicOr(&g_error_word, MBE_DEVERR_CAPACITY);
@@ -229,6 +327,8 @@ __global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p
 
 // ------------------------------------------------------------------ main kernel
 struct AttnParams {
+  PlanSig sig;
+  int batch, total_tokens;
   const int32_t* block_table;
   const int32_t* cu_window;
   __nv_bfloat16* out;
@@ -318,7 +418,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tmem_base_s;
-  const int n_units = p.hdr->n_units;
+  // a work list planned for other parameters (or never planned) is not used
+  const bool plan_ok = sig_equal(p.hdr->sig, p.sig);
+  if (!plan_ok && blockIdx.x == 0 && tid == 0) atomicOr(&g_error_word, MBE_DEVERR_PLAN);
+  const int n_units = plan_ok ? p.hdr->n_units : 0;
 
   if (warp == 0) {
     // ---------------------------------------------------------------- producer
@@ -350,6 +453,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         wu.seq = -1;
       } else {
         wu = p.units[uidx];
+        const int W = wu.window_mode & 0x3FFFFFFF;
+        const bool sane = wu.seq >= 0 && wu.seq < p.batch && wu.kv_head >= 0 && wu.tile_begin >= 0 &&
+                          wu.tile_end > wu.tile_begin && W > 0;
+        const int cu = sane ? p.cu_window[wu.seq] : -1;
+        if (!sane || cu < 0 || static_cast<int64_t>(cu) + W > p.total_tokens) {
+          if (lane == 0) atomicOr(&g_error_word, MBE_DEVERR_LENGTH);
+          continue;  // skip this unit; every role only ever sees published units
+        }
       }
       if (lane == 0) {
         unit_ring[uslot] = wu;
@@ -728,6 +839,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // ------------------------------------------------------------------ split merge
 struct MergeParams {
+  PlanSig sig;
+  int batch, total_tokens;
   Header* hdr;
   const MergeGroup* groups;
   const float* part_o;
@@ -739,17 +852,12 @@ struct MergeParams {
 };
 
 template <int D>
-__global__ void __launch_bounds__(kUnitRows) attn_merge_kernel(const MergeParams p) {
-  const int gi = blockIdx.x;
-  // the attention kernel has finished: re-arm the work counter so that the same
-  // plan can serve the next run
-  if (gi == 0 && threadIdx.x == 0) p.hdr->counter = 0;
-  if (gi >= p.hdr->n_groups) return;
-  const MergeGroup grp = p.groups[gi];
-  const int r = threadIdx.x;
+__device__ __forceinline__ void merge_group_row(const MergeParams& p, const MergeGroup& grp, int r) {
   const int R = grp.row0 + r;
   const int qi = R / p.G, hh = R - qi * p.G;
   if (qi >= grp.window) return;
+  const int cu = p.cu_window[grp.seq];
+  if (cu < 0 || static_cast<int64_t>(cu) + grp.window > p.total_tokens) return;
   float M = neg_inf();
   for (int k = 0; k < grp.n_splits; ++k)
     M = fmaxf(M, p.part_lse[static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r]);
@@ -762,7 +870,8 @@ __global__ void __launch_bounds__(kUnitRows) attn_merge_kernel(const MergeParams
     const float w = (lk == neg_inf()) ? 0.f : ex2f(lk - M);
     if (w == 0.f) continue;
     wsum += w;
-    const float4* src = reinterpret_cast<const float4*>(p.part_o + (static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r) * D);
+    const float4* src =
+        reinterpret_cast<const float4*>(p.part_o + (static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r) * D);
 #pragma unroll
     for (int d4 = 0; d4 < D / 4; ++d4) {
       const float4 v = src[d4];
@@ -773,7 +882,6 @@ __global__ void __launch_bounds__(kUnitRows) attn_merge_kernel(const MergeParams
     }
   }
   const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
-  const int cu = p.cu_window[grp.seq];
   const int64_t orow = static_cast<int64_t>(cu + qi) * p.Hq + grp.kv_head * p.G + hh;
   uint4* dst = reinterpret_cast<uint4*>(p.out + orow * D);
 #pragma unroll
@@ -781,6 +889,22 @@ __global__ void __launch_bounds__(kUnitRows) attn_merge_kernel(const MergeParams
     dst[d / 8] = make_uint4(pack_bf16x2(acc[d] * inv, acc[d + 1] * inv), pack_bf16x2(acc[d + 2] * inv, acc[d + 3] * inv),
                             pack_bf16x2(acc[d + 4] * inv, acc[d + 5] * inv), pack_bf16x2(acc[d + 6] * inv, acc[d + 7] * inv));
   if (p.lse) p.lse[orow] = (wsum > 0.f ? M + __log2f(wsum) : neg_inf()) * 0.6931471805599453f;
+}
+
+// One CTA per split group (looping when there are more groups than CTAs),
+// one thread per packed query row.
+template <int D>
+__global__ void __launch_bounds__(kUnitRows) attn_merge_kernel(const MergeParams p) {
+  // the attention kernel has finished: re-arm the work counter so that the same
+  // plan can serve the next run
+  if (blockIdx.x == 0 && threadIdx.x == 0) p.hdr->counter = 0;
+  if (!sig_equal(p.hdr->sig, p.sig)) return;
+  const int n_groups = p.hdr->n_groups;
+  for (int gi = blockIdx.x; gi < n_groups; gi += gridDim.x) {
+    const MergeGroup grp = p.groups[gi];
+    if (grp.seq < 0 || grp.seq >= p.batch) continue;
+    merge_group_row<D>(p, grp, threadIdx.x);
+  }
 }
 
 // ------------------------------------------------------------------ host side
@@ -848,7 +972,7 @@ mbe_status check_shapes(int32_t batch, int32_t Hq, int32_t Hkv, int32_t D, int32
   if (Hq % Hkv != 0) return MBE_ERR_INVALID_ARG;
   if (D != 64 && D != 128) return MBE_ERR_UNSUPPORTED;
   const int G = Hq / Hkv;
-  if (!pow2(G) || G > kTileRows) return MBE_ERR_UNSUPPORTED;
+  if (!pow2(G) || G > kTileRows || Hkv > 0xFFFF) return MBE_ERR_UNSUPPORTED;
   if (max_window > (1 << 20) || max_prefix > (1 << 28)) return MBE_ERR_UNSUPPORTED;
   return MBE_OK;
 }
@@ -890,14 +1014,18 @@ mbe_status run(const void* q, const void* k_win, const void* v_win, const void* 
   }
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   Header* hdr = reinterpret_cast<Header*>(ws);
+  const PlanSig sig = make_sig(batch, total_q_tokens, G, Hkv, D, block_size, max_window, max_prefix);
   SchedParams sp{prefix_len, window_len, mask_mode, cu_window, batch, G, Hkv, block_size, max_window, max_prefix,
-                 di->num_sms, total_q_tokens, hdr, reinterpret_cast<WorkUnit*>(ws + L.units_tmp), reinterpret_cast<WorkUnit*>(ws + L.units),
+                 di->num_sms, total_q_tokens, sig, hdr, reinterpret_cast<WorkUnit*>(ws + L.units_tmp), reinterpret_cast<WorkUnit*>(ws + L.units),
                  reinterpret_cast<MergeGroup*>(ws + L.groups), L.max_units, L.max_groups, L.max_slots};
   if (with_plan) {
     attn_schedule_kernel<<<1, kBuckets, 0, stream>>>(sp);
     if (launch_status("attn_schedule_kernel launch") != MBE_OK) return MBE_ERR_CUDA;
   }
   AttnParams ap;
+  ap.sig = sig;
+  ap.batch = batch;
+  ap.total_tokens = total_q_tokens;
   ap.block_table = block_table;
   ap.cu_window = cu_window;
   ap.out = static_cast<__nv_bfloat16*>(out);
@@ -917,9 +1045,10 @@ mbe_status run(const void* q, const void* k_win, const void* v_win, const void* 
   ap.scale_log2 = scale * 1.4426950408889634f;
   attn_kernel<D><<<di->num_sms, kThreads, Smem<D>::kBytes, stream>>>(tq, tkw, tvw, tkc, tvc, ap);
   if (launch_status("attn_kernel launch") != MBE_OK) return MBE_ERR_CUDA;
-  MergeParams mp{hdr, reinterpret_cast<const MergeGroup*>(ws + L.groups), ap.part_o, ap.part_lse, cu_window,
-                 ap.out, lse, Hq, G};
-  attn_merge_kernel<D><<<static_cast<unsigned>(L.max_groups), kUnitRows, 0, stream>>>(mp);
+  MergeParams mp{sig, batch, total_q_tokens, hdr, reinterpret_cast<const MergeGroup*>(ws + L.groups), ap.part_o,
+                 ap.part_lse, cu_window, ap.out, lse, Hq, G};
+  const int64_t merge_grid = std::min<int64_t>(L.max_groups, 2 * di->num_sms);
+  attn_merge_kernel<D><<<static_cast<unsigned>(merge_grid), kUnitRows, 0, stream>>>(mp);
   if (launch_status("attn_merge_kernel launch") != MBE_OK) return MBE_ERR_CUDA;
   return MBE_OK;
 }
@@ -1035,8 +1164,10 @@ extern "C" mbe_status mbe_window_attention_plan(const int32_t* prefix_len, const
                              pointers_ok, noop, c);
   if (st != MBE_OK || noop) return st;
   uint8_t* ws = static_cast<uint8_t*>(workspace);
+  const PlanSig sig = make_sig(batch, total_q_tokens, num_q_heads / num_kv_heads, num_kv_heads, head_dim, block_size,
+                               max_window, max_prefix);
   SchedParams sp{prefix_len, window_len, mask_mode, cu_window, batch, num_q_heads / num_kv_heads, num_kv_heads,
-                 block_size, max_window, max_prefix, c.di->num_sms, total_q_tokens, reinterpret_cast<Header*>(ws),
+                 block_size, max_window, max_prefix, c.di->num_sms, total_q_tokens, sig, reinterpret_cast<Header*>(ws),
                  reinterpret_cast<WorkUnit*>(ws + c.L.units_tmp), reinterpret_cast<WorkUnit*>(ws + c.L.units),
                  reinterpret_cast<MergeGroup*>(ws + c.L.groups), c.L.max_units, c.L.max_groups, c.L.max_slots};
   attn_schedule_kernel<<<1, kBuckets, 0, stream>>>(sp);

@@ -19,7 +19,7 @@ from . import build as _build
 MBE_OK = 0
 STATUS_NAMES = {0: "MBE_OK", 1: "MBE_ERR_INVALID_ARG", 2: "MBE_ERR_UNSUPPORTED", 3: "MBE_ERR_CUDA",
                 4: "MBE_ERR_TIMEOUT", 5: "MBE_ERR_WORKSPACE", 6: "MBE_ERR_DEVICE_CHECK"}
-DEVERR_TIMEOUT, DEVERR_LENGTH, DEVERR_PAGE, DEVERR_CAPACITY = 0x1, 0x2, 0x4, 0x8
+DEVERR_TIMEOUT, DEVERR_LENGTH, DEVERR_PAGE, DEVERR_CAPACITY, DEVERR_PLAN = 0x1, 0x2, 0x4, 0x8, 0x10
 BLOCK_CAUSAL, MULTI_BLOCK_BIDIRECTIONAL = 0, 1
 HEADER = _build.INCLUDE / "mbe.h"
 

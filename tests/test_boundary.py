@@ -32,7 +32,8 @@ def test_header_enums_match_binding():
         assert re.search(rf"\b{name}\s*=\s*{val}\b", text), name
         assert mbe.STATUS_NAMES[val] == name
     for name, val in (("MBE_DEVERR_TIMEOUT", mbe.DEVERR_TIMEOUT), ("MBE_DEVERR_LENGTH", mbe.DEVERR_LENGTH),
-                      ("MBE_DEVERR_PAGE", mbe.DEVERR_PAGE), ("MBE_DEVERR_CAPACITY", mbe.DEVERR_CAPACITY)):
+                      ("MBE_DEVERR_PAGE", mbe.DEVERR_PAGE), ("MBE_DEVERR_CAPACITY", mbe.DEVERR_CAPACITY),
+                      ("MBE_DEVERR_PLAN", mbe.DEVERR_PLAN)):
         m = re.search(rf"#define {name} (0x[0-9a-fA-F]+)u", text)
         assert m and int(m.group(1), 16) == val, name
 

@@ -210,3 +210,33 @@ def test_plan_once_run_many_layers_equals_per_call():
             out, lse = mbe.window_attention_run(*args, return_lse=True, workspace=ws, **kw)
             assert torch.equal(out, ref) and torch.equal(lse, ref_lse)
     assert mbe.get_device_error() == (0, 0)
+
+
+def test_run_without_matching_plan_sets_flag_and_writes_nothing():
+    """A run whose bounds differ from the plan's (a different workspace layout),
+    or a run on a workspace that holds no plan, must compute nothing and set
+    MBE_DEVERR_PLAN instead of reading the workspace as a work list."""
+    prob = attention_problem([300, 200], [64, 64], [BIDIRECTIONAL, BIDIRECTIONAL], 8, 2, 128, 32, 32, seed=3,
+                             device=DEV)
+    args = (prob.q, prob.k_win, prob.v_win, prob.k_cache, prob.v_cache, prob.block_table, prob.prefix_len,
+            prob.window_len, prob.cu_window, prob.mask_mode)
+    need = mbe.window_attention_workspace_size(2, 8, 2, 128, 128, 300)
+    ws = torch.zeros(need, dtype=torch.uint8, device=DEV)
+    mbe.window_attention_plan(prob.prefix_len, prob.window_len, prob.cu_window, prob.mask_mode,
+                              total_q_tokens=prob.total_tokens, num_q_heads=8, num_kv_heads=2, head_dim=128,
+                              block_size=32, max_window=64, max_prefix=300, workspace=ws)
+    out = torch.full_like(prob.q, 7.0)
+    mbe.window_attention_run(*args, block_size=32, max_window=128, max_prefix=300, out=out, workspace=ws)
+    st, flags = mbe.get_device_error()
+    assert st == 6 and flags & mbe.DEVERR_PLAN
+    assert torch.all(out == 7.0)
+    fresh = torch.zeros(need, dtype=torch.uint8, device=DEV)
+    mbe.window_attention_run(*args, block_size=32, max_window=64, max_prefix=300, out=out, workspace=fresh)
+    st, flags = mbe.get_device_error()
+    assert st == 6 and flags & mbe.DEVERR_PLAN
+    assert torch.all(out == 7.0)
+    # the matching run on the planned workspace works
+    ref = mbe.window_attention(*args, block_size=32, max_window=64, max_prefix=300)
+    mbe.window_attention_run(*args, block_size=32, max_window=64, max_prefix=300, out=out, workspace=ws)
+    assert torch.equal(out, ref)
+    assert mbe.get_device_error() == (0, 0)
