@@ -9,6 +9,9 @@ path computes, written from the paper (arXiv 2607.22663):
   threshold-and-replace).
 * ``kv_window_write``   -- Sec. 4.3 targeted refresh: window K/V written to
   the paged cache at positions [P, P+W).
+* ``denoise_update``    -- the full Eq. 2 step (M2T set Gamma_t with forced
+  unmasking, T2T set Delta_t), per-row entropies, changed-block flags.
+* ``tail_entropy_select`` -- Eqs. 6-7 tail-entropy scores and window start.
 
 Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
 ``bench.py`` may import it. It shares no code with the CUDA library and never
@@ -61,6 +64,11 @@ def _load():
                                                 i32, f64, i32, P, P, P, P]
         lib.oracle_edit_decide.restype = ctypes.c_int
         lib.oracle_edit_decide.argtypes = [P, i32, i64, i32, i32, P, P, f32, P, i32, P, P, P, P, P]
+        lib.oracle_denoise_update.restype = ctypes.c_int
+        lib.oracle_denoise_update.argtypes = [P, i32, i64, i32, P, i32, i32, i32, P, i32, f32, f32, P, P, P, P, P, P,
+                                              P, P]
+        lib.oracle_tail_entropy_select.restype = ctypes.c_int
+        lib.oracle_tail_entropy_select.argtypes = [P, P, i32, i32, i32, f64, i32, P, P, P]
         lib.oracle_kv_window_write.restype = ctypes.c_int
         lib.oracle_kv_window_write.argtypes = [P, P, P, P, P, i32, P, P, P, P, i32, i32, i32, i32, i32, i32, i32]
         _lib = lib
@@ -148,6 +156,46 @@ def edit_decide(logits, committed, tau=0.0, tau_per_row=None, editable=None, row
                                 _ptr(am))
     _check(rc)
     return {"new_tokens": new, "edit_mask": mask, "confidence": conf, "argmax": am}
+
+
+def denoise_update(logits, tokens, cu_rows, block_size, mask_id, omega_mask, omega_edit, editable=None,
+                   max_blocks=None, is_bf16=False):
+    """Full Eq. 2 update (Gamma_t, forced unmasking, Delta_t) with entropies,
+    changed-block flags and per-sequence change counts, in float64."""
+    lib = _load()
+    logits = np.ascontiguousarray(logits) if is_bf16 else np.ascontiguousarray(logits, dtype=np.float32)
+    R, V = logits.shape
+    cu = _c(cu_rows, np.int32)
+    ns = cu.shape[0] - 1
+    if max_blocks is None:
+        max_blocks = max([1] + [int((cu[s + 1] - cu[s] + block_size - 1) // block_size) for s in range(ns)])
+    tokens = _c(tokens, np.int32)
+    out = {"new_tokens": np.zeros(R, np.int32), "kind": np.zeros(R, np.uint8), "confidence": np.zeros(R),
+           "argmax": np.zeros(R, np.int32), "entropy": np.zeros(R), "block_changed": np.zeros((ns, max_blocks), np.uint8),
+           "seq_changes": np.zeros(ns, np.int32)}
+    rc = lib.oracle_denoise_update(_ptr(logits), 1 if is_bf16 else 0, V, V, _ptr(cu), ns, block_size, max_blocks,
+                                   _ptr(tokens), int(mask_id), float(omega_mask), float(omega_edit),
+                                   _ptr(_c(editable, np.uint8)), _ptr(out["new_tokens"]), _ptr(out["kind"]),
+                                   _ptr(out["confidence"]), _ptr(out["argmax"]), _ptr(out["entropy"]),
+                                   _ptr(out["block_changed"]), _ptr(out["seq_changes"]))
+    _check(rc)
+    return out
+
+
+def tail_entropy_select(block_entropy, n_valid, rho, k_max):
+    """Eqs. 6-7: tail-entropy scores of the candidate blocks and the chosen
+    window start. block_entropy: float32 [S, n_hist, B]; n_valid: int32 [S]."""
+    lib = _load()
+    be = np.ascontiguousarray(block_entropy, dtype=np.float32)
+    S, H, B = be.shape
+    nv = _c(n_valid, np.int32)
+    scores = np.zeros((S, H))
+    best = np.zeros(S, np.int32)
+    wb = np.zeros(S, np.int32)
+    rc = lib.oracle_tail_entropy_select(_ptr(be), _ptr(nv), S, H, B, float(rho), int(k_max), _ptr(scores), _ptr(best),
+                                        _ptr(wb))
+    _check(rc)
+    return {"scores": scores, "best_slot": best, "window_blocks": wb}
 
 
 def kv_window_write(k_win, v_win, k_cache, v_cache, block_table, prefix_len, window_len, cu_window, block_size,

@@ -290,3 +290,170 @@ int oracle_kv_window_write(const uint16_t* k_win, const uint16_t* v_win, uint16_
   }
   return ORC_OK;
 }
+
+/*
+ * Full threshold update of a decoding step (Eq. 2 with the forced unmasking
+ * rule of Sec. 2.3), plus the per-row entropy H = -sum_v p_v log p_v of the
+ * prediction (the quantity behind Eq. 4, PPL = exp(H), and Eq. 6).
+ *
+ * Rows are ragged: sequence s owns rows cu_rows[s] .. cu_rows[s+1]-1; window
+ * block b of sequence s holds its rows b*block_size .. (b+1)*block_size-1.
+ * For row r with current token x = tokens[r], argmax x_hat and confidence c
+ * (as in oracle_edit_decide):
+ *   masked (x == mask_id):  unmask to x_hat if c > omega_mask       (Gamma_t, kind 1)
+ *   visible:                replace by x_hat if editable[r], x_hat != x and
+ *                           c > omega_edit                          (Delta_t, kind 3)
+ * Then, per block: if the block has masked rows and none of them was unmasked,
+ * its masked row of highest confidence (lowest row on equal confidence) is
+ * unmasked anyway (kind 2). Confidence comparisons use c rounded to float.
+ * block_changed[s][b] = 1 iff some row of block b got a new token (new != x);
+ * seq_changes[s] = number of rows of s whose token changed.
+ */
+int oracle_denoise_update(const void* logits, int32_t dtype, int64_t row_stride, int32_t vocab,
+                          const int32_t* cu_rows, int32_t num_seqs, int32_t block_size, int32_t max_blocks,
+                          const int32_t* tokens, int32_t mask_id, float omega_mask, float omega_edit,
+                          const uint8_t* editable, int32_t* new_tokens, uint8_t* kind, double* confidence,
+                          int32_t* argmax_out, double* entropy, uint8_t* block_changed, int32_t* seq_changes) {
+  if (num_seqs < 0 || vocab <= 0 || block_size <= 0 || (dtype != 0 && dtype != 1) || row_stride < vocab)
+    return ORC_BAD_ARG;
+  const int32_t rows = num_seqs > 0 ? cu_rows[num_seqs] : 0;
+  int status = ORC_OK;
+#pragma omp parallel for schedule(static)
+  for (int32_t r = 0; r < rows; ++r) {
+    double* x = (double*)malloc(sizeof(double) * (size_t)vocab);
+    if (!x) {
+#pragma omp atomic write
+      status = ORC_NOMEM;
+      continue;
+    }
+    double m = -INFINITY;
+    int32_t xh = -1;
+    int finite = 1;
+    for (int32_t v = 0; v < vocab; ++v) {
+      x[v] = dtype == 0 ? (double)((const float*)logits)[(int64_t)r * row_stride + v]
+                        : bf16_to_double(((const uint16_t*)logits)[(int64_t)r * row_stride + v]);
+      if (!isfinite(x[v])) finite = 0;
+      if (x[v] > m) {
+        m = x[v];
+        xh = v;
+      }
+    }
+    if (!finite) {
+      free(x);
+#pragma omp atomic write
+      status = ORC_NONFINITE;
+      continue;
+    }
+    double ssum = 0.0;
+    for (int32_t v = 0; v < vocab; ++v) ssum += exp(x[v] - m);
+    double h = 0.0;
+    for (int32_t v = 0; v < vocab; ++v) {
+      const double pv = exp(x[v] - m) / ssum;
+      if (pv > 0.0) h -= pv * log(pv);
+    }
+    free(x);
+    const double c = 1.0 / ssum;
+    confidence[r] = c;
+    argmax_out[r] = xh;
+    if (entropy) entropy[r] = h;
+    const int32_t cur = tokens[r];
+    uint8_t k = 0;
+    if (cur == mask_id) {
+      if ((float)c > omega_mask) k = 1;
+    } else if ((editable == NULL || editable[r] != 0) && xh != cur && (float)c > omega_edit) {
+      k = 3;
+    }
+    kind[r] = k;
+    new_tokens[r] = k ? xh : cur;
+  }
+  if (status != ORC_OK) return status;
+  for (int32_t s = 0; s < num_seqs; ++s) {
+    const int32_t r0 = cu_rows[s], r1 = cu_rows[s + 1];
+    const int32_t nblocks = (r1 - r0 + block_size - 1) / block_size;
+    if (nblocks > max_blocks && block_changed) return ORC_BAD_ARG;
+    int32_t changes = 0;
+    for (int32_t b = 0; b < nblocks; ++b) {
+      const int32_t b0 = r0 + b * block_size, b1 = (b0 + block_size < r1) ? b0 + block_size : r1;
+      int any_masked = 0, any_unmasked = 0, best = -1;
+      float best_c = 0.f;
+      for (int32_t r = b0; r < b1; ++r) {
+        if (tokens[r] != mask_id) continue;
+        any_masked = 1;
+        if (kind[r] == 1) any_unmasked = 1;
+        if (best < 0 || (float)confidence[r] > best_c) {
+          best = r;
+          best_c = (float)confidence[r];
+        }
+      }
+      if (any_masked && !any_unmasked) {
+        kind[best] = 2;
+        new_tokens[best] = argmax_out[best];
+      }
+      int changed = 0;
+      for (int32_t r = b0; r < b1; ++r)
+        if (new_tokens[r] != tokens[r]) {
+          changed = 1;
+          ++changes;
+        }
+      if (block_changed) block_changed[(int64_t)s * max_blocks + b] = (uint8_t)changed;
+    }
+    if (block_changed)
+      for (int32_t b = nblocks; b < max_blocks; ++b) block_changed[(int64_t)s * max_blocks + b] = 0;
+    if (seq_changes) seq_changes[s] = changes;
+  }
+  return ORC_OK;
+}
+
+static int cmp_desc(const void* a, const void* b) {
+  const double x = *(const double*)a, y = *(const double*)b;
+  return (x < y) - (x > y);
+}
+
+/*
+ * Tail-entropy block selection, Eqs. 6-7. For each sequence s the caller keeps
+ * the final standard-scope entropies of its last n_hist blocks in
+ * block_entropy[s][0..n_hist-1][0..block_size-1], oldest block first (slot
+ * n_hist-1 is block j-1); n_valid[s] <= n_hist of them exist. The candidates
+ * of Eq. 7 are the last min(n_valid[s], k_max - 1) slots. For each candidate
+ *   S_rho(i) = mean of the ceil(rho * block_size) largest entropies of block i
+ * (Eq. 6); best_slot[s] is the candidate of largest score (the oldest one on
+ * equal scores) and window_blocks[s] = n_hist - best_slot[s] + 1 is the number
+ * of blocks of the editing window W_j = [j* B, (j+1) B) of Eq. 5. Sequences
+ * without candidates get best_slot -1 and window_blocks 1. scores (optional)
+ * receives S_rho for every candidate slot (NaN elsewhere).
+ */
+int oracle_tail_entropy_select(const float* block_entropy, const int32_t* n_valid, int32_t num_seqs, int32_t n_hist,
+                               int32_t block_size, double rho, int32_t k_max, double* scores, int32_t* best_slot,
+                               int32_t* window_blocks) {
+  if (num_seqs < 0 || n_hist < 1 || block_size < 1 || k_max < 1 || !(rho > 0.0) || rho > 1.0) return ORC_BAD_ARG;
+  const int32_t top = (int32_t)ceil(rho * block_size);
+  double* buf = (double*)malloc(sizeof(double) * (size_t)block_size);
+  if (!buf) return ORC_NOMEM;
+  for (int32_t s = 0; s < num_seqs; ++s) {
+    int32_t nv = n_valid[s] < n_hist ? n_valid[s] : n_hist;
+    if (nv < 0) nv = 0;
+    const int32_t ncand = nv < k_max - 1 ? nv : k_max - 1;
+    int32_t best = -1;
+    double best_score = -INFINITY;
+    for (int32_t slot = 0; slot < n_hist; ++slot) {
+      const int cand = slot >= n_hist - ncand;
+      if (scores) scores[(int64_t)s * n_hist + slot] = NAN;
+      if (!cand) continue;
+      for (int32_t r = 0; r < block_size; ++r)
+        buf[r] = (double)block_entropy[((int64_t)s * n_hist + slot) * block_size + r];
+      qsort(buf, (size_t)block_size, sizeof(double), cmp_desc);
+      double sum = 0.0;
+      for (int32_t r = 0; r < top; ++r) sum += buf[r];
+      const double sc = sum / top;
+      if (scores) scores[(int64_t)s * n_hist + slot] = sc;
+      if (best < 0 || (float)sc > (float)best_score) {
+        best = slot;
+        best_score = sc;
+      }
+    }
+    best_slot[s] = best;
+    window_blocks[s] = best < 0 ? 1 : n_hist - best + 1;
+  }
+  free(buf);
+  return ORC_OK;
+}
