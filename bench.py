@@ -303,6 +303,8 @@ def run_gpu(args, rank, world):
     per_step = len(attn) * 2 + (1 if plan_layers else len(attn)) + (1 if ep is not None else 0) + \
         (len(attn) if with_kv_write else 0)
     res["gpu_launches"] = per_step * K
+    if ep is not None:
+        res["extras"] = time_extras(w, a0, dev, stream, peaks)
     res["e2e"] = run_e2e(args, w, attention_call, edit_call, dev, stream, world, new_t if ep is not None else None,
                          mask_t if ep is not None else None, conf_t if ep is not None else None)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -311,6 +313,44 @@ def run_gpu(args, rank, world):
         res["cpu_baseline"] = {"value": round(v, 5), "unit": "windows/s", "cores": oracle.num_threads(),
                                "kind": "oracle", "sample": desc}
     return res
+
+
+def time_extras(w, a0, dev, stream, peaks, reps=10):
+    """Entry points around the editing pass, timed outside the step: the full
+    Eq. 2 update of a standard decoding step over the same logits (a third of
+    the rows masked) and the tail-entropy window choice for every sequence."""
+    from paper_2607_22663_gb300 import mbe
+    ep = w["edit"]
+    R, V = ep.logits.shape
+    mask_id = V - 1
+    tokens = ep.committed.clone()
+    tokens[torch.arange(R, device=dev) % 3 == 0] = mask_id
+    cu = a0.cu_window
+
+    def ev_time(fn):
+        for _ in range(3):
+            fn()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    ms = ev_time(lambda: mbe.denoise_update(ep.logits, tokens, cu, block_size=a0.block_size, mask_id=mask_id,
+                                            omega_mask=0.5, omega_edit=0.0))
+    byts = R * V * ep.logits.element_size() + R * (4 + 4 + 1 + 4 + 4 + 4)
+    ent = torch.rand(a0.batch, 3, a0.block_size, device=dev)
+    nv = torch.full((a0.batch,), 3, dtype=torch.int32, device=dev)
+    ms_sel = ev_time(lambda: mbe.tail_entropy_select(ent, nv, rho=0.25, k_max=4))
+    st, flags = mbe.get_device_error()
+    if st != 0:
+        raise RuntimeError(f"device error in extras: status {st} flags {flags:#x}")
+    return {"denoise_update": {"ms": round(ms, 4), "gbs": round(byts / (ms * 1e-3) / 1e9, 1),
+                               "frac_hbm": round(byts / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"], 4),
+                               "rows": R, "vocab": V},
+            "tail_entropy_select": {"us": round(ms_sel * 1e3, 2), "sequences": a0.batch, "k_max": 4, "rho": 0.25}}
 
 
 def run_e2e(args, w, attention_call, edit_call, dev, stream, world, new_t, mask_t, conf_t):

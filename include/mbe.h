@@ -16,6 +16,10 @@
  *   mbe_edit_decide        argmax / confidence / threshold-and-replace (Eq. 2)
  *   mbe_kv_window_write    scatter of window K/V into the paged cache (Sec. 4.3)
  *
+ * and, around them, the full decoding-step update (mbe_denoise_update: Eq. 2
+ * with forced unmasking, entropies, changed blocks) and the tail-entropy
+ * window choice (mbe_tail_entropy_select: Eqs. 6-7).
+ *
  * Conventions shared by every entry point
  *   - All pointers are DEVICE pointers unless stated otherwise; the caller
  *     owns every buffer. The library never allocates device memory.
@@ -220,6 +224,72 @@ mbe_status mbe_edit_decide(const void* logits, mbe_dtype dtype, int64_t row_stri
                            const int32_t* committed, const float* tau_per_row_or_null, float tau,
                            const uint8_t* editable_or_null, int32_t* new_tokens, uint8_t* edit_mask,
                            float* confidence, int32_t* argmax_or_null, cudaStream_t stream);
+
+/*
+ * mbe_denoise_update -- the full update of Eq. 2 for one forward of block
+ * diffusion (standard step or editing pass), with the forced unmasking of
+ * Sec. 2.3, the prediction entropy, and the changed-block record of Sec. 4.3.
+ * Paper: Eq. 2 (Gamma_t = masked positions with c > omega_mask, unmasked to
+ * x_hat; Delta_t = visible positions with x_hat != x and c > omega_edit,
+ * overwritten by x_hat); Sec. 2.3 (if Gamma_t is empty while masks remain, the
+ * most confident masked position is unmasked); Eq. 4 / Eq. 6 (entropy of the
+ * prediction); Sec. 4.1 / 4.3 (stop when no token changes; refresh only the
+ * blocks that changed).
+ *
+ * Rows are ragged by sequence: sequence s owns rows cu_rows[s] ..
+ * cu_rows[s+1]-1 (device array, cu_rows[num_seqs] = total_rows); block b of
+ * sequence s is its rows b*block_size .. (b+1)*block_size-1. Per row r with
+ * current token x = tokens[r], x_hat and c as in mbe_edit_decide:
+ *   update_kind[r] = 1 if x == mask_id and c > omega_mask            (Gamma_t)
+ *                    2 if x == mask_id, forced (see below)
+ *                    3 if x != mask_id, editable, x_hat != x, c > omega_edit (Delta_t)
+ *                    0 otherwise;  new_tokens[r] = kind ? x_hat : x
+ * A block with masked rows of which none is in Gamma_t unmasks its most
+ * confident masked row (lowest row on equal fp32 confidence).
+ *   entropy_or_null[r] = -sum_v p_v ln p_v (fp32)
+ *   block_changed_or_null[s * max_blocks_per_seq + b] = 1 iff some row of block
+ *     b changed token (0 for blocks past the sequence's rows); it is the
+ *     block_write_mask of mbe_kv_window_write for the refresh.
+ *   seq_changes_or_null[s] = number of rows of s whose token changed.
+ * logits: [total_rows, row_stride] of `dtype` (first `vocab` entries used);
+ * tokens, new_tokens, argmax: int32 [total_rows] (new_tokens must not alias
+ * tokens); update_kind uint8, confidence fp32 [total_rows]; editable_or_null
+ * uint8 [total_rows] (NULL: all rows). A cu_rows range outside [0, total_rows]
+ * or more than max_blocks_per_seq blocks set MBE_DEVERR_LENGTH.
+ * Errors: MBE_ERR_INVALID_ARG, MBE_ERR_CUDA.
+ */
+mbe_status mbe_denoise_update(const void* logits, mbe_dtype dtype, int64_t row_stride, int32_t vocab,
+                              const int32_t* cu_rows, int32_t num_seqs, int32_t total_rows, int32_t block_size,
+                              int32_t max_blocks_per_seq, const int32_t* tokens, int32_t mask_id, float omega_mask,
+                              float omega_edit, const uint8_t* editable_or_null, int32_t* new_tokens,
+                              uint8_t* update_kind, float* confidence, int32_t* argmax, float* entropy_or_null,
+                              uint8_t* block_changed_or_null, int32_t* seq_changes_or_null, cudaStream_t stream);
+
+/*
+ * mbe_tail_entropy_select -- tail-entropy choice of the editing window start.
+ * Paper: Eq. 6 (S_rho(i) = mean of the ceil(rho B) largest final standard-scope
+ * entropies of block i), Eq. 7 (j* = argmax of S_rho over the candidate blocks
+ * C_j = {max(0, j - K_max + 1) <= i < j}), Eq. 5 (window W_j = [j* B, (j+1) B)).
+ *
+ *   block_entropy fp32 [num_seqs, n_hist, block_size]: the entropies (e.g. from
+ *     mbe_denoise_update) of each sequence's last n_hist blocks, oldest first;
+ *     slot n_hist-1 is block j-1.
+ *   n_valid int32 [num_seqs]: how many of those slots hold blocks (<= n_hist).
+ *   Candidates are the last min(n_valid, k_max - 1) slots.
+ *   best_slot int32 [num_seqs]: the candidate with the largest score (the
+ *     oldest on equal fp32 scores), -1 if there is none (j = 0);
+ *   window_blocks int32 [num_seqs]: n_hist - best_slot + 1 (1 without candidate),
+ *     the number of blocks of W_j including the current block j;
+ *   scores_or_null fp32 [num_seqs, n_hist]: S_rho of each candidate, NaN elsewhere.
+ * ceil(rho * block_size) is evaluated in double precision from the float rho.
+ * The paper maintains the running argmax with a monotonic deque over
+ * consecutive blocks; here each call evaluates its <= k_max - 1 candidates.
+ * Errors: MBE_ERR_INVALID_ARG (rho outside (0, 1], k_max < 1, ...),
+ * MBE_ERR_UNSUPPORTED (block_size > 12288), MBE_ERR_CUDA.
+ */
+mbe_status mbe_tail_entropy_select(const float* block_entropy, const int32_t* n_valid, int32_t num_seqs,
+                                   int32_t n_hist, int32_t block_size, float rho, int32_t k_max, float* scores_or_null,
+                                   int32_t* best_slot, int32_t* window_blocks, cudaStream_t stream);
 
 /*
  * mbe_kv_window_write -- refresh of the cache with the window's K/V.

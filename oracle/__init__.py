@@ -192,7 +192,9 @@ def tail_entropy_select(block_entropy, n_valid, rho, k_max):
     scores = np.zeros((S, H))
     best = np.zeros(S, np.int32)
     wb = np.zeros(S, np.int32)
-    rc = lib.oracle_tail_entropy_select(_ptr(be), _ptr(nv), S, H, B, float(rho), int(k_max), _ptr(scores), _ptr(best),
+    # rho as the float32 the library receives, so ceil(rho * B) uses the same value
+    rc = lib.oracle_tail_entropy_select(_ptr(be), _ptr(nv), S, H, B, float(np.float32(rho)), int(k_max), _ptr(scores),
+                                        _ptr(best),
                                         _ptr(wb))
     _check(rc)
     return {"scores": scores, "best_slot": best, "window_blocks": wb}

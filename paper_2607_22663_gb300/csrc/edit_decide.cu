@@ -8,6 +8,7 @@
 // kernel is bound by HBM bandwidth.
 #include <cuda_bf16.h>
 #include "common.cuh"
+#include "row_stats.cuh"
 
 namespace mbe {
 
@@ -15,13 +16,7 @@ MBE_DEFINE_ERROR_WORD(edit_decide_take_error)
 
 namespace {
 
-constexpr float kLog2e = 1.4426950408889634f;
-
-__device__ __forceinline__ float ex2(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
+using namespace rows;
 
 struct Triple {
   float m;  // running maximum
@@ -63,37 +58,6 @@ __device__ __forceinline__ Triple shfl_xor(const Triple& t, int mask) {
   o.idx = __shfl_xor_sync(0xffffffffu, t.idx, mask);
   return o;
 }
-
-template <typename T>
-__device__ __forceinline__ float to_f32(T x);
-template <>
-__device__ __forceinline__ float to_f32<float>(float x) { return x; }
-template <>
-__device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 x) { return __bfloat162float(x); }
-
-// Unpacks one 16-byte vector into floats.
-template <typename T>
-struct Vec;
-template <>
-struct Vec<float> {
-  static constexpr int N = 4;
-  __device__ __forceinline__ static void unpack(const uint4& v, float (&x)[4]) {
-    x[0] = __uint_as_float(v.x); x[1] = __uint_as_float(v.y);
-    x[2] = __uint_as_float(v.z); x[3] = __uint_as_float(v.w);
-  }
-};
-template <>
-struct Vec<__nv_bfloat16> {
-  static constexpr int N = 8;
-  __device__ __forceinline__ static void unpack(const uint4& v, float (&x)[8]) {
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      x[2 * k] = __uint_as_float(w[k] << 16);
-      x[2 * k + 1] = __uint_as_float(w[k] & 0xFFFF0000u);
-    }
-  }
-};
 
 template <typename T>
 __device__ __forceinline__ void absorb_vector(Triple& t, const uint4& v, int col0) {

@@ -71,6 +71,11 @@ def lib(build_if_missing: bool = True):
     L.mbe_window_attention_workspace_size.argtypes = [i32, i32, i32, i32, i32, i32]
     L.mbe_edit_decide.restype = ctypes.c_int
     L.mbe_edit_decide.argtypes = [P, ctypes.c_int, i64, i32, i32, P, P, f32, P, P, P, P, P, P]
+    L.mbe_denoise_update.restype = ctypes.c_int
+    L.mbe_denoise_update.argtypes = [P, ctypes.c_int, i64, i32, P, i32, i32, i32, i32, P, i32, f32, f32, P, P, P, P, P,
+                                     P, P, P, P]
+    L.mbe_tail_entropy_select.restype = ctypes.c_int
+    L.mbe_tail_entropy_select.argtypes = [P, P, i32, i32, i32, f32, i32, P, P, P, P]
     L.mbe_kv_window_write.restype = ctypes.c_int
     L.mbe_kv_window_write.argtypes = [P, P, P, P, i32, P, i32, P, P, P, P, i32, i32, i32, i32, i32, i32, i32, P]
     L.mbe_get_device_error.restype = ctypes.c_int
@@ -228,6 +233,54 @@ def edit_decide(logits, committed, tau=0.0, tau_per_row=None, editable=None, *, 
                                _ptr(argmax), _stream(stream))
     _check("mbe_edit_decide", st)
     return new_tokens, edit_mask, confidence, argmax
+
+
+def denoise_update(logits, tokens, cu_rows, *, block_size, mask_id, omega_mask, omega_edit, editable=None,
+                   max_blocks=None, want_entropy=True, want_blocks=True, stream=None):
+    """mbe_denoise_update: see include/mbe.h. Returns a dict of device tensors."""
+    if logits.dim() != 2 or logits.stride(1) != 1 or not logits.is_cuda:
+        raise ValueError("logits must be a CUDA [rows, vocab] tensor with unit stride along the vocabulary")
+    dt = {torch.float32: 0, torch.bfloat16: 1}.get(logits.dtype)
+    if dt is None:
+        raise TypeError("logits must be float32 or bfloat16")
+    R, V = logits.shape
+    _need(tokens, "tokens", torch.int32)
+    _need(cu_rows, "cu_rows", torch.int32)
+    if editable is not None:
+        _need(editable, "editable", torch.uint8)
+    ns = cu_rows.shape[0] - 1
+    dev = logits.device
+    if max_blocks is None:
+        max_blocks = max(1, (int((cu_rows[1:] - cu_rows[:-1]).max().item()) + block_size - 1) // block_size) if ns else 1
+    out = {"new_tokens": torch.empty(R, dtype=torch.int32, device=dev),
+           "kind": torch.empty(R, dtype=torch.uint8, device=dev),
+           "confidence": torch.empty(R, dtype=torch.float32, device=dev),
+           "argmax": torch.empty(R, dtype=torch.int32, device=dev),
+           "entropy": torch.empty(R, dtype=torch.float32, device=dev) if want_entropy else None,
+           "block_changed": torch.empty((ns, max_blocks), dtype=torch.uint8, device=dev) if want_blocks else None,
+           "seq_changes": torch.empty(ns, dtype=torch.int32, device=dev) if want_blocks else None}
+    st = lib().mbe_denoise_update(_ptr(logits), dt, logits.stride(0), V, _ptr(cu_rows), ns, R, block_size, max_blocks,
+                                  _ptr(tokens), int(mask_id), float(omega_mask), float(omega_edit), _ptr(editable),
+                                  _ptr(out["new_tokens"]), _ptr(out["kind"]), _ptr(out["confidence"]),
+                                  _ptr(out["argmax"]), _ptr(out["entropy"]), _ptr(out["block_changed"]),
+                                  _ptr(out["seq_changes"]), _stream(stream))
+    _check("mbe_denoise_update", st)
+    return out
+
+
+def tail_entropy_select(block_entropy, n_valid, *, rho, k_max, want_scores=True, stream=None):
+    """mbe_tail_entropy_select: see include/mbe.h. Returns (best_slot, window_blocks, scores)."""
+    _need(block_entropy, "block_entropy", torch.float32)
+    _need(n_valid, "n_valid", torch.int32)
+    S, H, B = block_entropy.shape
+    dev = block_entropy.device
+    best = torch.empty(S, dtype=torch.int32, device=dev)
+    wb = torch.empty(S, dtype=torch.int32, device=dev)
+    scores = torch.empty((S, H), dtype=torch.float32, device=dev) if want_scores else None
+    st = lib().mbe_tail_entropy_select(_ptr(block_entropy), _ptr(n_valid), S, H, B, float(rho), int(k_max),
+                                       _ptr(scores), _ptr(best), _ptr(wb), _stream(stream))
+    _check("mbe_tail_entropy_select", st)
+    return best, wb, scores
 
 
 def kv_window_write(k_win, v_win, k_cache, v_cache, block_table, prefix_len, window_len, cu_window, *, block_size,

@@ -125,3 +125,25 @@ def test_attention_plan_host_validation():
     assert f(None, P(16), P(16), P(16), 1, 64, 4, 1, 128, 32, 64, 64, P(16), 1 << 20, None) == 1
     assert f(None, None, None, None, 0, 0, 4, 1, 128, 32, 64, 64, None, 0, None) == 0
     assert f(P(16), P(16), P(16), P(16), 1, 64, 6, 4, 128, 32, 64, 64, P(16), 1 << 20, None) == 1   # heads
+
+
+def test_denoise_and_tail_entropy_host_validation():
+    L = mbe.lib()
+    P = ctypes.c_void_p
+    d = L.mbe_denoise_update
+    ok = [P(16), 1, 100, 100, P(16), 1, 8, 4, 2, P(16), 9, 0.5, 0.0, None, P(32), P(16), P(16), P(16), None, None, None,
+          None]
+    bad = list(ok); bad[3] = 0          # vocab 0
+    assert d(*bad) == 1
+    bad = list(ok); bad[14] = P(16)     # new_tokens aliases tokens
+    assert d(*bad) == 1
+    bad = list(ok); bad[9] = None       # null tokens
+    assert d(*bad) == 1
+    zero = list(ok); zero[5] = 0        # no sequences: nothing to do
+    assert d(*zero) == 0
+    t = L.mbe_tail_entropy_select
+    assert t(P(16), P(16), 2, 3, 32, 0.0, 4, None, P(16), P(16), None) == 1     # rho 0
+    assert t(P(16), P(16), 2, 3, 32, 1.5, 4, None, P(16), P(16), None) == 1     # rho > 1
+    assert t(P(16), P(16), 2, 3, 32, 0.25, 0, None, P(16), P(16), None) == 1    # k_max 0
+    assert t(P(16), P(16), 2, 3, 20000, 0.25, 4, None, P(16), P(16), None) == 2  # block too large
+    assert t(None, None, 0, 3, 32, 0.25, 4, None, None, None, None) == 0
