@@ -12,6 +12,8 @@ path computes, written from the paper (arXiv 2607.22663):
 * ``denoise_update``    -- the full Eq. 2 step (M2T set Gamma_t with forced
   unmasking, T2T set Delta_t), per-row entropies, changed-block flags.
 * ``tail_entropy_select`` -- Eqs. 6-7 tail-entropy scores and window start.
+* ``refresh_plan``      -- Sec. 4.3 targeted refresh: one block-causal
+  recompute problem per changed block, laid out as a ragged batch.
 
 Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
 ``bench.py`` may import it. It shares no code with the CUDA library and never
@@ -71,6 +73,8 @@ def _load():
         lib.oracle_tail_entropy_select.argtypes = [P, P, i32, i32, i32, f64, i32, P, P, P]
         lib.oracle_kv_window_write.restype = ctypes.c_int
         lib.oracle_kv_window_write.argtypes = [P, P, P, P, P, i32, P, P, P, P, i32, i32, i32, i32, i32, i32, i32]
+        lib.oracle_refresh_plan.restype = ctypes.c_int
+        lib.oracle_refresh_plan.argtypes = [P, i32, P, P, P, P, i32, i32, i32, i32, P, P, P, P, P, P, P]
         _lib = lib
     return _lib
 
@@ -217,3 +221,28 @@ def kv_window_write(k_win, v_win, k_cache, v_cache, block_table, prefix_len, win
                                     batch, Hkv, D, block_size, page_size, num_pages)
     _check(rc)
     return kc, vc
+
+
+def refresh_plan(block_changed, prefix_len, window_len, cu_window, block_table, block_size, total_rows=None):
+    """Targeted refresh layout (Sec. 4.3): one entry per (sequence, window
+    block), non-empty for the changed blocks. Returns a dict of numpy arrays
+    prefix_len, window_len, cu_window, mask_mode, block_table, src_row, count."""
+    lib = _load()
+    bc = _c(block_changed, np.uint8)
+    batch, max_blocks = bc.shape
+    bt = _c(block_table, np.int32)
+    cu = _c(cu_window, np.int32)
+    if total_rows is None:
+        total_rows = int(cu[batch]) if batch else 0
+    E = batch * max_blocks
+    out = {"prefix_len": np.zeros(E, np.int32), "window_len": np.zeros(E, np.int32),
+           "cu_window": np.zeros(E + 1, np.int32), "mask_mode": np.zeros(E, np.uint8),
+           "block_table": np.zeros((E, bt.shape[1]), np.int32), "src_row": np.zeros(total_rows, np.int32),
+           "count": np.zeros(2, np.int32)}
+    rc = lib.oracle_refresh_plan(_ptr(bc), max_blocks, _ptr(_c(prefix_len, np.int32)), _ptr(_c(window_len, np.int32)),
+                                 _ptr(cu), _ptr(bt), bt.shape[1], batch, block_size, total_rows,
+                                 _ptr(out["prefix_len"]), _ptr(out["window_len"]), _ptr(out["cu_window"]),
+                                 _ptr(out["mask_mode"]), _ptr(out["block_table"]), _ptr(out["src_row"]),
+                                 _ptr(out["count"]))
+    _check(rc)
+    return out

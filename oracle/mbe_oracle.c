@@ -457,3 +457,62 @@ int oracle_tail_entropy_select(const float* block_entropy, const int32_t* n_vali
   free(buf);
   return ORC_OK;
 }
+
+/*
+ * Targeted refresh of the blocks that changed (Sec. 4.3 with the block-causal
+ * conditioning of Sec. 2.2). Recomputing window block b of sequence s under
+ * standard attention means that its queries see the cached prefix, the window
+ * blocks before b as they stand in the cache (the changed ones are written
+ * there first), and all of block b itself. That is one attention problem per
+ * changed block: prefix P_s + b*B, a one-block window in bidirectional mode.
+ * This lays those problems out as a ragged batch of E = batch * max_blocks
+ * entries, entry e = s * max_blocks + b, empty unless block b of s changed:
+ *   r_prefix_len[e] = P_s + b*B and r_window_len[e] = min(B, W_s - b*B)
+ *                     for a changed block inside the window; 0 and 0 otherwise
+ *   r_cu_window[e]  = sum of r_window_len[0..e-1]  (E + 1 values)
+ *   r_mask_mode[e]  = 1 (bidirectional)
+ *   r_block_table[e][:] = block_table[s][:] for a changed block, -1 otherwise
+ *   r_src_row[k]    = cu_window[s] + b*B + i for refresh row k = r_cu_window[e] + i,
+ *                     and -1 for k from r_cu_window[E] up to total_rows
+ *   r_count[0] = changed entries, r_count[1] = r_cu_window[E]
+ * A window longer than max_blocks * B, or more refresh rows than total_rows,
+ * is an argument error.
+ */
+int oracle_refresh_plan(const uint8_t* block_changed, int32_t max_blocks, const int32_t* prefix_len,
+                        const int32_t* window_len, const int32_t* cu_window, const int32_t* block_table,
+                        int32_t max_pages_per_seq, int32_t batch, int32_t block_size, int32_t total_rows,
+                        int32_t* r_prefix_len, int32_t* r_window_len, int32_t* r_cu_window, uint8_t* r_mask_mode,
+                        int32_t* r_block_table, int32_t* r_src_row, int32_t* r_count) {
+  if (batch < 0 || max_blocks < 1 || block_size < 1 || total_rows < 0 || max_pages_per_seq < 0) return ORC_BAD_ARG;
+  for (int32_t s = 0; s < batch; ++s)
+    if (window_len[s] < 0 || window_len[s] > max_blocks * block_size) return ORC_BAD_ARG;
+  int32_t rows = 0, entries = 0;
+  for (int32_t s = 0; s < batch; ++s) {
+    for (int32_t b = 0; b < max_blocks; ++b) {
+      const int64_t e = (int64_t)s * max_blocks + b;
+      const int32_t start = b * block_size;
+      const int changed = block_changed[e] != 0 && start < window_len[s];
+      int32_t len = 0;
+      if (changed) {
+        len = window_len[s] - start;
+        if (len > block_size) len = block_size;
+      }
+      r_cu_window[e] = rows;
+      r_prefix_len[e] = changed ? prefix_len[s] + start : 0;
+      r_window_len[e] = len;
+      r_mask_mode[e] = 1;
+      for (int32_t p = 0; p < max_pages_per_seq; ++p)
+        r_block_table[e * max_pages_per_seq + p] = changed ? block_table[(int64_t)s * max_pages_per_seq + p] : -1;
+      for (int32_t i = 0; i < len; ++i) {
+        if (rows >= total_rows) return ORC_BAD_ARG;
+        r_src_row[rows++] = cu_window[s] + start + i;
+      }
+      entries += changed;
+    }
+  }
+  r_cu_window[(int64_t)batch * max_blocks] = rows;
+  for (int32_t k = rows; k < total_rows; ++k) r_src_row[k] = -1;
+  r_count[0] = entries;
+  r_count[1] = rows;
+  return ORC_OK;
+}
