@@ -17,12 +17,15 @@
  *   mbe_kv_window_write    scatter of window K/V into the paged cache (Sec. 4.3)
  *
  * and, around them, the full decoding-step update (mbe_denoise_update: Eq. 2
- * with forced unmasking, entropies, changed blocks) and the tail-entropy
- * window choice (mbe_tail_entropy_select: Eqs. 6-7).
+ * with forced unmasking, entropies, changed blocks), the tail-entropy
+ * window choice (mbe_tail_entropy_select: Eqs. 6-7), the targeted refresh of
+ * the changed blocks (mbe_refresh_plan, mbe_gather_rows: Sec. 4.3) and a
+ * device-side loop over editing passes (mbe_pass_loop_*: Sec. 4.1).
  *
  * Conventions shared by every entry point
  *   - All pointers are DEVICE pointers unless stated otherwise; the caller
- *     owns every buffer. The library never allocates device memory.
+ *     owns every buffer. The library never allocates device memory (the
+ *     CUDA graph that mbe_pass_loop_end instantiates aside).
  *   - Every call validates its host-visible arguments synchronously and returns
  *     a status; on any status other than MBE_OK nothing was launched.
  *   - Work is enqueued asynchronously on `stream`. Conditions that only the
@@ -313,6 +316,92 @@ mbe_status mbe_kv_window_write(const void* k_win, const void* v_win, void* k_cac
                                const uint8_t* block_write_mask_or_null, int32_t max_blocks_per_seq, int32_t batch,
                                int32_t max_window, int32_t num_kv_heads, int32_t head_dim, int32_t block_size,
                                int32_t page_size, cudaStream_t stream);
+
+/*
+ * mbe_refresh_plan -- lays out the targeted refresh of the blocks that changed.
+ * Paper: Sec. 4.3 (after an editing pass, only the blocks whose tokens changed
+ * are recomputed under standard attention and their KV written back) with the
+ * block-causal conditioning of Sec. 2.2 and Eq. 5's window W_j.
+ *
+ * Recomputing window block b of sequence s under standard attention means its
+ * queries see the cached prefix, the window blocks before b as they stand in
+ * the cache (write the changed blocks first, with mbe_kv_window_write on this
+ * layout), and all of block b. That is one attention problem per changed
+ * block: prefix P_s + b*B and a one-block bidirectional window. This writes
+ * those problems as a ragged batch of E = batch * max_blocks_per_seq entries,
+ * entry e = s * max_blocks_per_seq + b, empty unless block b of s changed:
+ *   r_prefix_len int32 [E]   P_s + b*B for a changed block, else 0
+ *   r_window_len int32 [E]   min(B, W_s - b*B) for a changed block inside the
+ *                            window, else 0
+ *   r_cu_window int32 [E+1]  exclusive prefix sum of r_window_len
+ *   r_mask_mode uint8 [E]    MBE_MULTI_BLOCK_BIDIRECTIONAL
+ *   r_block_table int32 [E, max_pages_per_seq]  block_table row s, or -1
+ *   r_src_row int32 [total_rows]  window row (index into the pass's rows,
+ *                            cu_window) of refresh row k < r_cu_window[E];
+ *                            -1 for the rest (see mbe_gather_rows)
+ *   r_count int32 [2]        {changed entries, refresh rows}
+ * Pass the result to mbe_window_attention / mbe_kv_window_write with batch E,
+ * max_window B and max_prefix >= max_s(P_s + B * floor((W_s - 1) / B)) (the
+ * start of the last block; max_s(P_s + W_s) - 1 always suffices; the block
+ * tables must cover it, as they do P_s + W_s for the write); total_rows = rows of the
+ * pass (cu_window[batch]) always suffices. Inputs: block_changed uint8
+ * [batch, max_blocks_per_seq] (as written by mbe_denoise_update), prefix_len,
+ * window_len int32 [batch], cu_window int32 [batch+1], block_table int32
+ * [batch, max_pages_per_seq]. Everything stays on the device, so the call can
+ * be captured in a CUDA graph. Device checks: a window longer than max_window
+ * or than max_blocks_per_seq * B is treated as unchanged and sets
+ * MBE_DEVERR_LENGTH; more refresh rows than total_rows sets MBE_DEVERR_CAPACITY.
+ * Errors: MBE_ERR_INVALID_ARG (null pointers, negative sizes),
+ * MBE_ERR_UNSUPPORTED (more than 2^24 entries), MBE_ERR_CUDA.
+ */
+mbe_status mbe_refresh_plan(const uint8_t* block_changed, int32_t max_blocks_per_seq, const int32_t* prefix_len,
+                            const int32_t* window_len, const int32_t* cu_window, const int32_t* block_table,
+                            int32_t max_pages_per_seq, int32_t batch, int32_t block_size, int32_t max_window,
+                            int32_t total_rows, int32_t* r_prefix_len, int32_t* r_window_len, int32_t* r_cu_window,
+                            uint8_t* r_mask_mode, int32_t* r_block_table, int32_t* r_src_row, int32_t* r_count,
+                            cudaStream_t stream);
+
+/*
+ * mbe_gather_rows -- dst[k] = src[src_row[k]] for rows of row_bytes bytes
+ * (k < rows): the compaction of per-row inputs (token ids, hidden states,
+ * Q/K/V) for the refresh batch of mbe_refresh_plan. A negative src_row[k]
+ * gives a zero row; src_row[k] >= src_rows gives a zero row and sets
+ * MBE_DEVERR_LENGTH. src and dst are device buffers that must not overlap;
+ * 16-byte rows and alignment give vectorised copies.
+ * Errors: MBE_ERR_INVALID_ARG, MBE_ERR_CUDA.
+ */
+mbe_status mbe_gather_rows(const void* src, int64_t src_rows, int64_t row_bytes, const int32_t* src_row,
+                           int64_t rows, void* dst, cudaStream_t stream);
+
+/*
+ * Editing-pass loop on the device. Paper: Sec. 4.1 (the window is edited by
+ * repeated passes until a pass changes no token or N_MBE passes have run) and
+ * Sec. 4.3 (one graph serves every shape of the pass).
+ *
+ * mbe_pass_loop_begin creates a CUDA graph made of a reset of *passes_done
+ * and a conditional WHILE node, and starts capturing `stream` (not the legacy
+ * default stream) into the node's body in relaxed capture mode: everything
+ * enqueued on `stream` until mbe_pass_loop_end is one pass. The body must
+ * end with mbe_pass_loop_until_stable, which counts the pass in *passes_done
+ * (device int32) and runs another pass only if some seq_changes[s] != 0 (as
+ * written by mbe_denoise_update in the same pass) and fewer than max_passes
+ * passes ran. mbe_pass_loop_end instantiates the graph; mbe_pass_loop_launch
+ * runs all passes with one launch and no host synchronisation. Buffers used in
+ * the body must outlive the loop. mbe_pass_loop_destroy releases everything
+ * (it also ends a capture still open).
+ * Errors: MBE_ERR_INVALID_ARG (max_passes < 1, null pointers, a stream already
+ * capturing or the default stream, until_stable missing or repeated, another
+ * stream), MBE_ERR_CUDA (capture or instantiation failed; see
+ * mbe_last_error_string).
+ */
+typedef struct mbe_pass_loop mbe_pass_loop;
+mbe_status mbe_pass_loop_begin(int32_t max_passes, int32_t* passes_done, cudaStream_t stream,
+                               mbe_pass_loop** loop_out);
+mbe_status mbe_pass_loop_until_stable(mbe_pass_loop* loop, const int32_t* seq_changes, int32_t num_seqs,
+                                      cudaStream_t stream);
+mbe_status mbe_pass_loop_end(mbe_pass_loop* loop, cudaStream_t stream);
+mbe_status mbe_pass_loop_launch(mbe_pass_loop* loop, cudaStream_t stream);
+void mbe_pass_loop_destroy(mbe_pass_loop* loop);
 
 /* Synchronises `stream`, then reads and clears the device error word of the
  * current device. Returns MBE_OK if it was clear, MBE_ERR_TIMEOUT if the

@@ -78,6 +78,20 @@ def lib(build_if_missing: bool = True):
     L.mbe_tail_entropy_select.argtypes = [P, P, i32, i32, i32, f32, i32, P, P, P, P]
     L.mbe_kv_window_write.restype = ctypes.c_int
     L.mbe_kv_window_write.argtypes = [P, P, P, P, i32, P, i32, P, P, P, P, i32, i32, i32, i32, i32, i32, i32, P]
+    L.mbe_refresh_plan.restype = ctypes.c_int
+    L.mbe_refresh_plan.argtypes = [P, i32, P, P, P, P, i32, i32, i32, i32, i32, P, P, P, P, P, P, P, P]
+    L.mbe_gather_rows.restype = ctypes.c_int
+    L.mbe_gather_rows.argtypes = [P, i64, i64, P, i64, P, P]
+    L.mbe_pass_loop_begin.restype = ctypes.c_int
+    L.mbe_pass_loop_begin.argtypes = [i32, P, P, ctypes.POINTER(ctypes.c_void_p)]
+    L.mbe_pass_loop_until_stable.restype = ctypes.c_int
+    L.mbe_pass_loop_until_stable.argtypes = [P, P, i32, P]
+    L.mbe_pass_loop_end.restype = ctypes.c_int
+    L.mbe_pass_loop_end.argtypes = [P, P]
+    L.mbe_pass_loop_launch.restype = ctypes.c_int
+    L.mbe_pass_loop_launch.argtypes = [P, P]
+    L.mbe_pass_loop_destroy.restype = None
+    L.mbe_pass_loop_destroy.argtypes = [P]
     L.mbe_get_device_error.restype = ctypes.c_int
     L.mbe_get_device_error.argtypes = [P, ctypes.POINTER(ctypes.c_uint32)]
     L.mbe_status_string.restype = ctypes.c_char_p
@@ -236,8 +250,12 @@ def edit_decide(logits, committed, tau=0.0, tau_per_row=None, editable=None, *, 
 
 
 def denoise_update(logits, tokens, cu_rows, *, block_size, mask_id, omega_mask, omega_edit, editable=None,
-                   max_blocks=None, want_entropy=True, want_blocks=True, stream=None):
-    """mbe_denoise_update: see include/mbe.h. Returns a dict of device tensors."""
+                   max_blocks=None, want_entropy=True, want_blocks=True, out=None, stream=None):
+    """mbe_denoise_update: see include/mbe.h. Returns a dict of device tensors.
+
+    `out` (a dict as returned by an earlier call) reuses its buffers, so the
+    call allocates nothing and can be captured in a CUDA graph; max_blocks is
+    then taken from out["block_changed"]."""
     if logits.dim() != 2 or logits.stride(1) != 1 or not logits.is_cuda:
         raise ValueError("logits must be a CUDA [rows, vocab] tensor with unit stride along the vocabulary")
     dt = {torch.float32: 0, torch.bfloat16: 1}.get(logits.dtype)
@@ -250,20 +268,38 @@ def denoise_update(logits, tokens, cu_rows, *, block_size, mask_id, omega_mask, 
         _need(editable, "editable", torch.uint8)
     ns = cu_rows.shape[0] - 1
     dev = logits.device
-    if max_blocks is None:
-        max_blocks = max(1, (int((cu_rows[1:] - cu_rows[:-1]).max().item()) + block_size - 1) // block_size) if ns else 1
-    out = {"new_tokens": torch.empty(R, dtype=torch.int32, device=dev),
-           "kind": torch.empty(R, dtype=torch.uint8, device=dev),
-           "confidence": torch.empty(R, dtype=torch.float32, device=dev),
-           "argmax": torch.empty(R, dtype=torch.int32, device=dev),
-           "entropy": torch.empty(R, dtype=torch.float32, device=dev) if want_entropy else None,
-           "block_changed": torch.empty((ns, max_blocks), dtype=torch.uint8, device=dev) if want_blocks else None,
-           "seq_changes": torch.empty(ns, dtype=torch.int32, device=dev) if want_blocks else None}
+    if out is not None:
+        for k, dtype in (("new_tokens", torch.int32), ("kind", torch.uint8), ("confidence", torch.float32),
+                         ("argmax", torch.int32)):
+            _need(out[k], k, dtype)
+            if out[k].numel() != R:
+                raise ValueError(f"out[{k!r}] must hold {R} rows")
+        if out.get("block_changed") is not None:
+            _need(out["block_changed"], "block_changed", torch.uint8)
+            max_blocks = out["block_changed"].shape[1]
+            if out["block_changed"].shape[0] != ns or out.get("seq_changes") is None or \
+                    out["seq_changes"].numel() != ns:
+                raise ValueError("out['block_changed'] / out['seq_changes'] must cover every sequence")
+            _need(out["seq_changes"], "seq_changes", torch.int32)
+        if out.get("entropy") is not None:
+            _need(out["entropy"], "entropy", torch.float32)
+        max_blocks = max_blocks or 1
+    else:
+        if max_blocks is None:
+            max_blocks = max(1, (int((cu_rows[1:] - cu_rows[:-1]).max().item()) + block_size - 1) // block_size) \
+                if ns else 1
+        out = {"new_tokens": torch.empty(R, dtype=torch.int32, device=dev),
+               "kind": torch.empty(R, dtype=torch.uint8, device=dev),
+               "confidence": torch.empty(R, dtype=torch.float32, device=dev),
+               "argmax": torch.empty(R, dtype=torch.int32, device=dev),
+               "entropy": torch.empty(R, dtype=torch.float32, device=dev) if want_entropy else None,
+               "block_changed": torch.empty((ns, max_blocks), dtype=torch.uint8, device=dev) if want_blocks else None,
+               "seq_changes": torch.empty(ns, dtype=torch.int32, device=dev) if want_blocks else None}
     st = lib().mbe_denoise_update(_ptr(logits), dt, logits.stride(0), V, _ptr(cu_rows), ns, R, block_size, max_blocks,
                                   _ptr(tokens), int(mask_id), float(omega_mask), float(omega_edit), _ptr(editable),
                                   _ptr(out["new_tokens"]), _ptr(out["kind"]), _ptr(out["confidence"]),
-                                  _ptr(out["argmax"]), _ptr(out["entropy"]), _ptr(out["block_changed"]),
-                                  _ptr(out["seq_changes"]), _stream(stream))
+                                  _ptr(out["argmax"]), _ptr(out.get("entropy")), _ptr(out.get("block_changed")),
+                                  _ptr(out.get("seq_changes")), _stream(stream))
     _check("mbe_denoise_update", st)
     return out
 
@@ -302,6 +338,108 @@ def kv_window_write(k_win, v_win, k_cache, v_cache, block_table, prefix_len, win
                                    _ptr(block_write_mask), max_blocks, batch, max_window, Hkv, D, block_size,
                                    page_size, _stream(stream))
     _check("mbe_kv_window_write", st)
+
+
+def refresh_plan(block_changed, prefix_len, window_len, cu_window, block_table, *, block_size, max_window,
+                 total_rows=None, out=None, stream=None):
+    """mbe_refresh_plan: see include/mbe.h. Returns a dict of device tensors
+    prefix_len, window_len, cu_window, mask_mode, block_table, src_row, count
+    (reusing `out` when given, so that the call can be captured in a graph)."""
+    _need(block_changed, "block_changed", torch.uint8)
+    for t, n in ((prefix_len, "prefix_len"), (window_len, "window_len"), (cu_window, "cu_window"),
+                 (block_table, "block_table")):
+        _need(t, n, torch.int32)
+    batch, max_blocks = block_changed.shape
+    max_pages = block_table.shape[1]
+    if block_table.shape[0] != batch or prefix_len.numel() != batch or window_len.numel() != batch or \
+            cu_window.numel() != batch + 1:
+        raise ValueError("block_changed, prefix_len, window_len, cu_window and block_table disagree on the batch")
+    E = batch * max_blocks
+    dev = block_changed.device
+    if out is None:
+        if total_rows is None:
+            raise ValueError("total_rows (rows of the pass) is required when out is not given")
+        out = {"prefix_len": torch.empty(E, dtype=torch.int32, device=dev),
+               "window_len": torch.empty(E, dtype=torch.int32, device=dev),
+               "cu_window": torch.empty(E + 1, dtype=torch.int32, device=dev),
+               "mask_mode": torch.empty(E, dtype=torch.uint8, device=dev),
+               "block_table": torch.empty((E, max_pages), dtype=torch.int32, device=dev),
+               "src_row": torch.empty(int(total_rows), dtype=torch.int32, device=dev),
+               "count": torch.empty(2, dtype=torch.int32, device=dev)}
+    shapes = {"prefix_len": (E,), "window_len": (E,), "cu_window": (E + 1,), "mask_mode": (E,),
+              "block_table": (E, max_pages), "count": (2,)}
+    for k, shp in shapes.items():
+        _need(out[k], k, torch.uint8 if k == "mask_mode" else torch.int32)
+        if tuple(out[k].shape) != shp:
+            raise ValueError(f"out[{k!r}] must have shape {shp}")
+    _need(out["src_row"], "src_row", torch.int32)
+    st = lib().mbe_refresh_plan(_ptr(block_changed), max_blocks, _ptr(prefix_len), _ptr(window_len), _ptr(cu_window),
+                                _ptr(block_table), max_pages, batch, block_size, max_window, out["src_row"].numel(),
+                                _ptr(out["prefix_len"]), _ptr(out["window_len"]), _ptr(out["cu_window"]),
+                                _ptr(out["mask_mode"]), _ptr(out["block_table"]), _ptr(out["src_row"]),
+                                _ptr(out["count"]), _stream(stream))
+    _check("mbe_refresh_plan", st)
+    return out
+
+
+def gather_rows(src, src_row, out=None, stream=None):
+    """mbe_gather_rows: out[k] = src[src_row[k]] (zero rows where src_row[k] < 0)."""
+    _need(src, "src", None)
+    _need(src_row, "src_row", torch.int32)
+    rows = src_row.numel()
+    if out is None:
+        out = torch.empty((rows,) + tuple(src.shape[1:]), dtype=src.dtype, device=src.device)
+    _need(out, "out", src.dtype)
+    if tuple(out.shape[1:]) != tuple(src.shape[1:]) or out.shape[0] != rows:
+        raise ValueError("out must be [len(src_row)] + src.shape[1:]")
+    row_bytes = (src[0].numel() if src.shape[0] else out[0].numel() if rows else 1) * src.element_size()
+    st = lib().mbe_gather_rows(_ptr(src), src.shape[0], row_bytes, _ptr(src_row), rows, _ptr(out), _stream(stream))
+    _check("mbe_gather_rows", st)
+    return out
+
+
+class PassLoop:
+    """mbe_pass_loop_*: see include/mbe.h. Usage::
+
+        loop = PassLoop(max_passes, passes_done, stream)   # starts capturing `stream`
+        with torch.cuda.stream(stream):
+            ...one pass: library calls on `stream` with preallocated buffers...
+        loop.until_stable(seq_changes)
+        loop.end()
+        loop.launch()          # all passes, one graph launch
+        loop.close()
+    """
+
+    def __init__(self, max_passes, passes_done, stream):
+        _need(passes_done, "passes_done", torch.int32)
+        if stream is None or stream.cuda_stream == 0:
+            raise ValueError("the pass loop needs a non-default stream")
+        self.stream = stream
+        self._h = ctypes.c_void_p(None)
+        st = lib().mbe_pass_loop_begin(int(max_passes), _ptr(passes_done), _stream(stream), ctypes.byref(self._h))
+        _check("mbe_pass_loop_begin", st)
+
+    def until_stable(self, seq_changes):
+        _need(seq_changes, "seq_changes", torch.int32)
+        st = lib().mbe_pass_loop_until_stable(self._h, _ptr(seq_changes), seq_changes.numel(), _stream(self.stream))
+        _check("mbe_pass_loop_until_stable", st)
+
+    def end(self):
+        _check("mbe_pass_loop_end", lib().mbe_pass_loop_end(self._h, _stream(self.stream)))
+
+    def launch(self, stream=None):
+        _check("mbe_pass_loop_launch", lib().mbe_pass_loop_launch(self._h, _stream(stream or self.stream)))
+
+    def close(self):
+        if self._h:
+            lib().mbe_pass_loop_destroy(self._h)
+            self._h = ctypes.c_void_p(None)
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
 
 
 def get_device_error(stream=None):
