@@ -344,13 +344,163 @@ def time_extras(w, a0, dev, stream, peaks, reps=10):
     ent = torch.rand(a0.batch, 3, a0.block_size, device=dev)
     nv = torch.full((a0.batch,), 3, dtype=torch.int32, device=dev)
     ms_sel = ev_time(lambda: mbe.tail_entropy_select(ent, nv, rho=0.25, k_max=4))
+    refresh = time_refresh(w, dev, stream, peaks, ev_time)
+    loop = time_pass_loop(w, dev, reps=3)
     st, flags = mbe.get_device_error()
     if st != 0:
         raise RuntimeError(f"device error in extras: status {st} flags {flags:#x}")
     return {"denoise_update": {"ms": round(ms, 4), "gbs": round(byts / (ms * 1e-3) / 1e9, 1),
                                "frac_hbm": round(byts / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"], 4),
                                "rows": R, "vocab": V},
-            "tail_entropy_select": {"us": round(ms_sel * 1e3, 2), "sequences": a0.batch, "k_max": 4, "rho": 0.25}}
+            "tail_entropy_select": {"us": round(ms_sel * 1e3, 2), "sequences": a0.batch, "k_max": 4, "rho": 0.25},
+            "refresh": refresh, "pass_loop": loop}
+
+
+class RefreshBuffers:
+    """Preallocated buffers of the targeted refresh of one pass (every layer
+    reuses them; the layers run in order on one stream)."""
+
+    def __init__(self, a0, dev, max_blocks):
+        from paper_2607_22663_gb300 import mbe
+        B = a0.block_size
+        self.E = a0.batch * max_blocks
+        self.max_prefix = max(p + B * ((wl - 1) // B) for p, wl in zip(a0.prefix_host, a0.window_host) if wl > 0)
+        self.q, self.k, self.v = torch.empty_like(a0.q), torch.empty_like(a0.k_win), torch.empty_like(a0.v_win)
+        self.out = torch.empty_like(a0.q)
+        self.ws = torch.empty(mbe.window_attention_workspace_size(self.E, a0.num_q_heads, a0.num_kv_heads, a0.head_dim,
+                                                                  B, self.max_prefix), dtype=torch.uint8, device=dev)
+        self.plan = None
+
+
+def refresh_pass(attn, changed, rb, stream=None):
+    """Sec. 4.3 refresh of the changed blocks over every layer: plan once, then
+    per layer gather the changed rows' Q/K/V, write their K/V, attend."""
+    from paper_2607_22663_gb300 import mbe
+    a0 = attn[0]
+    B = a0.block_size
+    rb.plan = mbe.refresh_plan(changed, a0.prefix_len, a0.window_len, a0.cu_window, a0.block_table, block_size=B,
+                               max_window=a0.max_window, total_rows=a0.total_tokens, out=rb.plan, stream=stream)
+    p = rb.plan
+    for i, a in enumerate(attn):
+        for src, dst in ((a.q, rb.q), (a.k_win, rb.k), (a.v_win, rb.v)):
+            mbe.gather_rows(src, p["src_row"], out=dst, stream=stream)
+        mbe.kv_window_write(rb.k, rb.v, a.k_cache, a.v_cache, p["block_table"], p["prefix_len"], p["window_len"],
+                            p["cu_window"], block_size=B, max_window=B, stream=stream)
+        fn = mbe.window_attention if i == 0 else mbe.window_attention_run
+        fn(rb.q, rb.k, rb.v, a.k_cache, a.v_cache, p["block_table"], p["prefix_len"], p["window_len"], p["cu_window"],
+           p["mask_mode"], block_size=B, max_window=B, max_prefix=rb.max_prefix, out=rb.out, workspace=rb.ws,
+           stream=stream)
+
+
+def time_refresh(w, dev, stream, peaks, ev_time, frac=0.125):
+    """Targeted refresh of a seeded eighth of the window blocks, all layers."""
+    attn = w["attn"]
+    a0 = attn[0]
+    B = a0.block_size
+    max_blocks = (a0.max_window + B - 1) // B
+    g = torch.Generator(device="cpu").manual_seed(99)
+    changed = (torch.rand(a0.batch, max_blocks, generator=g) < frac).to(torch.uint8)
+    nblk = [(wl + B - 1) // B for wl in a0.window_host]
+    for s, n in enumerate(nblk):
+        changed[s, n:] = 0
+    rb = RefreshBuffers(a0, dev, max_blocks)
+    d_changed = changed.to(dev)
+    ms = ev_time(lambda: refresh_pass(attn, d_changed, rb))
+    # algorithmic bytes of the refresh attention: each changed block reads K/V of
+    # its prefix and of itself, and its Q and O
+    kv_row = 2 * a0.num_kv_heads * a0.head_dim * 2
+    qo_row = 2 * a0.num_q_heads * a0.head_dim * 2
+    byts = 0
+    for s in range(a0.batch):
+        for b in range(nblk[s]):
+            if changed[s, b]:
+                ln = min(B, a0.window_host[s] - b * B)
+                byts += (a0.prefix_host[s] + b * B + ln) * kv_row + ln * qo_row
+    byts *= len(attn)
+    return {"ms_per_pass": round(ms, 4), "changed_blocks": int(changed.sum()), "blocks": int(sum(nblk)),
+            "layers": len(attn), "attention_gbs": round(byts / (ms * 1e-3) / 1e9, 1),
+            "frac_hbm": round(byts / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"], 4),
+            "note": "plan + per layer (3 row gathers, KV write, attention of the changed blocks)"}
+
+
+def time_pass_loop(w, dev, reps=3, max_passes=5):
+    """The editing loop of Sec. 4.1 (pass = window attention of every layer,
+    Eq. 2 update, refresh of the changed blocks, commit) until no token
+    changes or max_passes passes: one conditional-graph launch against the same
+    calls issued from the host with a host read of the change count per pass."""
+    from paper_2607_22663_gb300 import mbe
+    from paper_2607_22663_gb300.workloads import editable_historical
+    attn = w["attn"]
+    ep = w["edit"]
+    a0 = attn[0]
+    B = a0.block_size
+    R, V = ep.logits.shape
+    max_blocks = (a0.max_window + B - 1) // B
+    editable = editable_historical(a0.window_host, B, dev)
+    outs = [torch.empty_like(a.q) for a in attn]
+    ws = torch.empty(max(mbe.window_attention_workspace_size(a.batch, a.num_q_heads, a.num_kv_heads, a.head_dim,
+                                                             a.max_window, a.max_prefix) for a in attn),
+                     dtype=torch.uint8, device=dev)
+    tokens = torch.empty_like(ep.committed)
+    ident = torch.arange(R, dtype=torch.int32, device=dev)
+    rb = RefreshBuffers(a0, dev, max_blocks)
+    upd = mbe.denoise_update(ep.logits, ep.committed, a0.cu_window, block_size=B, mask_id=V - 1, omega_mask=0.5,
+                             omega_edit=ep.tau, editable=editable, max_blocks=max_blocks)
+
+    def one_pass(stream):
+        for i, a in enumerate(attn):
+            fn = mbe.window_attention if i == 0 else mbe.window_attention_run
+            fn(a.q, a.k_win, a.v_win, a.k_cache, a.v_cache, a.block_table, a.prefix_len, a.window_len, a.cu_window,
+               a.mask_mode, block_size=B, max_window=a.max_window, max_prefix=a.max_prefix, out=outs[i], workspace=ws,
+               stream=stream)
+        mbe.denoise_update(ep.logits, tokens, a0.cu_window, block_size=B, mask_id=V - 1, omega_mask=0.5,
+                           omega_edit=ep.tau, editable=editable, out=upd, stream=stream)
+        refresh_pass(attn, upd["block_changed"], rb, stream=stream)
+        mbe.gather_rows(upd["new_tokens"], ident, out=tokens, stream=stream)
+
+    s = torch.cuda.Stream(dev)
+    with torch.cuda.stream(s):
+        tokens.copy_(ep.committed)
+        one_pass(s)          # allocates the refresh layout buffers outside the capture
+    s.synchronize()
+    passes = torch.zeros(1, dtype=torch.int32, device=dev)
+    loop = mbe.PassLoop(max_passes, passes, s)
+    try:
+        one_pass(s)
+        loop.until_stable(upd["seq_changes"])
+        loop.end()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        graph_ms = []
+        for r in range(reps + 1):
+            with torch.cuda.stream(s):
+                tokens.copy_(ep.committed)
+                e0.record(s)
+                loop.launch()
+                e1.record(s)
+            s.synchronize()
+            if r:
+                graph_ms.append(e0.elapsed_time(e1))
+        n_graph = int(passes.item())
+    finally:
+        loop.close()
+    eager_ms = []
+    for r in range(reps + 1):
+        with torch.cuda.stream(s):
+            tokens.copy_(ep.committed)
+            s.synchronize()
+            t0 = time.perf_counter()
+            n = 0
+            while True:
+                one_pass(s)
+                n += 1
+                if int(upd["seq_changes"].sum().item()) == 0 or n >= max_passes:
+                    break
+            s.synchronize()
+            if r:
+                eager_ms.append((time.perf_counter() - t0) * 1e3)
+    return {"passes": n_graph, "eager_passes": n, "max_passes": max_passes,
+            "graph_ms": round(statistics.median(graph_ms), 4), "eager_ms": round(statistics.median(eager_ms), 4),
+            "note": "pass = window attention of every layer + Eq. 2 update + refresh of changed blocks + commit"}
 
 
 def run_e2e(args, w, attention_call, edit_call, dev, stream, world, new_t, mask_t, conf_t):
