@@ -89,30 +89,30 @@ __device__ __forceinline__ void absorb_vector(Stats& a, const uint4& v, int col0
   constexpr int N = Vec<T>::N;
   float x[N];
   Vec<T>::unpack(v, x);
-  float lm = x[0];
-  int li = 0;
-#pragma unroll
-  for (int k = 1; k < N; ++k)
-    if (x[k] > lm) { lm = x[k]; li = k; }
-  if (a.idx < 0) {
-    a.m = lm;
-    a.idx = col0 + li;
-    a.s = 0.f;
-    a.t = 0.f;
-  } else if (lm > a.m) {
-    rebase(a, lm);
-    a.idx = col0 + li;
+  const float lm = vec_max(x);
+  if (lm > a.m) {  // rare after the first vectors; a.m starts at -inf
+    if (a.idx < 0) {
+      a.s = 0.f;
+      a.t = 0.f;
+      a.m = lm;
+    } else {
+      rebase(a, lm);
+    }
+    a.idx = col0 + first_index(x, lm);
   }
-  float s = 0.f, t = 0.f;
+  // u = l log2e - m log2e and e = 2^u, two elements per packed FMA / add
+  const float2 L = make_float2(kLog2e, kLog2e);
+  const float2 ms = make_float2(-a.m * kLog2e, -a.m * kLog2e);
+  float2 s = make_float2(0.f, 0.f), t = make_float2(0.f, 0.f);
 #pragma unroll
-  for (int k = 0; k < N; ++k) {
-    const float u = (x[k] - a.m) * kLog2e;
-    const float e = ex2(u);
-    s += e;
-    t = fmaf(e, u, t);
+  for (int k = 0; k < N; k += 2) {
+    const float2 u = ffma2(make_float2(x[k], x[k + 1]), L, ms);
+    const float2 e = make_float2(ex2(u.x), ex2(u.y));
+    s = fadd2(s, e);
+    t = ffma2(e, u, t);
   }
-  a.s += s;
-  a.t += t;
+  a.s += s.x + s.y;
+  a.t += t.x + t.y;
 }
 
 struct RowArgs {
@@ -136,7 +136,7 @@ __global__ void __launch_bounds__(kThreads) denoise_row_kernel(const T* __restri
   constexpr int kUnroll = 4;
   const int row = blockIdx.x;
   const T* rp = logits + static_cast<int64_t>(row) * a.row_stride;
-  Stats st{0.f, 0.f, 0.f, -1};
+  Stats st{__int_as_float(0xff800000u), 0.f, 0.f, -1};  // empty: m = -inf
   int scalar_from = 0;
   if (a.vec_ok) {
     const uint4* vp = reinterpret_cast<const uint4*>(rp);

@@ -3,6 +3,7 @@
 #pragma once
 #include <cstdint>
 #include <cuda_bf16.h>
+#include "ptx_sm103.cuh"
 
 namespace mbe {
 namespace rows {
@@ -45,6 +46,22 @@ struct Vec<__nv_bfloat16> {
     }
   }
 };
+
+// Maximum of a vector's elements (3-input max instructions).
+__device__ __forceinline__ float vec_max(const float (&x)[8]) {
+  return fmax3(fmax3(x[0], x[1], x[2]), fmax3(x[3], x[4], x[5]), fmaxf(x[6], x[7]));
+}
+__device__ __forceinline__ float vec_max(const float (&x)[4]) { return fmax3(x[0], x[1], fmaxf(x[2], x[3])); }
+
+// Lowest k with x[k] == v (v is one of the elements).
+template <int N>
+__device__ __forceinline__ int first_index(const float (&x)[N], float v) {
+  int i = N - 1;
+#pragma unroll
+  for (int k = N - 2; k >= 0; --k)
+    if (x[k] == v) i = k;
+  return i;
+}
 
 }  // namespace rows
 }  // namespace mbe
