@@ -14,6 +14,8 @@ path computes, written from the paper (arXiv 2607.22663):
 * ``tail_entropy_select`` -- Eqs. 6-7 tail-entropy scores and window start.
 * ``refresh_plan``      -- Sec. 4.3 targeted refresh: one block-causal
   recompute problem per changed block, laid out as a ragged batch.
+* ``lm_head_logits``    -- the LM-head projection whose rows the T2T rule
+  reads (float64 logits for ``edit_decide`` / ``denoise_update``).
 
 Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
 ``bench.py`` may import it. It shares no code with the CUDA library and never
@@ -73,6 +75,8 @@ def _load():
         lib.oracle_tail_entropy_select.argtypes = [P, P, i32, i32, i32, f64, i32, P, P, P]
         lib.oracle_kv_window_write.restype = ctypes.c_int
         lib.oracle_kv_window_write.argtypes = [P, P, P, P, P, i32, P, P, P, P, i32, i32, i32, i32, i32, i32, i32]
+        lib.oracle_lm_head_logits.restype = ctypes.c_int
+        lib.oracle_lm_head_logits.argtypes = [P, P, i32, i32, i32, i32, P, P]
         lib.oracle_refresh_plan.restype = ctypes.c_int
         lib.oracle_refresh_plan.argtypes = [P, i32, P, P, P, P, i32, i32, i32, i32, P, P, P, P, P, P, P]
         _lib = lib
@@ -89,6 +93,13 @@ def _ptr(a):
 
 def _c(a, dtype):
     return None if a is None else np.ascontiguousarray(a, dtype=dtype)
+
+
+def _logit_dtype(logits, is_bf16):
+    """0 float32, 1 bf16 bits (uint16, is_bf16), 2 float64."""
+    if is_bf16:
+        return 1
+    return 2 if np.asarray(logits).dtype == np.float64 else 0
 
 
 def _check(rc):
@@ -137,7 +148,7 @@ def window_attention(q, k_win, v_win, k_cache, v_cache, block_table, prefix_len,
 def edit_decide(logits, committed, tau=0.0, tau_per_row=None, editable=None, rows=None, is_bf16=False):
     """T2T edit decision of Eq. 2 in float64.
 
-    logits: float32 [R, V] or uint16 bf16 bits [R, V] (set is_bf16).
+    logits: float32 [R, V], float64 [R, V] or uint16 bf16 bits [R, V] (set is_bf16).
     Returns dict of new_tokens int32, edit_mask uint8, confidence float64,
     argmax int32 (all [R]; rows not in `rows` are left as -1 / 0 / NaN).
     """
@@ -152,8 +163,8 @@ def edit_decide(logits, committed, tau=0.0, tau_per_row=None, editable=None, row
     conf = np.full(R, np.nan, dtype=np.float64)
     am = np.full(R, -1, dtype=np.int32)
     sel = None if rows is None else np.ascontiguousarray(rows, dtype=np.int32)
-    dtype = 1 if is_bf16 else 0
-    if not is_bf16:
+    dtype = _logit_dtype(logits, is_bf16)
+    if dtype == 0:
         logits = np.ascontiguousarray(logits, dtype=np.float32)
     rc = lib.oracle_edit_decide(_ptr(logits), dtype, V, R, V, _ptr(committed), _ptr(tpr), float(tau), _ptr(ed),
                                 -1 if sel is None else sel.shape[0], _ptr(sel), _ptr(new), _ptr(mask), _ptr(conf),
@@ -167,7 +178,8 @@ def denoise_update(logits, tokens, cu_rows, block_size, mask_id, omega_mask, ome
     """Full Eq. 2 update (Gamma_t, forced unmasking, Delta_t) with entropies,
     changed-block flags and per-sequence change counts, in float64."""
     lib = _load()
-    logits = np.ascontiguousarray(logits) if is_bf16 else np.ascontiguousarray(logits, dtype=np.float32)
+    dtype = _logit_dtype(logits, is_bf16)
+    logits = np.ascontiguousarray(logits) if dtype else np.ascontiguousarray(logits, dtype=np.float32)
     R, V = logits.shape
     cu = _c(cu_rows, np.int32)
     ns = cu.shape[0] - 1
@@ -177,7 +189,7 @@ def denoise_update(logits, tokens, cu_rows, block_size, mask_id, omega_mask, ome
     out = {"new_tokens": np.zeros(R, np.int32), "kind": np.zeros(R, np.uint8), "confidence": np.zeros(R),
            "argmax": np.zeros(R, np.int32), "entropy": np.zeros(R), "block_changed": np.zeros((ns, max_blocks), np.uint8),
            "seq_changes": np.zeros(ns, np.int32)}
-    rc = lib.oracle_denoise_update(_ptr(logits), 1 if is_bf16 else 0, V, V, _ptr(cu), ns, block_size, max_blocks,
+    rc = lib.oracle_denoise_update(_ptr(logits), dtype, V, V, _ptr(cu), ns, block_size, max_blocks,
                                    _ptr(tokens), int(mask_id), float(omega_mask), float(omega_edit),
                                    _ptr(_c(editable, np.uint8)), _ptr(out["new_tokens"]), _ptr(out["kind"]),
                                    _ptr(out["confidence"]), _ptr(out["argmax"]), _ptr(out["entropy"]),
@@ -244,5 +256,22 @@ def refresh_plan(block_changed, prefix_len, window_len, cu_window, block_table, 
                                  _ptr(out["prefix_len"]), _ptr(out["window_len"]), _ptr(out["cu_window"]),
                                  _ptr(out["mask_mode"]), _ptr(out["block_table"]), _ptr(out["src_row"]),
                                  _ptr(out["count"]))
+    _check(rc)
+    return out
+
+
+def lm_head_logits(hidden, weight, rows=None):
+    """LM-head logits in float64 from bf16 bits: hidden uint16 [R, d], weight
+    uint16 [V, d]. Returns [R, V] (or [len(rows), V] for the selected rows)."""
+    lib = _load()
+    h = _c(hidden, np.uint16)
+    w = _c(weight, np.uint16)
+    R, d = h.shape
+    V = w.shape[0]
+    assert w.shape[1] == d
+    sel = None if rows is None else np.ascontiguousarray(rows, dtype=np.int32)
+    n = R if sel is None else sel.shape[0]
+    out = np.zeros((n, V), dtype=np.float64)
+    rc = lib.oracle_lm_head_logits(_ptr(h), _ptr(w), R, V, d, -1 if sel is None else n, _ptr(sel), _ptr(out))
     _check(rc)
     return out

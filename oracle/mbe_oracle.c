@@ -44,6 +44,13 @@ static double bf16_to_double(uint16_t b) {
   return (double)f;
 }
 
+/* logit v of row r: dtype 0 float32, 1 bf16 bits, 2 float64 */
+static double load_logit(const void* logits, int32_t dtype, int64_t idx) {
+  if (dtype == 0) return (double)((const float*)logits)[idx];
+  if (dtype == 1) return bf16_to_double(((const uint16_t*)logits)[idx]);
+  return ((const double*)logits)[idx];
+}
+
 int oracle_num_threads(void) {
 #ifdef _OPENMP
   return omp_get_max_threads();
@@ -196,14 +203,15 @@ int oracle_window_attention(const uint16_t* q, const uint16_t* k_win, const uint
  * taken on c rounded to float, the precision of tau. editable == NULL means
  * every row is editable (the caller restricts edits to the historical part of
  * the window, Sec. 4.1).
- * dtype 0: float32 logits, dtype 1: bf16 logits. If n_sel >= 0 only rows
+ * dtype 0: float32 logits, 1: bf16 logits, 2: float64 logits (the LM-head
+ * projection of oracle_lm_head_logits). If n_sel >= 0 only rows
  * sel_rows[0..n_sel-1] are computed; outputs are indexed by row.
  */
 int oracle_edit_decide(const void* logits, int32_t dtype, int64_t row_stride, int32_t rows, int32_t vocab,
                        const int32_t* committed, const float* tau_per_row, float tau, const uint8_t* editable,
                        int32_t n_sel, const int32_t* sel_rows, int32_t* new_tokens, uint8_t* edit_mask,
                        double* confidence, int32_t* argmax_out) {
-  if (rows < 0 || vocab <= 0 || (dtype != 0 && dtype != 1) || row_stride < vocab) return ORC_BAD_ARG;
+  if (rows < 0 || vocab <= 0 || dtype < 0 || dtype > 2 || row_stride < vocab) return ORC_BAD_ARG;
   const int64_t total = n_sel >= 0 ? n_sel : rows;
   int status = ORC_OK;
 #pragma omp parallel for schedule(static)
@@ -218,12 +226,7 @@ int oracle_edit_decide(const void* logits, int32_t dtype, int64_t row_stride, in
     int32_t xh = -1;
     int finite = 1;
     for (int32_t v = 0; v < vocab; ++v) {
-      double x;
-      if (dtype == 0) {
-        x = (double)((const float*)logits)[(int64_t)r * row_stride + v];
-      } else {
-        x = bf16_to_double(((const uint16_t*)logits)[(int64_t)r * row_stride + v]);
-      }
+      const double x = load_logit(logits, dtype, (int64_t)r * row_stride + v);
       if (!isfinite(x)) finite = 0;
       if (x > m) {
         m = x;
@@ -237,12 +240,7 @@ int oracle_edit_decide(const void* logits, int32_t dtype, int64_t row_stride, in
     }
     double ssum = 0.0;
     for (int32_t v = 0; v < vocab; ++v) {
-      double x;
-      if (dtype == 0) {
-        x = (double)((const float*)logits)[(int64_t)r * row_stride + v];
-      } else {
-        x = bf16_to_double(((const uint16_t*)logits)[(int64_t)r * row_stride + v]);
-      }
+      const double x = load_logit(logits, dtype, (int64_t)r * row_stride + v);
       ssum += exp(x - m);
     }
     const double c = 1.0 / ssum;
@@ -314,7 +312,7 @@ int oracle_denoise_update(const void* logits, int32_t dtype, int64_t row_stride,
                           const int32_t* tokens, int32_t mask_id, float omega_mask, float omega_edit,
                           const uint8_t* editable, int32_t* new_tokens, uint8_t* kind, double* confidence,
                           int32_t* argmax_out, double* entropy, uint8_t* block_changed, int32_t* seq_changes) {
-  if (num_seqs < 0 || vocab <= 0 || block_size <= 0 || (dtype != 0 && dtype != 1) || row_stride < vocab)
+  if (num_seqs < 0 || vocab <= 0 || block_size <= 0 || dtype < 0 || dtype > 2 || row_stride < vocab)
     return ORC_BAD_ARG;
   const int32_t rows = num_seqs > 0 ? cu_rows[num_seqs] : 0;
   int status = ORC_OK;
@@ -330,8 +328,7 @@ int oracle_denoise_update(const void* logits, int32_t dtype, int64_t row_stride,
     int32_t xh = -1;
     int finite = 1;
     for (int32_t v = 0; v < vocab; ++v) {
-      x[v] = dtype == 0 ? (double)((const float*)logits)[(int64_t)r * row_stride + v]
-                        : bf16_to_double(((const uint16_t*)logits)[(int64_t)r * row_stride + v]);
+      x[v] = load_logit(logits, dtype, (int64_t)r * row_stride + v);
       if (!isfinite(x[v])) finite = 0;
       if (x[v] > m) {
         m = x[v];
@@ -514,5 +511,42 @@ int oracle_refresh_plan(const uint8_t* block_changed, int32_t max_blocks, const 
   for (int32_t k = rows; k < total_rows; ++k) r_src_row[k] = -1;
   r_count[0] = entries;
   r_count[1] = rows;
+  return ORC_OK;
+}
+
+/*
+ * LM-head projection of the final hidden states (the logits the T2T rule of
+ * Eq. 2 reads): l[r, v] = sum_k hidden[r, k] * weight[v, k] over k = 0..d-1,
+ * bf16 inputs widened exactly to double, products and sums in double in
+ * ascending k. If n_sel >= 0 only rows sel_rows[0..n_sel-1] are computed and
+ * out holds them in that order ([n_sel, vocab]); else out is [rows, vocab].
+ */
+int oracle_lm_head_logits(const uint16_t* hidden, const uint16_t* weight, int32_t rows, int32_t vocab, int32_t d,
+                          int32_t n_sel, const int32_t* sel_rows, double* out) {
+  if (rows < 0 || vocab <= 0 || d <= 0) return ORC_BAD_ARG;
+  const int64_t total = n_sel >= 0 ? n_sel : rows;
+  for (int64_t u = 0; u < total; ++u) {
+    const int32_t r = n_sel >= 0 ? sel_rows[u] : (int32_t)u;
+    if (r < 0 || r >= rows) return ORC_BAD_ARG;
+  }
+  double* hrow = (double*)malloc(sizeof(double) * (size_t)d * (size_t)(total > 0 ? total : 1));
+  if (!hrow) return ORC_NOMEM;
+  for (int64_t u = 0; u < total; ++u) {
+    const int32_t r = n_sel >= 0 ? sel_rows[u] : (int32_t)u;
+    for (int32_t k = 0; k < d; ++k) hrow[u * d + k] = bf16_to_double(hidden[(int64_t)r * d + k]);
+  }
+#pragma omp parallel for schedule(static)
+  for (int32_t v = 0; v < vocab; ++v) {
+    double* wrow = (double*)malloc(sizeof(double) * (size_t)d);
+    if (!wrow) continue;
+    for (int32_t k = 0; k < d; ++k) wrow[k] = bf16_to_double(weight[(int64_t)v * d + k]);
+    for (int64_t u = 0; u < total; ++u) {
+      double acc = 0.0;
+      for (int32_t k = 0; k < d; ++k) acc += hrow[u * d + k] * wrow[k];
+      out[u * vocab + v] = acc;
+    }
+    free(wrow);
+  }
+  free(hrow);
   return ORC_OK;
 }
