@@ -19,8 +19,9 @@
  * and, around them, the full decoding-step update (mbe_denoise_update: Eq. 2
  * with forced unmasking, entropies, changed blocks), the tail-entropy
  * window choice (mbe_tail_entropy_select: Eqs. 6-7), the targeted refresh of
- * the changed blocks (mbe_refresh_plan, mbe_gather_rows: Sec. 4.3) and a
- * device-side loop over editing passes (mbe_pass_loop_*: Sec. 4.1).
+ * the changed blocks (mbe_refresh_plan, mbe_gather_rows: Sec. 4.3), a
+ * device-side loop over editing passes (mbe_pass_loop_*: Sec. 4.1) and the
+ * LM-head projection fused with the edit decision (mbe_lm_head_edit_decide).
  *
  * Conventions shared by every entry point
  *   - All pointers are DEVICE pointers unless stated otherwise; the caller
@@ -316,6 +317,37 @@ mbe_status mbe_kv_window_write(const void* k_win, const void* v_win, void* k_cac
                                const uint8_t* block_write_mask_or_null, int32_t max_blocks_per_seq, int32_t batch,
                                int32_t max_window, int32_t num_kv_heads, int32_t head_dim, int32_t block_size,
                                int32_t page_size, cudaStream_t stream);
+
+/*
+ * mbe_lm_head_edit_decide -- the LM-head projection fused with the edit
+ * decision, so that the [rows, vocab] logits never reach memory.
+ * Paper: Eq. 2 (T2T set Delta_t: x_hat = argmax of the prediction, c its
+ * probability; replace where x_hat != x and c > omega_edit) on the logits
+ * l[r, v] = sum_k hidden[r, k] * weight[v, k] of the window rows (Sec. 4.1),
+ * and the prediction entropy of Eqs. 4 and 6.
+ *   hidden  bf16 [rows, hidden_dim]   final hidden states of the window rows
+ *   weight  bf16 [vocab, hidden_dim]  LM head, one row per token id
+ *   committed, tau_per_row_or_null, tau, editable_or_null, new_tokens,
+ *   edit_mask, confidence, argmax_or_null: as in mbe_edit_decide
+ *   entropy_or_null fp32 [rows]: -sum_v p_v ln p_v
+ *   workspace: device buffer of at least mbe_lm_head_workspace_size(rows,
+ *     vocab) bytes, 16-byte aligned (per-row partial states of 2048-token
+ *     vocabulary chunks).
+ * The logits are accumulated in fp32 on the tensor cores (bf16 products), so
+ * they differ from exact dot products by fp32 rounding of the running sums;
+ * decisions are taken on those fp32 values. hidden_dim must be a multiple of 8
+ * and hidden / weight 16-byte aligned.
+ * Errors: MBE_ERR_INVALID_ARG, MBE_ERR_WORKSPACE, MBE_ERR_UNSUPPORTED
+ * (rows or vocab above 2^30), MBE_ERR_CUDA; a bounded wait that expires sets
+ * MBE_DEVERR_TIMEOUT.
+ */
+size_t mbe_lm_head_workspace_size(int32_t rows, int32_t vocab);
+mbe_status mbe_lm_head_edit_decide(const void* hidden, const void* weight, int32_t rows, int32_t vocab,
+                                   int32_t hidden_dim, const int32_t* committed, const float* tau_per_row_or_null,
+                                   float tau, const uint8_t* editable_or_null, int32_t* new_tokens,
+                                   uint8_t* edit_mask, float* confidence, int32_t* argmax_or_null,
+                                   float* entropy_or_null, void* workspace, size_t workspace_bytes,
+                                   cudaStream_t stream);
 
 /*
  * mbe_refresh_plan -- lays out the targeted refresh of the blocks that changed.

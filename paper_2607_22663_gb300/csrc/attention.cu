@@ -32,6 +32,7 @@
 #include <mutex>
 #include "common.cuh"
 #include "ptx_sm103.cuh"
+#include "tma_host.cuh"
 
 namespace mbe {
 
@@ -908,34 +909,6 @@ __global__ void __launch_bounds__(kUnitRows) attn_merge_kernel(const MergeParams
 }
 
 // ------------------------------------------------------------------ host side
-typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
-                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFn encode_fn() {
-  static EncodeTiledFn fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* ptr = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-            cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<EncodeTiledFn>(ptr);
-  });
-  return fn;
-}
-
-bool encode(CUtensorMap* tm, const void* base, int rank, const cuuint64_t* dims, const cuuint64_t* strides,
-            const cuuint32_t* box) {
-  EncodeTiledFn fn = encode_fn();
-  if (!fn) return false;
-  cuuint32_t es[4] = {1, 1, 1, 1};
-  return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 struct DeviceInfo {
   int num_sms = 0;
   bool attr_set[2] = {false, false};
@@ -990,13 +963,14 @@ mbe_status run(const void* q, const void* k_win, const void* v_win, const void* 
     const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)Hq, (cuuint64_t)total_q_tokens};
     const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)Hq * D * 2};
     const cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)(kTileRows / G)};
-    if (!encode(&tq, q, 3, dims, strides, box)) return MBE_ERR_CUDA;
+    if (!encode_bf16_sw128(&tq, q, 3, dims, strides, box)) return MBE_ERR_CUDA;
   }
   {
     const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)Hkv, (cuuint64_t)total_q_tokens};
     const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)Hkv * D * 2};
     const cuuint32_t box[3] = {64, 1, (cuuint32_t)kTileKeys};
-    if (!encode(&tkw, k_win, 3, dims, strides, box) || !encode(&tvw, v_win, 3, dims, strides, box))
+    if (!encode_bf16_sw128(&tkw, k_win, 3, dims, strides, box) ||
+        !encode_bf16_sw128(&tvw, v_win, 3, dims, strides, box))
       return MBE_ERR_CUDA;
   }
   const int box_rows = std::min(page_size, kTileKeys);
@@ -1005,7 +979,8 @@ mbe_status run(const void* q, const void* k_win, const void* v_win, const void* 
     const cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)page_size * D * 2,
                                    (cuuint64_t)Hkv * page_size * D * 2};
     const cuuint32_t box[4] = {64, (cuuint32_t)box_rows, 1, 1};
-    if (!encode(&tkc, k_cache, 4, dims, strides, box) || !encode(&tvc, v_cache, 4, dims, strides, box))
+    if (!encode_bf16_sw128(&tkc, k_cache, 4, dims, strides, box) ||
+        !encode_bf16_sw128(&tvc, v_cache, 4, dims, strides, box))
       return MBE_ERR_CUDA;
   }
   if (!ensure_smem_attr<D>(di)) {

@@ -27,63 +27,6 @@ namespace {
 
 using namespace rows;
 
-struct Stats {
-  float m;   // running maximum
-  float s;   // sum of e = 2^u, u = (l - m) log2(e)
-  float t;   // sum of e * u
-  int idx;   // lowest index attaining m; -1 while empty
-};
-
-__device__ __forceinline__ void rebase(Stats& a, float m_new) {
-  // re-expresses (s, t) relative to a larger maximum
-  const float d = (a.m - m_new) * kLog2e;  // <= 0
-  const float f = ex2(d);
-  a.t = f * (a.t + d * a.s);
-  a.s *= f;
-  a.m = m_new;
-}
-
-__device__ __forceinline__ void absorb(Stats& a, float x, int col) {
-  if (a.idx < 0) {
-    a.m = x;
-    a.idx = col;
-    a.s = 1.f;
-    a.t = 0.f;
-    return;
-  }
-  if (x > a.m) {
-    rebase(a, x);
-    a.idx = col;
-  }
-  const float u = (x - a.m) * kLog2e;
-  const float e = ex2(u);
-  a.s += e;
-  a.t = fmaf(e, u, a.t);
-}
-
-__device__ __forceinline__ void merge(Stats& a, Stats b) {
-  if (b.idx < 0) return;
-  if (a.idx < 0) {
-    a = b;
-    return;
-  }
-  if (b.m > a.m) {
-    rebase(a, b.m);
-    a.idx = b.idx;
-  } else if (b.m < a.m) {
-    rebase(b, a.m);
-  } else {
-    a.idx = min(a.idx, b.idx);
-  }
-  a.s += b.s;
-  a.t += b.t;
-}
-
-__device__ __forceinline__ Stats shfl_xor(const Stats& t, int mask) {
-  return Stats{__shfl_xor_sync(0xffffffffu, t.m, mask), __shfl_xor_sync(0xffffffffu, t.s, mask),
-               __shfl_xor_sync(0xffffffffu, t.t, mask), __shfl_xor_sync(0xffffffffu, t.idx, mask)};
-}
-
 template <typename T>
 __device__ __forceinline__ void absorb_vector(Stats& a, const uint4& v, int col0) {
   constexpr int N = Vec<T>::N;

@@ -78,6 +78,10 @@ def lib(build_if_missing: bool = True):
     L.mbe_tail_entropy_select.argtypes = [P, P, i32, i32, i32, f32, i32, P, P, P, P]
     L.mbe_kv_window_write.restype = ctypes.c_int
     L.mbe_kv_window_write.argtypes = [P, P, P, P, i32, P, i32, P, P, P, P, i32, i32, i32, i32, i32, i32, i32, P]
+    L.mbe_lm_head_workspace_size.restype = sz
+    L.mbe_lm_head_workspace_size.argtypes = [i32, i32]
+    L.mbe_lm_head_edit_decide.restype = ctypes.c_int
+    L.mbe_lm_head_edit_decide.argtypes = [P, P, i32, i32, i32, P, P, f32, P, P, P, P, P, P, P, sz, P]
     L.mbe_refresh_plan.restype = ctypes.c_int
     L.mbe_refresh_plan.argtypes = [P, i32, P, P, P, P, i32, i32, i32, i32, i32, P, P, P, P, P, P, P, P]
     L.mbe_gather_rows.restype = ctypes.c_int
@@ -338,6 +342,47 @@ def kv_window_write(k_win, v_win, k_cache, v_cache, block_table, prefix_len, win
                                    _ptr(block_write_mask), max_blocks, batch, max_window, Hkv, D, block_size,
                                    page_size, _stream(stream))
     _check("mbe_kv_window_write", st)
+
+
+def lm_head_workspace_size(rows, vocab):
+    return int(lib().mbe_lm_head_workspace_size(int(rows), int(vocab)))
+
+
+def lm_head_edit_decide(hidden, weight, committed, tau=0.0, tau_per_row=None, editable=None, *, new_tokens=None,
+                        edit_mask=None, confidence=None, argmax=None, entropy=None, want_argmax=True,
+                        want_entropy=False, workspace=None, stream=None):
+    """mbe_lm_head_edit_decide: see include/mbe.h. Returns (new_tokens,
+    edit_mask, confidence, argmax, entropy) (argmax / entropy None unless wanted)."""
+    _need(hidden, "hidden", torch.bfloat16)
+    _need(weight, "weight", torch.bfloat16)
+    _need(committed, "committed", torch.int32)
+    if hidden.dim() != 2 or weight.dim() != 2 or hidden.shape[1] != weight.shape[1]:
+        raise ValueError("hidden must be [rows, d] and weight [vocab, d]")
+    R, d = hidden.shape
+    V = weight.shape[0]
+    if committed.numel() != R:
+        raise ValueError("committed must hold one token per row")
+    if tau_per_row is not None:
+        _need(tau_per_row, "tau_per_row", torch.float32)
+    if editable is not None:
+        _need(editable, "editable", torch.uint8)
+    dev = hidden.device
+    new_tokens = torch.empty(R, dtype=torch.int32, device=dev) if new_tokens is None else new_tokens
+    edit_mask = torch.empty(R, dtype=torch.uint8, device=dev) if edit_mask is None else edit_mask
+    confidence = torch.empty(R, dtype=torch.float32, device=dev) if confidence is None else confidence
+    if want_argmax and argmax is None:
+        argmax = torch.empty(R, dtype=torch.int32, device=dev)
+    if want_entropy and entropy is None:
+        entropy = torch.empty(R, dtype=torch.float32, device=dev)
+    need = lm_head_workspace_size(R, V)
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
+    st = lib().mbe_lm_head_edit_decide(_ptr(hidden), _ptr(weight), R, V, d, _ptr(committed), _ptr(tau_per_row),
+                                       float(tau), _ptr(editable), _ptr(new_tokens), _ptr(edit_mask),
+                                       _ptr(confidence), _ptr(argmax), _ptr(entropy), _ptr(workspace),
+                                       workspace.numel(), _stream(stream))
+    _check("mbe_lm_head_edit_decide", st)
+    return new_tokens, edit_mask, confidence, argmax, entropy
 
 
 def refresh_plan(block_changed, prefix_len, window_len, cu_window, block_table, *, block_size, max_window,
