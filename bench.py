@@ -344,6 +344,7 @@ def time_extras(w, a0, dev, stream, peaks, reps=10):
     ent = torch.rand(a0.batch, 3, a0.block_size, device=dev)
     nv = torch.full((a0.batch,), 3, dtype=torch.int32, device=dev)
     ms_sel = ev_time(lambda: mbe.tail_entropy_select(ent, nv, rho=0.25, k_max=4))
+    lm_head = time_lm_head(w, dev, peaks, ev_time)
     refresh = time_refresh(w, dev, stream, peaks, ev_time)
     loop = time_pass_loop(w, dev, reps=3)
     st, flags = mbe.get_device_error()
@@ -353,7 +354,41 @@ def time_extras(w, a0, dev, stream, peaks, reps=10):
                                "frac_hbm": round(byts / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"], 4),
                                "rows": R, "vocab": V},
             "tail_entropy_select": {"us": round(ms_sel * 1e3, 2), "sequences": a0.batch, "k_max": 4, "rho": 0.25},
-            "refresh": refresh, "pass_loop": loop}
+            "lm_head_edit_decide": lm_head, "refresh": refresh, "pass_loop": loop}
+
+
+def time_lm_head(w, dev, peaks, ev_time, hidden=4096):
+    """LM-head projection fused with the edit decision (the logits never reach
+    HBM) on random weights, against cuBLAS writing bf16 logits followed by the
+    HBM-streaming edit decision."""
+    from paper_2607_22663_gb300 import mbe
+    ep = w["edit"]
+    R, V = ep.logits.shape
+    g = torch.Generator(device=dev).manual_seed(123)
+    h = torch.randn(R, hidden, generator=g, device=dev).to(torch.bfloat16)
+    W = (torch.randn(V, hidden, generator=g, device=dev) * (2.0 / hidden ** 0.5)).to(torch.bfloat16)
+    ws = torch.empty(mbe.lm_head_workspace_size(R, V), dtype=torch.uint8, device=dev)
+    new = torch.empty(R, dtype=torch.int32, device=dev)
+    mask = torch.empty(R, dtype=torch.uint8, device=dev)
+    conf = torch.empty(R, dtype=torch.float32, device=dev)
+    fused = ev_time(lambda: mbe.lm_head_edit_decide(h, W, ep.committed, tau=ep.tau, new_tokens=new, edit_mask=mask,
+                                                    confidence=conf, want_argmax=False, workspace=ws))
+    logits = torch.empty(R, V, dtype=torch.bfloat16, device=dev)
+    gemm = ev_time(lambda: torch.matmul(h, W.t(), out=logits))
+
+    def unfused():
+        torch.matmul(h, W.t(), out=logits)
+        mbe.edit_decide(logits, ep.committed, tau=ep.tau, new_tokens=new, edit_mask=mask, confidence=conf,
+                        want_argmax=False)
+    unf = ev_time(unfused)
+    flops = 2.0 * R * V * hidden
+    tf = flops / (fused * 1e-3) / 1e12
+    del logits, W, h
+    return {"ms": round(fused, 4), "tflops": round(tf, 1), "frac_bf16_peak_burst": round(tf / peaks["bf16_tflops"], 4),
+            "frac_bf16_peak_sustained": round(tf / peaks["bf16_tflops_sustained"], 4), "rows": R, "vocab": V,
+            "hidden": hidden, "cublas_gemm_ms": round(gemm, 4),
+            "cublas_tflops": round(flops / (gemm * 1e-3) / 1e12, 1), "cublas_gemm_plus_edit_decide_ms": round(unf, 4),
+            "note": "random bf16 weights; roofline bound: tensor"}
 
 
 class RefreshBuffers:

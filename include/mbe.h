@@ -331,8 +331,8 @@ mbe_status mbe_kv_window_write(const void* k_win, const void* v_win, void* k_cac
  *   edit_mask, confidence, argmax_or_null: as in mbe_edit_decide
  *   entropy_or_null fp32 [rows]: -sum_v p_v ln p_v
  *   workspace: device buffer of at least mbe_lm_head_workspace_size(rows,
- *     vocab) bytes, 16-byte aligned (per-row partial states of 2048-token
- *     vocabulary chunks).
+ *     vocab) bytes, 16-byte aligned (per-row partial states of the vocabulary
+ *     chunks: 16 bytes per row and 256 tokens at most).
  * The logits are accumulated in fp32 on the tensor cores (bf16 products), so
  * they differ from exact dot products by fp32 rounding of the running sums;
  * decisions are taken on those fp32 values. hidden_dim must be a multiple of 8

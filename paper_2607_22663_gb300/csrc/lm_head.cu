@@ -13,8 +13,9 @@
 //   warps 4-7   epilogue: thread = accumulator row = TMEM lane; reads its
 //               row 32 columns at a time and updates the row state, so the
 //               epilogue of one tile overlaps the MMAs of the next.
-// A work unit is (128-row block, 2048-column vocabulary chunk); units go
-// chunk-major so the CTAs running at the same time share a weight chunk in L2.
+// A work unit is (128-row block, vocabulary chunk of 1..8 tiles of 256
+// columns, chosen so every SM gets at least ~16 units); units go chunk-major so
+// the CTAs running at the same time share a weight chunk in L2.
 // Each unit writes one partial state per row. lm_head_decide_kernel merges a
 // row's partial states and applies the threshold-and-replace rule.
 #include <cuda_bf16.h>
@@ -35,7 +36,8 @@ using namespace rows;
 
 constexpr int kBM = 128, kBN = 256, kBK = 64;
 constexpr int kStages = 4;
-constexpr int kTilesPerUnit = 8;  // 2048 vocabulary columns per work unit
+constexpr int kMaxTilesPerUnit = 8;  // up to 2048 vocabulary columns per work unit
+constexpr int kUnitsPerSm = 16;      // fewer tiles per unit until every SM gets this many units
 constexpr int kThreads = 256;
 constexpr uint32_t kABytes = kBM * kBK * 2;  // 16 KB
 constexpr uint32_t kBBytes = kBN * kBK * 2;  // 32 KB
@@ -51,6 +53,7 @@ struct Partial {
 
 struct Params {
   int rows, vocab, d;
+  int tpu;  // tiles per unit
   int n_m, n_chunks, n_units, n_kb;
   Partial* part;  // [rows, n_chunks]
 };
@@ -122,8 +125,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tmem_base_s;
-  // the tiles of unit u: columns [chunk * 2048, ...) up to the vocabulary end
-  auto tiles_of = [&](int chunk) { return min(kTilesPerUnit, (p.vocab + kBN - 1) / kBN - chunk * kTilesPerUnit); };
+  // tiles of a chunk: columns [chunk * tpu * 256, ...) up to the vocabulary end
+  auto tiles_of = [&](int chunk) { return min(p.tpu, (p.vocab + kBN - 1) / kBN - chunk * p.tpu); };
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
@@ -136,7 +139,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int chunk = u / p.n_m, mt = u - chunk * p.n_m;
         const int nt_count = tiles_of(chunk);
         for (int t = 0; t < nt_count && ok; ++t) {
-          const int nt = chunk * kTilesPerUnit + t;
+          const int nt = chunk * p.tpu + t;
           for (int kb = 0; kb < p.n_kb; ++kb, ++it) {
             const uint32_t s = it % kStages;
             if (it >= kStages && !mbar_wait(bar(bars.empty[s]), ((it / kStages) - 1) & 1, abort_flag)) {
@@ -219,7 +222,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.acc_full[acc]), (tile >> 1) & 1, abort_flag));
         if (!ok) break;
         tc_fence_after();
-        const int col0 = (chunk * kTilesPerUnit + t) * kBN;
+        const int col0 = (chunk * p.tpu + t) * kBN;
 #pragma unroll 1
         for (int c = 0; c < kBN / 32; ++c) {
           uint32_t v[32];
@@ -283,9 +286,15 @@ __global__ void __launch_bounds__(256) lm_head_decide_kernel(const Partial* __re
   if (entropy) entropy[row] = logf(st.s) - 0.6931471805599453f * st.t / st.s;
 }
 
-int num_chunks(int vocab) {
+int tiles_per_unit(int rows, int vocab, int num_sms) {
+  const int64_t tiles = static_cast<int64_t>((rows + kBM - 1) / kBM) * ((vocab + kBN - 1) / kBN);
+  const int64_t t = tiles / (static_cast<int64_t>(kUnitsPerSm) * num_sms);
+  return static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(kMaxTilesPerUnit, t)));
+}
+
+int num_chunks(int vocab, int tpu) {
   const int tiles = (vocab + kBN - 1) / kBN;
-  return (tiles + kTilesPerUnit - 1) / kTilesPerUnit;
+  return (tiles + tpu - 1) / tpu;
 }
 
 struct DeviceState {
@@ -314,7 +323,8 @@ DeviceState* device_state(int dev) {
 
 extern "C" size_t mbe_lm_head_workspace_size(int32_t rows, int32_t vocab) {
   if (rows <= 0 || vocab <= 0) return 0;
-  return static_cast<size_t>(rows) * mbe::lmh::num_chunks(vocab) * sizeof(mbe::lmh::Partial);
+  // sized for one tile per unit, the finest split the kernel uses
+  return static_cast<size_t>(rows) * mbe::lmh::num_chunks(vocab, 1) * sizeof(mbe::lmh::Partial);
 }
 
 extern "C" mbe_status mbe_lm_head_edit_decide(const void* hidden, const void* weight, int32_t rows, int32_t vocab,
@@ -362,7 +372,8 @@ extern "C" mbe_status mbe_lm_head_edit_decide(const void* hidden, const void* we
   p.vocab = vocab;
   p.d = hidden_dim;
   p.n_m = (rows + kBM - 1) / kBM;
-  p.n_chunks = num_chunks(vocab);
+  p.tpu = tiles_per_unit(rows, vocab, ds->num_sms);
+  p.n_chunks = num_chunks(vocab, p.tpu);
   p.n_units = p.n_m * p.n_chunks;
   p.n_kb = (hidden_dim + kBK - 1) / kBK;
   p.part = static_cast<Partial*>(workspace);
