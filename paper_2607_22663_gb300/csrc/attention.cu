@@ -44,6 +44,7 @@ constexpr int kTileKeys = 128;      // keys per K/V tile
 constexpr int kTileRows = 128;      // packed query rows per tile (= TMEM lanes)
 constexpr int kUnitRows = 256;      // packed query rows per work unit (two tiles)
 constexpr int kThreads = 384;       // 12 warps
+constexpr int kMergeThreads = 256;  // 8 rows per merge CTA
 constexpr int kMinChunk = 8;        // fewest key tiles in a split piece
 constexpr int kSplitFactor = 4;     // most pieces per SM when splitting (bounds the workspace)
 constexpr int kMaxGroupedSlabs = 8; // slabs of one (sequence, KV head) kept adjacent in the work list
@@ -231,12 +232,15 @@ __global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p
     }
     atomicAdd(&hist[b], count);
   };
-  for (int s = tid; s < p.batch; s += blockDim.x) {
+  // one thread per (sequence, KV head) pair, so that few long sequences still
+  // spread their pieces over many threads
+  for (int sg = tid; sg < p.batch * p.Hkv; sg += blockDim.x) {
+    const int s = sg / p.Hkv, g = sg - s * p.Hkv;
     const int P = p.prefix_len[s], W = p.window_len[s], mode = p.mask_mode[s];
     if (!seq_ok(p, s, P, W, mode)) continue;
     const int slabs = (W * p.G + kUnitRows - 1) / kUnitRows;
     const int ng = slabs <= kMaxGroupedSlabs ? slabs : 1;  // slabs per piece
-    for (int g = 0; g < p.Hkv; ++g) {
+    {
       for (int s0 = 0; s0 < slabs; s0 += ng) {
         const int cnt = min(ng, slabs - s0);
         int T[kMaxGroupedSlabs], n[kMaxGroupedSlabs], slot0[kMaxGroupedSlabs];
@@ -852,8 +856,12 @@ struct MergeParams {
   int Hq, G;
 };
 
+// One warp per packed query row of a split group: lane l holds D/32
+// consecutive output columns, so every partial row is read as one coalesced
+// 4 D-byte line; the weights 2^(lse_k - M) are common to the row.
 template <int D>
-__device__ __forceinline__ void merge_group_row(const MergeParams& p, const MergeGroup& grp, int r) {
+__device__ __forceinline__ void merge_row_warp(const MergeParams& p, const MergeGroup& grp, int r, int lane) {
+  constexpr int kPer = D / 32;  // 4 for D = 128, 2 for D = 64
   const int R = grp.row0 + r;
   const int qi = R / p.G, hh = R - qi * p.G;
   if (qi >= grp.window) return;
@@ -863,48 +871,52 @@ __device__ __forceinline__ void merge_group_row(const MergeParams& p, const Merg
   for (int k = 0; k < grp.n_splits; ++k)
     M = fmaxf(M, p.part_lse[static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r]);
   float wsum = 0.f;
-  float acc[D];
+  float acc[kPer];
 #pragma unroll
-  for (int d = 0; d < D; ++d) acc[d] = 0.f;
+  for (int d = 0; d < kPer; ++d) acc[d] = 0.f;
   for (int k = 0; k < grp.n_splits; ++k) {
     const float lk = p.part_lse[static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r];
     const float w = (lk == neg_inf()) ? 0.f : ex2f(lk - M);
     if (w == 0.f) continue;
     wsum += w;
-    const float4* src =
-        reinterpret_cast<const float4*>(p.part_o + (static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r) * D);
-#pragma unroll
-    for (int d4 = 0; d4 < D / 4; ++d4) {
-      const float4 v = src[d4];
-      acc[4 * d4] += w * v.x;
-      acc[4 * d4 + 1] += w * v.y;
-      acc[4 * d4 + 2] += w * v.z;
-      acc[4 * d4 + 3] += w * v.w;
+    const float* src = p.part_o + (static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r) * D + lane * kPer;
+    if constexpr (kPer == 4) {
+      const float4 v = *reinterpret_cast<const float4*>(src);
+      acc[0] += w * v.x;
+      acc[1] += w * v.y;
+      acc[2] += w * v.z;
+      acc[3] += w * v.w;
+    } else {
+      const float2 v = *reinterpret_cast<const float2*>(src);
+      acc[0] += w * v.x;
+      acc[1] += w * v.y;
     }
   }
   const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
   const int64_t orow = static_cast<int64_t>(cu + qi) * p.Hq + grp.kv_head * p.G + hh;
-  uint4* dst = reinterpret_cast<uint4*>(p.out + orow * D);
-#pragma unroll
-  for (int d = 0; d < D; d += 8)
-    dst[d / 8] = make_uint4(pack_bf16x2(acc[d] * inv, acc[d + 1] * inv), pack_bf16x2(acc[d + 2] * inv, acc[d + 3] * inv),
-                            pack_bf16x2(acc[d + 4] * inv, acc[d + 5] * inv), pack_bf16x2(acc[d + 6] * inv, acc[d + 7] * inv));
-  if (p.lse) p.lse[orow] = (wsum > 0.f ? M + __log2f(wsum) : neg_inf()) * 0.6931471805599453f;
+  __nv_bfloat16* dst = p.out + orow * D + lane * kPer;
+  if constexpr (kPer == 4)
+    *reinterpret_cast<uint2*>(dst) = make_uint2(pack_bf16x2(acc[0] * inv, acc[1] * inv), pack_bf16x2(acc[2] * inv, acc[3] * inv));
+  else
+    *reinterpret_cast<uint32_t*>(dst) = pack_bf16x2(acc[0] * inv, acc[1] * inv);
+  if (p.lse && lane == 0) p.lse[orow] = (wsum > 0.f ? M + __log2f(wsum) : neg_inf()) * 0.6931471805599453f;
 }
 
-// One CTA per split group (looping when there are more groups than CTAs),
-// one thread per packed query row.
+// Grid-stride over (split group, row) items, one warp per item.
 template <int D>
-__global__ void __launch_bounds__(kUnitRows) attn_merge_kernel(const MergeParams p) {
+__global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const MergeParams p) {
   // the attention kernel has finished: re-arm the work counter so that the same
   // plan can serve the next run
   if (blockIdx.x == 0 && threadIdx.x == 0) p.hdr->counter = 0;
   if (!sig_equal(p.hdr->sig, p.sig)) return;
-  const int n_groups = p.hdr->n_groups;
-  for (int gi = blockIdx.x; gi < n_groups; gi += gridDim.x) {
-    const MergeGroup grp = p.groups[gi];
+  const int64_t n_items = static_cast<int64_t>(p.hdr->n_groups) * kUnitRows;
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = static_cast<int64_t>(gridDim.x) * (kMergeThreads / 32);
+  for (int64_t it = static_cast<int64_t>(blockIdx.x) * (kMergeThreads / 32) + threadIdx.x / 32; it < n_items;
+       it += warps) {
+    const MergeGroup grp = p.groups[it / kUnitRows];
     if (grp.seq < 0 || grp.seq >= p.batch) continue;
-    merge_group_row<D>(p, grp, threadIdx.x);
+    merge_row_warp<D>(p, grp, static_cast<int>(it % kUnitRows), lane);
   }
 }
 
@@ -1022,8 +1034,9 @@ mbe_status run(const void* q, const void* k_win, const void* v_win, const void* 
   if (launch_status("attn_kernel launch") != MBE_OK) return MBE_ERR_CUDA;
   MergeParams mp{sig, batch, total_q_tokens, hdr, reinterpret_cast<const MergeGroup*>(ws + L.groups), ap.part_o,
                  ap.part_lse, cu_window, ap.out, lse, Hq, G};
-  const int64_t merge_grid = std::min<int64_t>(L.max_groups, 2 * di->num_sms);
-  attn_merge_kernel<D><<<static_cast<unsigned>(merge_grid), kUnitRows, 0, stream>>>(mp);
+  const int64_t merge_grid =
+      std::max<int64_t>(1, std::min<int64_t>(L.max_groups * (kUnitRows / (kMergeThreads / 32)), 2 * di->num_sms));
+  attn_merge_kernel<D><<<static_cast<unsigned>(merge_grid), kMergeThreads, 0, stream>>>(mp);
   if (launch_status("attn_merge_kernel launch") != MBE_OK) return MBE_ERR_CUDA;
   return MBE_OK;
 }
