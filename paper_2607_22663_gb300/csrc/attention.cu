@@ -867,29 +867,45 @@ __device__ __forceinline__ void merge_row_warp(const MergeParams& p, const Merge
   if (qi >= grp.window) return;
   const int cu = p.cu_window[grp.seq];
   if (cu < 0 || static_cast<int64_t>(cu) + grp.window > p.total_tokens) return;
+  const float* lse = p.part_lse + static_cast<int64_t>(grp.slot_base) * kUnitRows + r;  // split k at k * kUnitRows
+  const float* part = p.part_o + (static_cast<int64_t>(grp.slot_base) * kUnitRows + r) * D + lane * kPer;
+  const int n = grp.n_splits;
+  // the row's largest log-sum-exp: lanes read the splits' values in parallel
   float M = neg_inf();
-  for (int k = 0; k < grp.n_splits; ++k)
-    M = fmaxf(M, p.part_lse[static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r]);
+  for (int k = lane; k < n; k += 32) M = fmaxf(M, lse[static_cast<int64_t>(k) * kUnitRows]);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
   float wsum = 0.f;
   float acc[kPer];
 #pragma unroll
   for (int d = 0; d < kPer; ++d) acc[d] = 0.f;
-  for (int k = 0; k < grp.n_splits; ++k) {
-    const float lk = p.part_lse[static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r];
-    const float w = (lk == neg_inf()) ? 0.f : ex2f(lk - M);
-    if (w == 0.f) continue;
-    wsum += w;
-    const float* src = p.part_o + (static_cast<int64_t>(grp.slot_base + k) * kUnitRows + r) * D + lane * kPer;
-    if constexpr (kPer == 4) {
-      const float4 v = *reinterpret_cast<const float4*>(src);
-      acc[0] += w * v.x;
-      acc[1] += w * v.y;
-      acc[2] += w * v.z;
-      acc[3] += w * v.w;
-    } else {
-      const float2 v = *reinterpret_cast<const float2*>(src);
-      acc[0] += w * v.x;
-      acc[1] += w * v.y;
+  // four splits per step, their loads issued before any is used
+  for (int k0 = 0; k0 < n; k0 += 4) {
+    float lk[4], v[4][kPer];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int k = k0 + u;
+      lk[u] = neg_inf();
+#pragma unroll
+      for (int d = 0; d < kPer; ++d) v[u][d] = 0.f;
+      if (k < n) {
+        lk[u] = lse[static_cast<int64_t>(k) * kUnitRows];
+        const float* src = part + static_cast<int64_t>(k) * kUnitRows * D;
+        if constexpr (kPer == 4) {
+          const float4 x = *reinterpret_cast<const float4*>(src);
+          v[u][0] = x.x; v[u][1] = x.y; v[u][2] = x.z; v[u][3] = x.w;
+        } else {
+          const float2 x = *reinterpret_cast<const float2*>(src);
+          v[u][0] = x.x; v[u][1] = x.y;
+        }
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const float w = (lk[u] == neg_inf()) ? 0.f : ex2f(lk[u] - M);
+      wsum += w;
+#pragma unroll
+      for (int d = 0; d < kPer; ++d) acc[d] += w * v[u][d];
     }
   }
   const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
