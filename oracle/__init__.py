@@ -16,6 +16,9 @@ path computes, written from the paper (arXiv 2607.22663):
   recompute problem per changed block, laid out as a ragged batch.
 * ``lm_head_logits``    -- the LM-head projection whose rows the T2T rule
   reads (float64 logits for ``edit_decide`` / ``denoise_update``).
+* ``sft_block_mask``, ``block_mask_attention``, ``block_mask_attention_bwd`` --
+  the cross-block training mask of Multi-Block Edit SFT (Sec. 3) and attention
+  (forward and gradients) under a block mask.
 
 Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
 ``bench.py`` may import it. It shares no code with the CUDA library and never
@@ -77,6 +80,12 @@ def _load():
         lib.oracle_kv_window_write.argtypes = [P, P, P, P, P, i32, P, P, P, P, i32, i32, i32, i32, i32, i32, i32]
         lib.oracle_lm_head_logits.restype = ctypes.c_int
         lib.oracle_lm_head_logits.argtypes = [P, P, i32, i32, i32, i32, P, P]
+        lib.oracle_sft_block_mask.restype = ctypes.c_int
+        lib.oracle_sft_block_mask.argtypes = [i32, i32, i32, i32, P]
+        lib.oracle_block_mask_attention.restype = ctypes.c_int
+        lib.oracle_block_mask_attention.argtypes = [P, P, P, i32, i32, i32, i32, i32, P, i32, f64, P, P]
+        lib.oracle_block_mask_attention_bwd.restype = ctypes.c_int
+        lib.oracle_block_mask_attention_bwd.argtypes = [P, P, P, P, i32, i32, i32, i32, i32, P, i32, f64, P, P, P]
         lib.oracle_refresh_plan.restype = ctypes.c_int
         lib.oracle_refresh_plan.argtypes = [P, i32, P, P, P, P, i32, i32, i32, i32, P, P, P, P, P, P, P]
         _lib = lib
@@ -275,3 +284,51 @@ def lm_head_logits(hidden, weight, rows=None):
     rc = lib.oracle_lm_head_logits(_ptr(h), _ptr(w), R, V, d, -1 if sel is None else n, _ptr(sel), _ptr(out))
     _check(rc)
     return out
+
+
+def sft_block_mask(n_prompt_blocks, n_blocks, K, words_per_row=None):
+    """Cross-block SFT mask (Sec. 3) as uint32 bits [nb, words_per_row]."""
+    lib = _load()
+    nb = n_prompt_blocks + 2 * n_blocks
+    wpr = words_per_row or max(1, (nb + 31) // 32)
+    m = np.zeros((nb, wpr), dtype=np.uint32)
+    _check(lib.oracle_sft_block_mask(n_prompt_blocks, n_blocks, K, wpr, _ptr(m)))
+    return m
+
+
+def mask_bits_to_dense(mask, nb):
+    """Boolean [nb, nb] view of a uint32 bit mask."""
+    m = np.asarray(mask, dtype=np.uint32)
+    cols = np.arange(nb)
+    return ((m[:, cols // 32] >> (cols % 32).astype(np.uint32)) & 1).astype(bool)[:nb]
+
+
+def block_mask_attention(q, k, v, block_size, mask, scale=None):
+    """Attention of one sequence under a block mask, float64 (out [T,Hq,D], lse [T,Hq])."""
+    lib = _load()
+    q, k, v = _c(q, np.uint16), _c(k, np.uint16), _c(v, np.uint16)
+    T, Hq, D = q.shape
+    Hkv = k.shape[1]
+    m = _c(mask, np.uint32)
+    scale = 1.0 / np.sqrt(D) if scale is None else scale
+    out = np.zeros((T, Hq, D))
+    lse = np.zeros((T, Hq))
+    _check(lib.oracle_block_mask_attention(_ptr(q), _ptr(k), _ptr(v), T, Hq, Hkv, D, block_size, _ptr(m), m.shape[1],
+                                           float(scale), _ptr(out), _ptr(lse)))
+    return out, lse
+
+
+def block_mask_attention_bwd(q, k, v, dout, block_size, mask, scale=None):
+    """Gradients (dq [T,Hq,D], dk, dv [T,Hkv,D]) of block-masked attention, float64."""
+    lib = _load()
+    q, k, v, do = _c(q, np.uint16), _c(k, np.uint16), _c(v, np.uint16), _c(dout, np.uint16)
+    T, Hq, D = q.shape
+    Hkv = k.shape[1]
+    m = _c(mask, np.uint32)
+    scale = 1.0 / np.sqrt(D) if scale is None else scale
+    dq = np.zeros((T, Hq, D))
+    dk = np.zeros((T, Hkv, D))
+    dv = np.zeros((T, Hkv, D))
+    _check(lib.oracle_block_mask_attention_bwd(_ptr(q), _ptr(k), _ptr(v), _ptr(do), T, Hq, Hkv, D, block_size, _ptr(m),
+                                               m.shape[1], float(scale), _ptr(dq), _ptr(dk), _ptr(dv)))
+    return dq, dk, dv

@@ -550,3 +550,193 @@ int oracle_lm_head_logits(const uint16_t* hidden, const uint16_t* weight, int32_
   free(hrow);
   return ORC_OK;
 }
+
+/*
+ * Cross-block attention mask of Multi-Block Edit SFT (Sec. 3, "Cross-block
+ * attention mask"), at block granularity. The training sequence is
+ * [prompt blocks 0..Np-1 | noisy blocks n_0..n_{N-1} | clean blocks c_0..c_{N-1}],
+ * block b = Np + i for n_i and Np + N + j for c_j. Links (reading of the paper;
+ * its supplement with the exact construction is not available):
+ *   prompt -> prompt (all prompt blocks; prompt tokens are their own category)
+ *   n_i -> prompt, n_i (NN), c_j for j < i (NC), c_j for i < j <= i+K-1 (NF)
+ *   c_j -> prompt, c_j, c_k for k <= j-K (CC whose target is not reachable by
+ *          a noisy block that sees c_j), n_i for j-K+1 <= i <= j-1 (CN)
+ * With K = 1 this is the standard block-diffusion SFT mask (NN, NC, block-causal
+ * CC). mask: nb = Np + 2N rows of words_per_row 32-bit words; bit k of row q is
+ * set iff block q attends to block k.
+ */
+int oracle_sft_block_mask(int32_t n_prompt_blocks, int32_t n_blocks, int32_t K, int32_t words_per_row,
+                          uint32_t* mask) {
+  const int32_t Np = n_prompt_blocks, N = n_blocks, nb = Np + 2 * N;
+  if (Np < 0 || N < 0 || K < 1 || words_per_row * 32 < nb) return ORC_BAD_ARG;
+  memset(mask, 0, sizeof(uint32_t) * (size_t)nb * (size_t)words_per_row);
+#define ORC_SET(q, k) (mask[(int64_t)(q) * words_per_row + (k) / 32] |= 1u << ((k) % 32))
+  for (int32_t q = 0; q < nb; ++q)
+    for (int32_t p = 0; p < Np; ++p) ORC_SET(q, p);
+  for (int32_t i = 0; i < N; ++i) {
+    const int32_t q = Np + i;
+    ORC_SET(q, q);
+    for (int32_t j = 0; j < N; ++j)
+      if (j < i || (j > i && j <= i + K - 1)) ORC_SET(q, Np + N + j);
+  }
+  for (int32_t j = 0; j < N; ++j) {
+    const int32_t q = Np + N + j;
+    ORC_SET(q, q);
+    for (int32_t k = 0; k <= j - K; ++k) ORC_SET(q, Np + N + k);
+    for (int32_t i = j - K + 1; i <= j - 1; ++i)
+      if (i >= 0) ORC_SET(q, Np + i);
+  }
+#undef ORC_SET
+  return ORC_OK;
+}
+
+static int mask_bit(const uint32_t* mask, int32_t words_per_row, int32_t qb, int32_t kb) {
+  return (mask[(int64_t)qb * words_per_row + kb / 32] >> (kb % 32)) & 1u;
+}
+
+/*
+ * Attention of one training sequence under a block mask: query token i (block
+ * i / B) attends to key token j iff bit (i / B, j / B) of the mask is set.
+ * q [T, Hq, D], k/v [T, Hkv, D] bf16; query head h uses KV head h / (Hq/Hkv).
+ * out [T, Hq, D] and lse [T, Hq] (natural log) in double; a row that sees no
+ * key gets out = 0 and lse = -inf.
+ */
+int oracle_block_mask_attention(const uint16_t* q, const uint16_t* k, const uint16_t* v, int32_t T, int32_t Hq,
+                                int32_t Hkv, int32_t D, int32_t B, const uint32_t* mask, int32_t words_per_row,
+                                double scale, double* out, double* lse) {
+  if (T < 0 || Hq <= 0 || Hkv <= 0 || Hq % Hkv != 0 || D <= 0 || B <= 0) return ORC_BAD_ARG;
+  const int32_t G = Hq / Hkv;
+  int status = ORC_OK;
+#pragma omp parallel for schedule(dynamic)
+  for (int64_t ih = 0; ih < (int64_t)T * Hq; ++ih) {
+    const int32_t i = (int32_t)(ih / Hq), h = (int32_t)(ih % Hq), g = h / G;
+    double* z = (double*)malloc(sizeof(double) * (size_t)(T > 0 ? T : 1));
+    if (!z) {
+#pragma omp atomic write
+      status = ORC_NOMEM;
+      continue;
+    }
+    double m = -INFINITY;
+    for (int32_t j = 0; j < T; ++j) {
+      if (!mask_bit(mask, words_per_row, i / B, j / B)) {
+        z[j] = -INFINITY;
+        continue;
+      }
+      double s = 0.0;
+      for (int32_t d = 0; d < D; ++d)
+        s += bf16_to_double(q[((int64_t)i * Hq + h) * D + d]) * bf16_to_double(k[((int64_t)j * Hkv + g) * D + d]);
+      z[j] = s * scale;
+      if (z[j] > m) m = z[j];
+    }
+    double* o = out + ((int64_t)i * Hq + h) * D;
+    for (int32_t d = 0; d < D; ++d) o[d] = 0.0;
+    if (m == -INFINITY) {
+      lse[(int64_t)i * Hq + h] = -INFINITY;
+      free(z);
+      continue;
+    }
+    double zs = 0.0;
+    for (int32_t j = 0; j < T; ++j) {
+      if (z[j] == -INFINITY) continue;
+      const double p = exp(z[j] - m);
+      zs += p;
+      for (int32_t d = 0; d < D; ++d) o[d] += p * bf16_to_double(v[((int64_t)j * Hkv + g) * D + d]);
+    }
+    for (int32_t d = 0; d < D; ++d) o[d] /= zs;
+    lse[(int64_t)i * Hq + h] = m + log(zs);
+    free(z);
+  }
+  return status;
+}
+
+/*
+ * Gradients of the block-masked attention above for an upstream gradient dO
+ * (bf16 [T, Hq, D]), from the definitions, in double: with P the attention
+ * probabilities (recomputed from q, k and the mask),
+ *   dV_g = sum over the G heads of g of P^T dO
+ *   dP   = dO V^T,  delta_i = sum_j P_ij dP_ij  (= dO_i . O_i)
+ *   dS   = P o (dP - delta)
+ *   dQ   = scale * dS K,  dK_g = scale * sum over the heads of g of dS^T Q
+ * dq [T, Hq, D], dk / dv [T, Hkv, D] are written (overwritten) in double.
+ */
+int oracle_block_mask_attention_bwd(const uint16_t* q, const uint16_t* k, const uint16_t* v, const uint16_t* dout,
+                                    int32_t T, int32_t Hq, int32_t Hkv, int32_t D, int32_t B, const uint32_t* mask,
+                                    int32_t words_per_row, double scale, double* dq, double* dk, double* dv) {
+  if (T < 0 || Hq <= 0 || Hkv <= 0 || Hq % Hkv != 0 || D <= 0 || B <= 0) return ORC_BAD_ARG;
+  const int32_t G = Hq / Hkv;
+  memset(dk, 0, sizeof(double) * (size_t)T * Hkv * D);
+  memset(dv, 0, sizeof(double) * (size_t)T * Hkv * D);
+  memset(dq, 0, sizeof(double) * (size_t)T * Hq * D);
+  int status = ORC_OK;
+  /* one KV head at a time so that dK / dV accumulate without races */
+  for (int32_t g = 0; g < Hkv; ++g) {
+    for (int32_t hh = 0; hh < G; ++hh) {
+      const int32_t h = g * G + hh;
+      double* P = (double*)malloc(sizeof(double) * (size_t)T * (size_t)(T > 0 ? T : 1));
+      double* dS = (double*)malloc(sizeof(double) * (size_t)T * (size_t)(T > 0 ? T : 1));
+      if (!P || !dS) {
+        free(P);
+        free(dS);
+        return ORC_NOMEM;
+      }
+#pragma omp parallel for schedule(dynamic)
+      for (int32_t i = 0; i < T; ++i) {
+        double* Pi = P + (int64_t)i * T;
+        double m = -INFINITY;
+        for (int32_t j = 0; j < T; ++j) {
+          if (!mask_bit(mask, words_per_row, i / B, j / B)) {
+            Pi[j] = -INFINITY;
+            continue;
+          }
+          double s = 0.0;
+          for (int32_t d = 0; d < D; ++d)
+            s += bf16_to_double(q[((int64_t)i * Hq + h) * D + d]) * bf16_to_double(k[((int64_t)j * Hkv + g) * D + d]);
+          Pi[j] = s * scale;
+          if (Pi[j] > m) m = Pi[j];
+        }
+        double zs = 0.0;
+        for (int32_t j = 0; j < T; ++j) {
+          Pi[j] = (m == -INFINITY || Pi[j] == -INFINITY) ? 0.0 : exp(Pi[j] - m);
+          zs += Pi[j];
+        }
+        for (int32_t j = 0; j < T; ++j) Pi[j] = zs > 0.0 ? Pi[j] / zs : 0.0;
+        /* dP_ij = dO_i . V_j; delta_i = sum_j P_ij dP_ij */
+        double* dSi = dS + (int64_t)i * T;
+        double delta = 0.0;
+        for (int32_t j = 0; j < T; ++j) {
+          double dp = 0.0;
+          if (Pi[j] != 0.0)
+            for (int32_t d = 0; d < D; ++d)
+              dp += bf16_to_double(dout[((int64_t)i * Hq + h) * D + d]) * bf16_to_double(v[((int64_t)j * Hkv + g) * D + d]);
+          dSi[j] = dp;
+          delta += Pi[j] * dp;
+        }
+        for (int32_t j = 0; j < T; ++j) dSi[j] = Pi[j] * (dSi[j] - delta);
+        /* dQ_i = scale * sum_j dS_ij K_j */
+        for (int32_t d = 0; d < D; ++d) {
+          double acc = 0.0;
+          for (int32_t j = 0; j < T; ++j)
+            if (dSi[j] != 0.0) acc += dSi[j] * bf16_to_double(k[((int64_t)j * Hkv + g) * D + d]);
+          dq[((int64_t)i * Hq + h) * D + d] = scale * acc;
+        }
+      }
+      /* dV_j += sum_i P_ij dO_i ; dK_j += scale * sum_i dS_ij Q_i */
+#pragma omp parallel for schedule(static)
+      for (int32_t j = 0; j < T; ++j) {
+        for (int32_t d = 0; d < D; ++d) {
+          double av = 0.0, ak = 0.0;
+          for (int32_t i = 0; i < T; ++i) {
+            const double p = P[(int64_t)i * T + j], ds = dS[(int64_t)i * T + j];
+            if (p != 0.0) av += p * bf16_to_double(dout[((int64_t)i * Hq + h) * D + d]);
+            if (ds != 0.0) ak += ds * bf16_to_double(q[((int64_t)i * Hq + h) * D + d]);
+          }
+          dv[((int64_t)j * Hkv + g) * D + d] += av;
+          dk[((int64_t)j * Hkv + g) * D + d] += scale * ak;
+        }
+      }
+      free(P);
+      free(dS);
+    }
+  }
+  return status;
+}
