@@ -20,8 +20,10 @@
  * with forced unmasking, entropies, changed blocks), the tail-entropy
  * window choice (mbe_tail_entropy_select: Eqs. 6-7), the targeted refresh of
  * the changed blocks (mbe_refresh_plan, mbe_gather_rows: Sec. 4.3), a
- * device-side loop over editing passes (mbe_pass_loop_*: Sec. 4.1) and the
- * LM-head projection fused with the edit decision (mbe_lm_head_edit_decide).
+ * device-side loop over editing passes (mbe_pass_loop_*: Sec. 4.1), the
+ * LM-head projection fused with the edit decision (mbe_lm_head_edit_decide)
+ * and the cross-block training attention of Multi-Block Edit SFT
+ * (mbe_sft_block_mask, mbe_block_mask_attention: Sec. 3).
  *
  * Conventions shared by every entry point
  *   - All pointers are DEVICE pointers unless stated otherwise; the caller
@@ -63,8 +65,9 @@ typedef enum {
 
 /* Attention mask of the window part (Sec. 2.2 and Eq. 5). */
 typedef enum {
-  MBE_BLOCK_CAUSAL = 0,              /* window query i sees window key j iff floor(j/B) <= floor(i/B) */
-  MBE_MULTI_BLOCK_BIDIRECTIONAL = 1  /* every window query sees every window key (full attention in W_j) */
+  MBE_BLOCK_CAUSAL = 0,               /* window query i sees window key j iff floor(j/B) <= floor(i/B) */
+  MBE_MULTI_BLOCK_BIDIRECTIONAL = 1,  /* every window query sees every window key (full attention in W_j) */
+  MBE_BLOCK_MASK = 2                  /* an explicit block-level mask (mbe_block_mask_attention only) */
 } mbe_mask_mode;
 
 typedef enum { MBE_F32 = 0, MBE_BF16 = 1 } mbe_dtype;
@@ -317,6 +320,55 @@ mbe_status mbe_kv_window_write(const void* k_win, const void* v_win, void* k_cac
                                const uint8_t* block_write_mask_or_null, int32_t max_blocks_per_seq, int32_t batch,
                                int32_t max_window, int32_t num_kv_heads, int32_t head_dim, int32_t block_size,
                                int32_t page_size, cudaStream_t stream);
+
+/*
+ * mbe_sft_block_mask -- the cross-block attention mask of Multi-Block Edit SFT.
+ * Paper: Sec. 3 ("Cross-block attention mask"): standard block SFT links
+ * noisy-to-noisy (NN), noisy-to-clean-prefix (NC) and clean-to-clean (CC);
+ * MBE adds noisy-sees-forward (NF) links from noisy block i to clean blocks
+ * i+1 .. i+K-1 and clean-sees-noisy (CN) links, and removes the CC links a
+ * noisy block could use to reach its own clean block; prompt tokens are their
+ * own category. The paper defers the exact construction to a supplement that
+ * is not available; this follows the reading below. Sequence s is laid out as
+ * [n_prompt_blocks[s] prompt blocks | N = n_blocks[s] noisy blocks n_i |
+ * N clean blocks c_j]; bit k of row q is set iff block q attends to block k:
+ *   prompt -> prompt;  n_i -> prompt, n_i, c_j (j < i), c_j (i < j <= i+K-1);
+ *   c_j -> prompt, c_j, c_k (k <= j-K), n_i (j-K+1 <= i <= j-1).
+ * K = 1 gives the standard block-diffusion SFT mask. mask uint32 [batch,
+ * mask_rows, mask_words] as mbe_block_mask_attention reads it; rows past the
+ * sequence's blocks are zero. A sequence with more than mask_rows blocks gets
+ * zero rows and sets MBE_DEVERR_LENGTH.
+ * Errors: MBE_ERR_INVALID_ARG (K < 1, mask_words * 32 < mask_rows, null
+ * pointers), MBE_ERR_UNSUPPORTED (batch > 65535), MBE_ERR_CUDA.
+ */
+mbe_status mbe_sft_block_mask(const int32_t* n_prompt_blocks, const int32_t* n_blocks, int32_t K, int32_t batch,
+                              int32_t mask_rows, int32_t mask_words, uint32_t* mask, cudaStream_t stream);
+
+/*
+ * mbe_block_mask_attention -- attention of whole training sequences under a
+ * block-level mask, the forward of Multi-Block Edit SFT's cross-block attention
+ * (Sec. 3, "Cross-block attention mask"; build the mask with mbe_sft_block_mask).
+ * Sequence s owns tokens cu_seqlens[s] .. cu_seqlens[s] + seq_len[s] - 1 of
+ *   q bf16 [total_tokens, num_q_heads, head_dim], k, v bf16 [total_tokens, num_kv_heads, head_dim];
+ * query token i (block i / block_size) attends to key token j iff bit
+ * (j / block_size) % 32 of word (j / block_size) / 32 of mask row i / block_size is set:
+ *   mask uint32 [batch, mask_rows, mask_words] (mask_rows >= ceil(max_seq_len /
+ *   block_size), mask_words * 32 >= mask_rows).
+ * out bf16 [total_tokens, num_q_heads, head_dim]; lse_or_null fp32 [total_tokens,
+ * num_q_heads] (natural-log sum of exp of the scaled scores; -inf and a zero
+ * output row for a token that sees no key). softmax_scale 0 means
+ * 1/sqrt(head_dim). Key tiles of 128 keys that no row of a 256-row work unit
+ * sees are skipped. block_size must be a power of two >= 8 and max_seq_len <=
+ * 65536; workspace as for mbe_window_attention_workspace_size(batch,
+ * num_q_heads, num_kv_heads, head_dim, max_seq_len, 0).
+ * Errors as mbe_window_attention.
+ */
+mbe_status mbe_block_mask_attention(const void* q, const void* k, const void* v, const int32_t* seq_len,
+                                    const int32_t* cu_seqlens, const uint32_t* mask, int32_t mask_rows,
+                                    int32_t mask_words, int32_t batch, int32_t total_tokens, int32_t num_q_heads,
+                                    int32_t num_kv_heads, int32_t head_dim, int32_t block_size, int32_t max_seq_len,
+                                    float softmax_scale, void* out, float* lse_or_null, void* workspace,
+                                    size_t workspace_bytes, cudaStream_t stream);
 
 /*
  * mbe_lm_head_edit_decide -- the LM-head projection fused with the edit

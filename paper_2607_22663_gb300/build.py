@@ -17,7 +17,7 @@ CSRC = PKG / "csrc"
 INCLUDE = ROOT / "include"
 BUILD = PKG / "_build"
 LIB = BUILD / "libmbe.so"
-SOURCES = ["attention.cu", "edit_decide.cu", "denoise.cu", "kv_write.cu", "refresh.cu", "lm_head.cu", "api.cu"]
+SOURCES = ["attention.cu", "edit_decide.cu", "denoise.cu", "kv_write.cu", "refresh.cu", "lm_head.cu", "train.cu", "api.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", str(INCLUDE)]
 

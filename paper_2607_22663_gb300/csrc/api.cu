@@ -16,8 +16,9 @@ extern "C" const char* mbe_last_error_string(void) { return mbe::g_last_error; }
 extern "C" mbe_status mbe_get_device_error(cudaStream_t stream, uint32_t* flags_or_null) {
   if (cudaStreamSynchronize(stream) != cudaSuccess) return MBE_ERR_CUDA;
   uint32_t bits = 0;
-  const uint32_t parts[6] = {mbe::edit_decide_take_error(), mbe::kv_write_take_error(), mbe::attention_take_error(),
-                             mbe::denoise_take_error(), mbe::refresh_take_error(), mbe::lm_head_take_error()};
+  const uint32_t parts[7] = {mbe::edit_decide_take_error(), mbe::kv_write_take_error(), mbe::attention_take_error(),
+                             mbe::denoise_take_error(),     mbe::refresh_take_error(),  mbe::lm_head_take_error(),
+                             mbe::train_take_error()};
   for (uint32_t v : parts) {
     if (v == 0xFFFFFFFFu) return MBE_ERR_CUDA;
     bits |= v;

@@ -45,6 +45,7 @@ constexpr int kTileRows = 128;      // packed query rows per tile (= TMEM lanes)
 constexpr int kUnitRows = 256;      // packed query rows per work unit (two tiles)
 constexpr int kThreads = 384;       // 12 warps
 constexpr int kMergeThreads = 256;  // 8 rows per merge CTA
+constexpr int kMaskTileWords = 16;   // block-mask mode: visible-tile bitmask of a unit (<= 512 key tiles)
 constexpr int kMinChunk = 8;        // fewest key tiles in a split piece
 constexpr int kSplitFactor = 4;     // most pieces per SM when splitting (bounds the workspace)
 constexpr int kMaxGroupedSlabs = 8; // slabs of one (sequence, KV head) kept adjacent in the work list
@@ -113,11 +114,12 @@ inline Layout make_layout(int batch, int Hq, int Hkv, int D, int max_window, int
 
 // ------------------------------------------------------------------ scheduler
 struct SchedParams {
-  const int32_t* prefix_len;
+  const int32_t* prefix_len;  // null: no prefix (block-mask mode)
   const int32_t* window_len;
-  const uint8_t* mask_mode;
+  const uint8_t* mask_mode;   // null: every sequence in block-mask mode
   const int32_t* cu_window;
   int batch, G, Hkv, block_size, max_window, max_prefix, num_sms, total_tokens;
+  bool block_mask;
   PlanSig sig;
   Header* hdr;
   WorkUnit* units_tmp;
@@ -127,6 +129,7 @@ struct SchedParams {
 };
 
 // Key tiles (prefix, then window) that packed query rows [row0, row0 + 256) need.
+// (block-mask mode: every window tile; the kernel skips the invisible ones)
 __device__ __forceinline__ int slab_tiles(int P, int W, int mode, int row0, int G, int B) {
   const int nP = (P + kTileKeys - 1) / kTileKeys;
   int lim = W;
@@ -137,10 +140,16 @@ __device__ __forceinline__ int slab_tiles(int P, int W, int mode, int row0, int 
   return nP + (lim + kTileKeys - 1) / kTileKeys;
 }
 
+__device__ __forceinline__ int seq_prefix(const SchedParams& p, int s) { return p.prefix_len ? p.prefix_len[s] : 0; }
+__device__ __forceinline__ int seq_mode(const SchedParams& p, int s) {
+  return p.mask_mode ? p.mask_mode[s] : MBE_BLOCK_MASK;
+}
+
 // A sequence is scheduled only if its lengths are within the declared bounds
 // and its window rows [cu, cu + W) lie inside the q/out tensors.
 __device__ __forceinline__ bool seq_ok(const SchedParams& p, int s, int P, int W, int mode) {
-  if (W < 0 || W > p.max_window || P < 0 || P > p.max_prefix || mode > 1) return false;
+  if (W < 0 || W > p.max_window || P < 0 || P > p.max_prefix || mode > 2) return false;
+  if ((mode == MBE_BLOCK_MASK) != p.block_mask) return false;
   const int cu = p.cu_window[s];
   return cu >= 0 && static_cast<int64_t>(cu) + W <= p.total_tokens;
 }
@@ -161,7 +170,7 @@ __global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p
   // pass 1: validate and count key tiles and (sequence, KV head) pairs
   int local = 0, bad = 0;
   for (int s = tid; s < p.batch; s += blockDim.x) {
-    const int P = p.prefix_len[s], W = p.window_len[s], mode = p.mask_mode[s];
+    const int P = seq_prefix(p, s), W = p.window_len[s], mode = seq_mode(p, s);
     if (!seq_ok(p, s, P, W, mode)) { bad = 1; continue; }
     const int slabs = (W * p.G + kUnitRows - 1) / kUnitRows;
     for (int sl = 0; sl < slabs; ++sl) local += slab_tiles(P, W, mode, sl * kUnitRows, p.G, p.block_size) * p.Hkv;
@@ -185,7 +194,7 @@ __global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p
   {
     int cnt[kSplitFactor] = {};
     for (int s = tid; s < p.batch; s += blockDim.x) {
-      const int P = p.prefix_len[s], W = p.window_len[s], mode = p.mask_mode[s];
+      const int P = seq_prefix(p, s), W = p.window_len[s], mode = seq_mode(p, s);
       if (!seq_ok(p, s, P, W, mode)) continue;
       const int slabs = (W * p.G + kUnitRows - 1) / kUnitRows;
       for (int sl = 0; sl < slabs; ++sl) {
@@ -236,7 +245,7 @@ __global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p
   // spread their pieces over many threads
   for (int sg = tid; sg < p.batch * p.Hkv; sg += blockDim.x) {
     const int s = sg / p.Hkv, g = sg - s * p.Hkv;
-    const int P = p.prefix_len[s], W = p.window_len[s], mode = p.mask_mode[s];
+    const int P = seq_prefix(p, s), W = p.window_len[s], mode = seq_mode(p, s);
     if (!seq_ok(p, s, P, W, mode)) continue;
     const int slabs = (W * p.G + kUnitRows - 1) / kUnitRows;
     const int ng = slabs <= kMaxGroupedSlabs ? slabs : 1;  // slabs per piece
@@ -344,7 +353,36 @@ struct AttnParams {
   float* part_lse;
   int max_pages, num_pages, Hq, G, block_size, page_size, box_rows, loads_per_tile;
   float scale_log2;
+  // block-mask mode: bit kb of word kb / 32 of row qb of sequence s (mask + (s * mask_rows + qb) * mask_words)
+  // is set iff query block qb attends to key block kb; block_log2 = log2(block_size)
+  const uint32_t* mask;
+  int mask_rows, mask_words, block_log2;
 };
+
+// Block-mask mode: does any query block of packed rows [row0, row0 + 256) see a
+// key block of window tile t? W is the sequence length.
+__device__ __forceinline__ bool tile_visible(const AttnParams& p, int seq, int row0, int W, int t) {
+  const int q0 = row0 / p.G, q1 = min(W, (row0 + kUnitRows) / p.G) - 1;
+  const int k0 = t * kTileKeys, k1 = min(W, k0 + kTileKeys) - 1;
+  if (q1 < q0 || k1 < k0) return false;
+  const int qb0 = q0 >> p.block_log2, qb1 = q1 >> p.block_log2;
+  const int kb0 = k0 >> p.block_log2, kb1 = k1 >> p.block_log2;
+  const uint32_t* m = p.mask + static_cast<int64_t>(seq) * p.mask_rows * p.mask_words;
+  for (int qb = qb0; qb <= qb1 && qb < p.mask_rows; ++qb)
+    for (int kb = kb0; kb <= kb1; ++kb)
+      if (kb / 32 < p.mask_words && ((m[static_cast<int64_t>(qb) * p.mask_words + kb / 32] >> (kb % 32)) & 1u)) return true;
+  return false;
+}
+
+// Next set bit after t in a unit's visible-tile bitmask (-1 if none).
+__device__ __forceinline__ int next_tile(const volatile uint32_t* bits, int t) {
+  for (int b = t + 1; b < kMaskTileWords * 32;) {
+    const uint32_t w = bits[b >> 5] >> (b & 31);
+    if (w) return b + __ffs(w) - 1;
+    b = (b & ~31) + 32;
+  }
+  return -1;
+}
 
 // Shared memory: two Q tiles, then a ring of kSlots K-or-V tiles. Items are
 // loaded in the order K(0), V(0), K(1), V(1), ...; K(t) is released once the
@@ -379,7 +417,7 @@ struct Bars {
   uint64_t u_full[2], u_empty[2];
 };
 
-template <int D>
+template <int D, bool kMask>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kw,
                 const __grid_constant__ CUtensorMap tm_vw, const __grid_constant__ CUtensorMap tm_kc,
@@ -389,6 +427,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   __shared__ __align__(8) Bars bars;
   __shared__ WorkUnit unit_ring[2];
+  // block-mask mode: visible key tiles of each ring unit (bit t - tile_begin)
+  __shared__ uint32_t unit_tiles[kMask ? 2 : 1][kMask ? kMaskTileWords : 1];
   __shared__ uint32_t tmem_base_s;
   __shared__ int abort_s;
   volatile int* abort_flag = &abort_s;
@@ -460,11 +500,29 @@ __global__ void __launch_bounds__(kThreads, 1)
         wu = p.units[uidx];
         const int W = wu.window_mode & 0x3FFFFFFF;
         const bool sane = wu.seq >= 0 && wu.seq < p.batch && wu.kv_head >= 0 && wu.tile_begin >= 0 &&
-                          wu.tile_end > wu.tile_begin && W > 0;
+                          wu.tile_end > wu.tile_begin && W > 0 &&
+                          (!kMask || wu.tile_end - wu.tile_begin <= kMaskTileWords * 32);
         const int cu = sane ? p.cu_window[wu.seq] : -1;
         if (!sane || cu < 0 || static_cast<int64_t>(cu) + W > p.total_tokens) {
           if (lane == 0) atomicOr(&g_error_word, MBE_DEVERR_LENGTH);
           continue;  // skip this unit; every role only ever sees published units
+        }
+      }
+      if constexpr (kMask) {
+        if (!done) {
+          // visible key tiles of this unit (relative to tile_begin); an empty set keeps
+          // its first tile (fully masked) so that every role still sees one tile
+          const int n_rel = wu.tile_end - wu.tile_begin;
+          const int W = wu.window_mode & 0x3FFFFFFF;
+          bool any = false;
+          for (int w = 0; w < kMaskTileWords; ++w) {
+            const int rel = 32 * w + lane;
+            const bool vis = rel < n_rel && tile_visible(p, wu.seq, wu.row0, W, wu.tile_begin + rel);
+            const uint32_t word = __ballot_sync(kAll, vis);
+            any |= word != 0;
+            if (lane == 0) unit_tiles[uslot][w] = word;
+          }
+          if (!any && lane == 0) unit_tiles[uslot][0] = 1u;
         }
       }
       if (lane == 0) {
@@ -521,7 +579,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           pg_hi = fetch_page(pg_base + 32 + lane);
         }
       };
-      for (int t = wu.tile_begin; t < wu.tile_end && ok; ++t) {
+      // block-mask mode walks the unit's visible tiles, the other modes every tile
+      const volatile uint32_t* tbits = unit_tiles[kMask ? uslot : 0];
+      auto advance = [&](int t) {
+        if (!kMask) return t + 1;
+        const int r = next_tile(tbits, t - wu.tile_begin);
+        return r < 0 ? wu.tile_end : wu.tile_begin + r;
+      };
+      for (int t = kMask ? advance(wu.tile_begin - 1) : wu.tile_begin; t < wu.tile_end && ok; t = advance(t)) {
         if (t < nP) ensure_window((t * kTileKeys) / p.page_size);
         for (int kv = 0; kv < 2; ++kv, ++item) {
           const uint32_t sl = slot_of(item), use = item / S::kSlots;
@@ -590,12 +655,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int slot = u_it & 1;
         if (!mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag)) { ok = false; break; }
         const WorkUnit wu = unit_ring[slot];
+        int n_t = wu.tile_end - wu.tile_begin;
+        if constexpr (kMask) {
+          n_t = 0;
+          for (int w = 0; w < kMaskTileWords; ++w) n_t += __popc(unit_tiles[slot][w]);
+        }
         mbar_arrive(bar(bars.u_empty[slot]));
         ++u_it;
         if (wu.seq < 0) break;
         const int W = wu.window_mode & 0x3FFFFFFF;
         const int n_qt = (W * p.G - wu.row0) > kTileRows ? 2 : 1;
-        const int n_t = wu.tile_end - wu.tile_begin;
         if (!mbar_wait(bar(bars.q_full), q_it & 1, abort_flag)) { ok = false; break; }
         ++q_it;
         // items of tile ki: K = 2 ki, V = 2 ki + 1
@@ -664,37 +733,74 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag));
       if (!ok) break;
       const WorkUnit wu = unit_ring[slot];
-      __syncwarp();
-      if (lane == 0) mbar_arrive(bar(bars.u_empty[slot]));
+      // block-mask mode keeps the ring slot (and its tile bitmask) until its tiles are done
+      auto release_unit = [&]() {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(bars.u_empty[slot]));
+      };
+      if (!kMask) release_unit();
       ++u_it;
-      if (wu.seq < 0) break;
+      if (wu.seq < 0) {
+        if (kMask) release_unit();
+        break;
+      }
       const int W = wu.window_mode & 0x3FFFFFFF;
-      const int mode = wu.window_mode >> 30;
+      const int mode = static_cast<int>(static_cast<uint32_t>(wu.window_mode) >> 30);
       const int n_qt = (W * p.G - wu.row0) > kTileRows ? 2 : 1;
-      const int n_t = wu.tile_end - wu.tile_begin;
+      int n_t = wu.tile_end - wu.tile_begin;
+      const volatile uint32_t* tbits = unit_tiles[kMask ? slot : 0];
+      if constexpr (kMask) {
+        n_t = 0;
+        for (int w = 0; w < kMaskTileWords; ++w) n_t += __popc(tbits[w]);
+      }
       const int P = wu.prefix;
       const int nP = (P + kTileKeys - 1) / kTileKeys;
       if (wg >= n_qt) {
         kv_it += n_t;
+        if (kMask) release_unit();
         continue;
       }
       const int R = wu.row0 + kTileRows * wg + r;
       const int qi = R / p.G, hh = R - qi * p.G;
       const bool valid = qi < W;
-      const int lim = (mode == MBE_MULTI_BLOCK_BIDIRECTIONAL) ? W : min(W, (qi / p.block_size + 1) * p.block_size);
+      const int lim = (mode == MBE_BLOCK_CAUSAL) ? min(W, (qi / p.block_size + 1) * p.block_size) : W;
+      // block-mask mode: this row's mask row (query block of token qi)
+      const uint32_t* mrow = nullptr;
+      int kbpt = 1;
+      uint32_t all_bits = 1u;
+      if constexpr (kMask) {
+        const int qb = min(qi, W - 1) >> p.block_log2;
+        mrow = p.mask + (static_cast<int64_t>(wu.seq) * p.mask_rows + min(qb, p.mask_rows - 1)) * p.mask_words;
+        kbpt = max(1, kTileKeys >> p.block_log2);
+        all_bits = kbpt >= 32 ? 0xFFFFFFFFu : ((1u << kbpt) - 1u);
+      }
       float m = neg_inf(), l = 0.f;
+      int t = wu.tile_begin - 1;
       for (int j = 0; j < n_t; ++j) {
-        const int t = wu.tile_begin + j;
+        if constexpr (kMask) {
+          const int rnext = next_tile(tbits, t - wu.tile_begin);
+          t = wu.tile_begin + max(rnext, 0);
+        } else {
+          t = wu.tile_begin + j;
+        }
         const uint32_t ki = kv_it + j;
         ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.s_full[wg]), s_cnt & 1, abort_flag));
         if (!ok) break;
         ++s_cnt;
         tc_fence_after();
         const int n_vis = t < nP ? min(kTileKeys, P - t * kTileKeys) : max(0, min(kTileKeys, lim - (t - nP) * kTileKeys));
+        // block-mask mode: bit c >> block_log2 of nib tells whether column c's key block is visible
+        uint32_t nib = 0xFFFFFFFFu;
+        if constexpr (kMask) {
+          const int kb0 = ((t - nP) * kTileKeys) >> p.block_log2;
+          const uint32_t word = (kb0 >> 5) < p.mask_words ? mrow[kb0 >> 5] : 0u;
+          nib = (word >> (kb0 & 31)) & all_bits;
+        }
+        auto visible = [&](int k) { return k < n_vis && (!kMask || ((nib >> (k >> p.block_log2)) & 1u)); };
         // The whole S row (128 fp32) comes from TMEM in one load; P is packed to
         // bf16 in place (entry k <- columns 2k, 2k+1) and stored as 64 columns
         // over the start of the same TMEM region.
-        const bool full = __all_sync(0xffffffffu, n_vis == kTileKeys);
+        const bool full = __all_sync(0xffffffffu, n_vis == kTileKeys && (!kMask || nib == all_bits));
         uint32_t v[128];
         tmem_ld128(tS, v);
         float mx = neg_inf();
@@ -709,7 +815,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         } else {
 #pragma unroll
           for (int k = 0; k < 128; ++k)
-            if (k < n_vis) mx = fmaxf(mx, __uint_as_float(v[k]));
+            if (visible(k)) mx = fmaxf(mx, __uint_as_float(v[k]));
         }
         // Lazy rescaling: the reference max m only moves when the tile's max
         // exceeds it by more than 2^8; P, l and O then all use the new m.
@@ -738,8 +844,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         } else {
 #pragma unroll
           for (int k = 0; k < 64; ++k) {
-            const float p0 = 2 * k < n_vis ? ex2f(fmaf(__uint_as_float(v[2 * k]), p.scale_log2, neg_mu)) : 0.f;
-            const float p1 = 2 * k + 1 < n_vis ? ex2f(fmaf(__uint_as_float(v[2 * k + 1]), p.scale_log2, neg_mu)) : 0.f;
+            const float p0 = visible(2 * k) ? ex2f(fmaf(__uint_as_float(v[2 * k]), p.scale_log2, neg_mu)) : 0.f;
+            const float p1 = visible(2 * k + 1) ? ex2f(fmaf(__uint_as_float(v[2 * k + 1]), p.scale_log2, neg_mu)) : 0.f;
             l0 += p0;
             l1 += p1;
             v[k] = pack_bf16x2(p0, p1);
@@ -780,6 +886,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (!ok) break;
       kv_it += n_t;
+      if (kMask) release_unit();
       // epilogue: O_i is complete once o_full fires
       ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.o_full[wg]), o_cnt & 1, abort_flag));
       if (!ok) break;
@@ -939,7 +1046,7 @@ __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const MergePa
 // ------------------------------------------------------------------ host side
 struct DeviceInfo {
   int num_sms = 0;
-  bool attr_set[2] = {false, false};
+  bool attr_set[4] = {false, false, false, false};
 };
 
 DeviceInfo* device_info(int dev) {
@@ -954,11 +1061,11 @@ DeviceInfo* device_info(int dev) {
   return &d;
 }
 
-template <int D>
+template <int D, bool kMask>
 bool ensure_smem_attr(DeviceInfo* di) {
-  const int idx = D == 128 ? 1 : 0;
+  const int idx = (D == 128 ? 1 : 0) + (kMask ? 2 : 0);
   if (!di->attr_set[idx]) {
-    if (cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<D>::kBytes) !=
+    if (cudaFuncSetAttribute(attn_kernel<D, kMask>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<D>::kBytes) !=
         cudaSuccess)
       return false;
     di->attr_set[idx] = true;
@@ -978,13 +1085,19 @@ mbe_status check_shapes(int32_t batch, int32_t Hq, int32_t Hkv, int32_t D, int32
   return MBE_OK;
 }
 
-template <int D>
+// Block mask of the block-mask mode (null otherwise).
+struct MaskArgs {
+  const uint32_t* bits = nullptr;
+  int rows = 0, words = 0;
+};
+
+template <int D, bool kMask>
 mbe_status run(const void* q, const void* k_win, const void* v_win, const void* k_cache, const void* v_cache,
                int32_t num_pages, const int32_t* block_table, int32_t max_pages, const int32_t* prefix_len,
                const int32_t* window_len, const int32_t* cu_window, const uint8_t* mask_mode, int32_t batch,
                int32_t total_q_tokens, int32_t Hq, int32_t Hkv, int32_t block_size, int32_t page_size,
                int32_t max_window, int32_t max_prefix, float scale, void* out, float* lse, void* workspace,
-               const Layout& L, DeviceInfo* di, bool with_plan, cudaStream_t stream) {
+               const Layout& L, DeviceInfo* di, bool with_plan, const MaskArgs& mask, cudaStream_t stream) {
   const int G = Hq / Hkv;
   CUtensorMap tq, tkw, tvw, tkc, tvc;
   {
@@ -1011,7 +1124,7 @@ mbe_status run(const void* q, const void* k_win, const void* v_win, const void* 
         !encode_bf16_sw128(&tvc, v_cache, 4, dims, strides, box))
       return MBE_ERR_CUDA;
   }
-  if (!ensure_smem_attr<D>(di)) {
+  if (!ensure_smem_attr<D, kMask>(di)) {
     record_cuda_error(cudaGetLastError(), "cudaFuncSetAttribute(attn_kernel)");
     return MBE_ERR_CUDA;
   }
@@ -1019,8 +1132,9 @@ mbe_status run(const void* q, const void* k_win, const void* v_win, const void* 
   Header* hdr = reinterpret_cast<Header*>(ws);
   const PlanSig sig = make_sig(batch, total_q_tokens, G, Hkv, D, block_size, max_window, max_prefix);
   SchedParams sp{prefix_len, window_len, mask_mode, cu_window, batch, G, Hkv, block_size, max_window, max_prefix,
-                 di->num_sms, total_q_tokens, sig, hdr, reinterpret_cast<WorkUnit*>(ws + L.units_tmp), reinterpret_cast<WorkUnit*>(ws + L.units),
-                 reinterpret_cast<MergeGroup*>(ws + L.groups), L.max_units, L.max_groups, L.max_slots};
+                 di->num_sms, total_q_tokens, kMask, sig, hdr, reinterpret_cast<WorkUnit*>(ws + L.units_tmp),
+                 reinterpret_cast<WorkUnit*>(ws + L.units), reinterpret_cast<MergeGroup*>(ws + L.groups), L.max_units,
+                 L.max_groups, L.max_slots};
   if (with_plan) {
     attn_schedule_kernel<<<1, kBuckets, 0, stream>>>(sp);
     if (launch_status("attn_schedule_kernel launch") != MBE_OK) return MBE_ERR_CUDA;
@@ -1046,7 +1160,12 @@ mbe_status run(const void* q, const void* k_win, const void* v_win, const void* 
   ap.box_rows = box_rows;
   ap.loads_per_tile = kTileKeys / box_rows;
   ap.scale_log2 = scale * 1.4426950408889634f;
-  attn_kernel<D><<<di->num_sms, kThreads, Smem<D>::kBytes, stream>>>(tq, tkw, tvw, tkc, tvc, ap);
+  ap.mask = mask.bits;
+  ap.mask_rows = mask.rows;
+  ap.mask_words = mask.words;
+  ap.block_log2 = 0;
+  while ((1 << ap.block_log2) < block_size) ++ap.block_log2;
+  attn_kernel<D, kMask><<<di->num_sms, kThreads, Smem<D>::kBytes, stream>>>(tq, tkw, tvw, tkc, tvc, ap);
   if (launch_status("attn_kernel launch") != MBE_OK) return MBE_ERR_CUDA;
   MergeParams mp{sig, batch, total_q_tokens, hdr, reinterpret_cast<const MergeGroup*>(ws + L.groups), ap.part_o,
                  ap.part_lse, cu_window, ap.out, lse, Hq, G};
@@ -1127,13 +1246,14 @@ mbe_status attention_call(const void* q, const void* k_win, const void* v_win, c
                              pointers_ok, noop, c);
   if (st != MBE_OK || noop) return st;
   if (head_dim == 128)
-    return run<128>(q, k_win, v_win, k_cache, v_cache, num_pages, block_table, max_pages_per_seq, prefix_len,
+    return run<128, false>(q, k_win, v_win, k_cache, v_cache, num_pages, block_table, max_pages_per_seq, prefix_len,
                     window_len, cu_window, mask_mode, batch, total_q_tokens, num_q_heads, num_kv_heads, block_size,
                     page_size, max_window, max_prefix, c.scale, out, lse_or_null, workspace, c.L, c.di, with_plan,
-                    stream);
-  return run<64>(q, k_win, v_win, k_cache, v_cache, num_pages, block_table, max_pages_per_seq, prefix_len, window_len,
+                    MaskArgs{}, stream);
+  return run<64, false>(q, k_win, v_win, k_cache, v_cache, num_pages, block_table, max_pages_per_seq, prefix_len, window_len,
                  cu_window, mask_mode, batch, total_q_tokens, num_q_heads, num_kv_heads, block_size, page_size,
-                 max_window, max_prefix, c.scale, out, lse_or_null, workspace, c.L, c.di, with_plan, stream);
+                 max_window, max_prefix, c.scale, out, lse_or_null, workspace, c.L, c.di, with_plan, MaskArgs{},
+                 stream);
 }
 
 }  // namespace
@@ -1171,7 +1291,7 @@ extern "C" mbe_status mbe_window_attention_plan(const int32_t* prefix_len, const
   const PlanSig sig = make_sig(batch, total_q_tokens, num_q_heads / num_kv_heads, num_kv_heads, head_dim, block_size,
                                max_window, max_prefix);
   SchedParams sp{prefix_len, window_len, mask_mode, cu_window, batch, num_q_heads / num_kv_heads, num_kv_heads,
-                 block_size, max_window, max_prefix, c.di->num_sms, total_q_tokens, sig, reinterpret_cast<Header*>(ws),
+                 block_size, max_window, max_prefix, c.di->num_sms, total_q_tokens, false, sig, reinterpret_cast<Header*>(ws),
                  reinterpret_cast<WorkUnit*>(ws + c.L.units_tmp), reinterpret_cast<WorkUnit*>(ws + c.L.units),
                  reinterpret_cast<MergeGroup*>(ws + c.L.groups), c.L.max_units, c.L.max_groups, c.L.max_slots};
   attn_schedule_kernel<<<1, kBuckets, 0, stream>>>(sp);
@@ -1245,4 +1365,34 @@ extern "C" mbe_status mbe_window_attention_noalloc(const void* q, const void* k_
                               prefix_len, window_len, cu_window, mask_mode, batch, total_q_tokens, num_q_heads,
                               num_kv_heads, head_dim, block_size, page_size, max_window, max_prefix, softmax_scale,
                               out, lse_or_null, scratch, mbe::attn::kNoAllocScratchBytes, stream);
+}
+
+extern "C" mbe_status mbe_block_mask_attention(const void* q, const void* k, const void* v, const int32_t* seq_len,
+                                               const int32_t* cu_seqlens, const uint32_t* mask, int32_t mask_rows,
+                                               int32_t mask_words, int32_t batch, int32_t total_tokens,
+                                               int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim,
+                                               int32_t block_size, int32_t max_seq_len, float softmax_scale,
+                                               void* out, float* lse_or_null, void* workspace,
+                                               size_t workspace_bytes, cudaStream_t stream) {
+  if (block_size < 8 || (block_size & (block_size - 1)) != 0 || mask_rows < 1 || mask_words < 1 ||
+      static_cast<int64_t>(mask_words) * 32 < mask_rows || max_seq_len < 0)
+    return MBE_ERR_INVALID_ARG;
+  if (max_seq_len > kMaskTileWords * 32 * kTileKeys) return MBE_ERR_UNSUPPORTED;
+  if ((max_seq_len + block_size - 1) / block_size > mask_rows) return MBE_ERR_INVALID_ARG;
+  bool noop = false;
+  Checked c;
+  const bool pointers_ok = q && k && v && seq_len && cu_seqlens && mask && out && aligned16(q) && aligned16(k) &&
+                           aligned16(v) && aligned16(out);
+  mbe_status st = check_call(1, 1, batch, total_tokens, num_q_heads, num_kv_heads, head_dim, block_size, kTileKeys,
+                             max_seq_len, 0, softmax_scale, workspace, workspace_bytes, pointers_ok, noop, c);
+  if (st != MBE_OK || noop) return st;
+  const MaskArgs ma{mask, mask_rows, mask_words};
+  // the sequence is the window; the (unused) paged-cache maps point at k / v
+  if (head_dim == 128)
+    return run<128, true>(q, k, v, k, v, 1, nullptr, 1, nullptr, seq_len, cu_seqlens, nullptr, batch, total_tokens,
+                          num_q_heads, num_kv_heads, block_size, kTileKeys, max_seq_len, 0, c.scale, out, lse_or_null,
+                          workspace, c.L, c.di, true, ma, stream);
+  return run<64, true>(q, k, v, k, v, 1, nullptr, 1, nullptr, seq_len, cu_seqlens, nullptr, batch, total_tokens,
+                       num_q_heads, num_kv_heads, block_size, kTileKeys, max_seq_len, 0, c.scale, out, lse_or_null,
+                       workspace, c.L, c.di, true, ma, stream);
 }

@@ -23,6 +23,7 @@ uint32_t attention_take_error();
 uint32_t denoise_take_error();
 uint32_t refresh_take_error();
 uint32_t lm_head_take_error();
+uint32_t train_take_error();
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 

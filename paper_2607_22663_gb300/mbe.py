@@ -20,7 +20,7 @@ MBE_OK = 0
 STATUS_NAMES = {0: "MBE_OK", 1: "MBE_ERR_INVALID_ARG", 2: "MBE_ERR_UNSUPPORTED", 3: "MBE_ERR_CUDA",
                 4: "MBE_ERR_TIMEOUT", 5: "MBE_ERR_WORKSPACE", 6: "MBE_ERR_DEVICE_CHECK"}
 DEVERR_TIMEOUT, DEVERR_LENGTH, DEVERR_PAGE, DEVERR_CAPACITY, DEVERR_PLAN = 0x1, 0x2, 0x4, 0x8, 0x10
-BLOCK_CAUSAL, MULTI_BLOCK_BIDIRECTIONAL = 0, 1
+BLOCK_CAUSAL, MULTI_BLOCK_BIDIRECTIONAL, BLOCK_MASK = 0, 1, 2
 HEADER = _build.INCLUDE / "mbe.h"
 
 _lib = None
@@ -82,6 +82,11 @@ def lib(build_if_missing: bool = True):
     L.mbe_lm_head_workspace_size.argtypes = [i32, i32]
     L.mbe_lm_head_edit_decide.restype = ctypes.c_int
     L.mbe_lm_head_edit_decide.argtypes = [P, P, i32, i32, i32, P, P, f32, P, P, P, P, P, P, P, sz, P]
+    L.mbe_sft_block_mask.restype = ctypes.c_int
+    L.mbe_sft_block_mask.argtypes = [P, P, i32, i32, i32, i32, P, P]
+    L.mbe_block_mask_attention.restype = ctypes.c_int
+    L.mbe_block_mask_attention.argtypes = [P, P, P, P, P, P, i32, i32, i32, i32, i32, i32, i32, i32, i32, f32, P, P, P,
+                                           sz, P]
     L.mbe_refresh_plan.restype = ctypes.c_int
     L.mbe_refresh_plan.argtypes = [P, i32, P, P, P, P, i32, i32, i32, i32, i32, P, P, P, P, P, P, P, P]
     L.mbe_gather_rows.restype = ctypes.c_int
@@ -383,6 +388,50 @@ def lm_head_edit_decide(hidden, weight, committed, tau=0.0, tau_per_row=None, ed
                                        workspace.numel(), _stream(stream))
     _check("mbe_lm_head_edit_decide", st)
     return new_tokens, edit_mask, confidence, argmax, entropy
+
+
+def sft_block_mask(n_prompt_blocks, n_blocks, K, mask_rows, mask_words=None, out=None, stream=None):
+    """mbe_sft_block_mask: see include/mbe.h. Returns uint32 bits as int32 [batch, mask_rows, mask_words]."""
+    _need(n_prompt_blocks, "n_prompt_blocks", torch.int32)
+    _need(n_blocks, "n_blocks", torch.int32)
+    batch = n_blocks.numel()
+    mask_words = mask_words or max(1, (mask_rows + 31) // 32)
+    if out is None:
+        out = torch.empty((batch, mask_rows, mask_words), dtype=torch.int32, device=n_blocks.device)
+    _need(out, "out", torch.int32)
+    st = lib().mbe_sft_block_mask(_ptr(n_prompt_blocks), _ptr(n_blocks), int(K), batch, mask_rows, mask_words,
+                                  _ptr(out), _stream(stream))
+    _check("mbe_sft_block_mask", st)
+    return out
+
+
+def block_mask_attention(q, k, v, seq_len, cu_seqlens, mask, *, block_size, max_seq_len, softmax_scale=0.0,
+                         out=None, lse=None, return_lse=False, workspace=None, stream=None):
+    """mbe_block_mask_attention: see include/mbe.h. mask: int32 (uint32 bits)
+    [batch, mask_rows, mask_words]. Returns out (and lse if requested)."""
+    for t, n in ((q, "q"), (k, "k"), (v, "v")):
+        _need(t, n, torch.bfloat16)
+    for t, n in ((seq_len, "seq_len"), (cu_seqlens, "cu_seqlens"), (mask, "mask")):
+        _need(t, n, torch.int32)
+    T, Hq, D = q.shape
+    Hkv = k.shape[1]
+    batch, mask_rows, mask_words = mask.shape
+    if out is None:
+        out = torch.empty_like(q)
+    _need(out, "out", torch.bfloat16)
+    if return_lse and lse is None:
+        lse = torch.empty((T, Hq), dtype=torch.float32, device=q.device)
+    if lse is not None:
+        _need(lse, "lse", torch.float32)
+    need = window_attention_workspace_size(batch, Hq, Hkv, D, max_seq_len, 0)
+    if workspace is None:
+        workspace = torch.empty(max(need, 1), dtype=torch.uint8, device=q.device)
+    st = lib().mbe_block_mask_attention(_ptr(q), _ptr(k), _ptr(v), _ptr(seq_len), _ptr(cu_seqlens), _ptr(mask),
+                                        mask_rows, mask_words, batch, T, Hq, Hkv, D, block_size, max_seq_len,
+                                        float(softmax_scale), _ptr(out), _ptr(lse), _ptr(workspace), workspace.numel(),
+                                        _stream(stream))
+    _check("mbe_block_mask_attention", st)
+    return (out, lse) if return_lse else out
 
 
 def refresh_plan(block_changed, prefix_len, window_len, cu_window, block_table, *, block_size, max_window,

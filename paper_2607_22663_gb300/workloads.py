@@ -283,6 +283,51 @@ def serving128(device="cpu", layers=24, vocab=131072, batch=128, page_size=64):
 WORKLOADS = {"tiny": tiny, "batch8": batch8, "varlen64": varlen64, "long32k": long32k, "serving128": serving128}
 
 
+@dataclass
+class SftProblem:
+    """A packed batch of Multi-Block Edit SFT training sequences: sequence s is
+    [prompt blocks | noisy blocks | clean blocks] of block_size tokens
+    (its last block may be cut short by `trim`)."""
+    q: torch.Tensor        # bf16 [T, Hq, D]
+    k: torch.Tensor        # bf16 [T, Hkv, D]
+    v: torch.Tensor        # bf16 [T, Hkv, D]
+    dout: torch.Tensor     # bf16 [T, Hq, D], upstream gradient of the attention output
+    seq_len: torch.Tensor  # int32 [batch]
+    cu_seqlens: torch.Tensor  # int32 [batch + 1]
+    n_prompt_blocks: torch.Tensor  # int32 [batch]
+    n_blocks: torch.Tensor  # int32 [batch]
+    block_size: int
+    seq_host: list
+
+    @property
+    def max_seq_len(self):
+        return max(self.seq_host) if self.seq_host else 0
+
+    @property
+    def mask_rows(self):
+        return max(1, (self.max_seq_len + self.block_size - 1) // self.block_size)
+
+
+def sft_problem(n_prompt_blocks, n_blocks, num_q_heads, num_kv_heads, head_dim, block_size, seed, device="cpu",
+                trim=None, g=None) -> SftProblem:
+    """Random N(0,1) bf16 q/k/v/dout for SFT sequences of (Np + 2N) blocks each,
+    optionally shortened by trim[s] tokens (a ragged last block)."""
+    g = g or _gen(seed, device)
+    trim = trim or [0] * len(n_blocks)
+    lens = [(p + 2 * n) * block_size - t for p, n, t in zip(n_prompt_blocks, n_blocks, trim)]
+    T = sum(lens)
+    cu = [0]
+    for n in lens:
+        cu.append(cu[-1] + n)
+    t32 = lambda x: torch.tensor(x, dtype=torch.int32, device=device)
+    return SftProblem(q=_randn_bf16((T, num_q_heads, head_dim), g, device),
+                      k=_randn_bf16((T, num_kv_heads, head_dim), g, device),
+                      v=_randn_bf16((T, num_kv_heads, head_dim), g, device),
+                      dout=_randn_bf16((T, num_q_heads, head_dim), g, device), seq_len=t32(lens), cu_seqlens=t32(cu),
+                      n_prompt_blocks=t32(list(n_prompt_blocks)), n_blocks=t32(list(n_blocks)),
+                      block_size=block_size, seq_host=lens)
+
+
 def extract_sequences(prob: AttnProblem, seqs):
     """The given sequences of `prob` as a standalone CPU problem (their pages
     copied into a compact cache, block table renumbered)."""
