@@ -22,8 +22,8 @@
  * the changed blocks (mbe_refresh_plan, mbe_gather_rows: Sec. 4.3), a
  * device-side loop over editing passes (mbe_pass_loop_*: Sec. 4.1), the
  * LM-head projection fused with the edit decision (mbe_lm_head_edit_decide)
- * and the cross-block training attention of Multi-Block Edit SFT
- * (mbe_sft_block_mask, mbe_block_mask_attention: Sec. 3).
+ * and the cross-block training attention of Multi-Block Edit SFT, forward
+ * and backward (mbe_sft_block_mask, mbe_block_mask_attention[_bwd]: Sec. 3).
  *
  * Conventions shared by every entry point
  *   - All pointers are DEVICE pointers unless stated otherwise; the caller
@@ -369,6 +369,33 @@ mbe_status mbe_block_mask_attention(const void* q, const void* k, const void* v,
                                     int32_t num_kv_heads, int32_t head_dim, int32_t block_size, int32_t max_seq_len,
                                     float softmax_scale, void* out, float* lse_or_null, void* workspace,
                                     size_t workspace_bytes, cudaStream_t stream);
+
+/*
+ * mbe_block_mask_attention_bwd -- gradients of mbe_block_mask_attention (the
+ * backward of Multi-Block Edit SFT's cross-block attention, Sec. 3).
+ * With P the attention probabilities under the mask (recomputed from q, k and
+ * the forward's lse), dO = dout and delta_i = dO_i . O_i:
+ *   dV = P^T dO,  dS = P o (dO V^T - delta),  dQ = scale dS K,  dK = scale dS^T Q
+ * summed over the query heads that share a KV head. Inputs as in
+ * mbe_block_mask_attention plus out (its bf16 output), dout bf16 [total_tokens,
+ * num_q_heads, head_dim] and lse fp32 [total_tokens, num_q_heads] (its natural-
+ * log output). Outputs (fp32, overwritten): dq [total_tokens, num_q_heads,
+ * head_dim], dk, dv [total_tokens, num_kv_heads, head_dim]. P and dS are
+ * rounded to bf16 before their products (tensor cores), as in the forward's P.
+ * workspace: mbe_block_mask_attention_bwd_workspace_size(batch, total_tokens,
+ * num_q_heads) bytes, 16-byte aligned. head_dim must be 128; num_q_heads /
+ * num_kv_heads must divide 128; max_seq_len * that ratio <= 65536.
+ * Errors: MBE_ERR_INVALID_ARG, MBE_ERR_UNSUPPORTED, MBE_ERR_WORKSPACE,
+ * MBE_ERR_CUDA; a bounded wait that expires sets MBE_DEVERR_TIMEOUT.
+ */
+size_t mbe_block_mask_attention_bwd_workspace_size(int32_t batch, int32_t total_tokens, int32_t num_q_heads);
+mbe_status mbe_block_mask_attention_bwd(const void* q, const void* k, const void* v, const void* out,
+                                        const void* dout, const float* lse, const int32_t* seq_len,
+                                        const int32_t* cu_seqlens, const uint32_t* mask, int32_t mask_rows,
+                                        int32_t mask_words, int32_t batch, int32_t total_tokens, int32_t num_q_heads,
+                                        int32_t num_kv_heads, int32_t head_dim, int32_t block_size,
+                                        int32_t max_seq_len, float softmax_scale, float* dq, float* dk, float* dv,
+                                        void* workspace, size_t workspace_bytes, cudaStream_t stream);
 
 /*
  * mbe_lm_head_edit_decide -- the LM-head projection fused with the edit

@@ -1,9 +1,34 @@
 // Multi-Block Edit SFT attention support (Sec. 3): the cross-block attention
-// mask. The forward under the mask is mbe_block_mask_attention (attention.cu).
+// mask and the backward of attention under a block mask. The forward under the
+// mask is mbe_block_mask_attention (attention.cu).
 //
 // sft_mask_kernel: one CTA per (mask row, sequence); thread w builds 32-bit
 // word w of the row from the link rules, so a row of nb blocks costs nb bits.
+//
+// bwd_prep_kernel: delta = rowsum(dO o O) per (token, head), dQ zeroed, the
+// work counter armed.
+// bwd_kernel (persistent, one CTA per SM, 256 threads): a work unit is
+// (sequence, KV head g, 128-key tile); K and V stay in shared memory while the
+// unit walks the 128-row query tiles (packed rows token * G + head of the heads
+// of g) that see any of its key blocks. Per query tile:
+//   warp 0     TMA: Q_i and dO_i into a 2-stage ring (K, V once per unit)
+//   warp 1     MMA: S^T = K Q_i^T and dP^T = V dO_i^T (SS, into TMEM);
+//              then dV += P^T dO_i and dK += dS^T Q_i (TS, P^T and dS^T from
+//              TMEM) and dQ_i = dS K (SS, dS from shared memory)
+//   warps 4-7  thread = key row: P^T = exp(S^T * scale - lse), masked;
+//              dS^T = P^T o (dP^T - delta); P^T and dS^T back to TMEM as bf16,
+//              dS also into shared memory in the layout TMA gives a V tile;
+//              then thread = query row: dQ_i * scale added to dQ (fp32
+//              atomics); at the unit's end, thread = key row: dK * scale and dV
+//              stored (fp32).
+// TMEM: dK, dV, S^T/P^T/dQ and dP^T/dS^T, 128 columns each.
+#include <cuda_bf16.h>
+#include <algorithm>
+#include <cmath>
+#include <mutex>
 #include "common.cuh"
+#include "ptx_sm103.cuh"
+#include "tma_host.cuh"
 
 namespace mbe {
 
@@ -49,7 +74,608 @@ __global__ void __launch_bounds__(128) sft_mask_kernel(const int32_t* __restrict
 }
 
 }  // namespace
+
+namespace bwd {
+
+constexpr int kD = 128;                      // head size of the backward
+constexpr int kTile = 128;                   // keys per key tile = packed rows per query tile
+constexpr int kThreads = 256;
+constexpr int kMaxQWords = 16;               // query-tile bitmask of a unit (<= 512 query tiles)
+constexpr uint32_t kHalf = 128 * 128;        // a 64-column half of a 128-row bf16 tile (16 KB)
+constexpr uint32_t kTileBytes = 2 * kHalf;   // 32 KB
+constexpr uint32_t kK = 0, kV = kTileBytes, kQ = 2 * kTileBytes, kDO = 4 * kTileBytes, kDS = 6 * kTileBytes;
+constexpr uint32_t kSmemBytes = 7 * kTileBytes + 1024;
+constexpr uint32_t kTmDK = 0, kTmDV = 128, kTmS = 256, kTmDP = 384, kTmCols = 512;
+constexpr float kLog2e = 1.4426950408889634f;
+
+struct Params {
+  const int32_t* seq_len;
+  const int32_t* cu;
+  const uint32_t* mask;
+  const float* lse;
+  const float* delta;
+  const int32_t* unit_start;  // [batch + 1]: first work unit of each sequence
+  int* counter;
+  float* dq;
+  float* dk;
+  float* dv;
+  int mask_rows, mask_words, block_log2;
+  int batch, total_tokens, Hq, Hkv, G;
+  float scale, scale_log2;
+};
+
+struct Unit {
+  int32_t seq, g, kt, len, cu;
+};
+
+struct Bars {
+  uint64_t u_full[2], u_empty[2], q_full[2], q_empty[2], kv_full, kv_empty, s_full, p_full, dq_full, dq_empty,
+      acc_full, acc_empty, mma_done, group;
+};
+
+__device__ __forceinline__ float ex2f(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ bool mask_bit(const Params& p, int seq, int qb, int kb) {
+  if (qb < 0 || qb >= p.mask_rows || kb < 0 || (kb >> 5) >= p.mask_words) return false;
+  return (p.mask[(static_cast<int64_t>(seq) * p.mask_rows + qb) * p.mask_words + (kb >> 5)] >> (kb & 31)) & 1u;
+}
+
+// Does any query block of query tile i see a key block of key tile kt?
+__device__ __forceinline__ bool qtile_visible(const Params& p, const Unit& u, int i) {
+  const int q0 = (i * kTile) / p.G, q1 = min(u.len, ((i + 1) * kTile) / p.G) - 1;
+  const int k0 = u.kt * kTile, k1 = min(u.len, k0 + kTile) - 1;
+  if (q1 < q0 || k1 < k0) return false;
+  for (int qb = q0 >> p.block_log2; qb <= (q1 >> p.block_log2); ++qb)
+    for (int kb = k0 >> p.block_log2; kb <= (k1 >> p.block_log2); ++kb)
+      if (mask_bit(p, u.seq, qb, kb)) return true;
+  return false;
+}
+
+__device__ __forceinline__ int next_bit(const volatile uint32_t* bits, int i) {
+  for (int b = i + 1; b < kMaxQWords * 32;) {
+    const uint32_t w = bits[b >> 5] >> (b & 31);
+    if (w) return b + __ffs(w) - 1;
+    b = (b & ~31) + 32;
+  }
+  return -1;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    bwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_do,
+               const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v, const Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  __shared__ __align__(8) Bars bars;
+  __shared__ Unit ring[2];
+  __shared__ uint32_t ring_bits[2][kMaxQWords];
+  __shared__ float lse2_s[kTile], delta_s[kTile];
+  __shared__ int qrel_s[kTile];
+  __shared__ uint32_t tmem_base_s;
+  __shared__ int abort_s;
+  volatile int* abort_flag = &abort_s;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t sbase = smem_u32(smem);
+  auto bar = [](uint64_t& b) { return smem_u32(&b); };
+  const int n_units = p.unit_start[p.batch];
+
+  if (tid == 0) {
+    abort_s = 0;
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(bar(bars.u_full[i]), 1);
+      mbar_init(bar(bars.u_empty[i]), 5);  // MMA issuer + 4 compute warps
+      mbar_init(bar(bars.q_full[i]), 1);
+      mbar_init(bar(bars.q_empty[i]), 1);
+    }
+    mbar_init(bar(bars.kv_full), 1);
+    mbar_init(bar(bars.kv_empty), 1);
+    mbar_init(bar(bars.s_full), 1);
+    mbar_init(bar(bars.p_full), 4);
+    mbar_init(bar(bars.dq_full), 1);
+    mbar_init(bar(bars.dq_empty), 4);
+    mbar_init(bar(bars.acc_full), 1);
+    mbar_init(bar(bars.acc_empty), 4);
+    mbar_init(bar(bars.mma_done), 1);
+    mbar_init(bar(bars.group), 4);  // the compute warps among themselves
+    mbar_fence_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&tmem_base_s), kTmCols);
+    tmem_relinquish();
+  }
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_s;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- producer
+    constexpr unsigned kAll = 0xffffffffu;
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_q);
+      tma_prefetch_desc(&tm_do);
+      tma_prefetch_desc(&tm_k);
+      tma_prefetch_desc(&tm_v);
+    }
+    uint32_t u_it = 0, kv_loads = 0, q_it = 0;
+    bool ok = true;
+    for (;;) {
+      int uidx = 0;
+      if (lane == 0) uidx = atomicAdd(p.counter, 1);
+      uidx = __shfl_sync(kAll, uidx, 0);
+      const bool done = uidx >= n_units;
+      const int slot = u_it & 1;
+      if (u_it >= 2) {
+        ok = __all_sync(kAll, mbar_wait(bar(bars.u_empty[slot]), ((u_it >> 1) - 1) & 1, abort_flag));
+        if (!ok) break;
+      }
+      Unit un{-1, 0, 0, 0, 0};
+      if (!done) {
+        int lo = 0, hi = p.batch - 1;  // the sequence whose unit range holds uidx
+        while (lo < hi) {
+          const int mid = (lo + hi + 1) >> 1;
+          if (p.unit_start[mid] <= uidx) lo = mid; else hi = mid - 1;
+        }
+        const int len = p.seq_len[lo];
+        const int tiles = (len + kTile - 1) / kTile;
+        const int r = uidx - p.unit_start[lo];
+        un = Unit{lo, r / max(tiles, 1), r % max(tiles, 1), len, p.cu[lo]};
+        const int n_qt = (len * p.G + kTile - 1) / kTile;
+        for (int w = 0; w < kMaxQWords; ++w) {
+          const int i = 32 * w + lane;
+          const uint32_t word = __ballot_sync(kAll, i < n_qt && qtile_visible(p, un, i));
+          if (lane == 0) ring_bits[slot][w] = word;
+        }
+      }
+      if (lane == 0) {
+        ring[slot] = un;
+        mbar_arrive(bar(bars.u_full[slot]));
+      }
+      __syncwarp();
+      ++u_it;
+      if (done) break;
+      const volatile uint32_t* bits = ring_bits[slot];
+      int n_q = 0;
+      for (int w = 0; w < kMaxQWords; ++w) n_q += __popc(bits[w]);
+      if (n_q == 0) continue;
+      if (kv_loads >= 1) {
+        ok = __all_sync(kAll, mbar_wait(bar(bars.kv_empty), (kv_loads - 1) & 1, abort_flag));
+        if (!ok) break;
+      }
+      if (lane == 0) {
+        mbar_arrive_expect_tx(bar(bars.kv_full), 2 * kTileBytes);
+        for (int h = 0; h < 2; ++h) {
+          tma_load_3d(sbase + kK + h * kHalf, &tm_k, bar(bars.kv_full), h * 64, un.g, un.cu + un.kt * kTile);
+          tma_load_3d(sbase + kV + h * kHalf, &tm_v, bar(bars.kv_full), h * 64, un.g, un.cu + un.kt * kTile);
+        }
+      }
+      ++kv_loads;
+      for (int i = next_bit(bits, -1); i >= 0 && ok; i = next_bit(bits, i)) {
+        const uint32_t st = q_it & 1;
+        if (q_it >= 2) {
+          ok = __all_sync(kAll, mbar_wait(bar(bars.q_empty[st]), ((q_it >> 1) - 1) & 1, abort_flag));
+          if (!ok) break;
+        }
+        if (lane == 0) {
+          mbar_arrive_expect_tx(bar(bars.q_full[st]), 2 * kTileBytes);
+          const int tok = un.cu + (i * kTile) / p.G;
+          for (int h = 0; h < 2; ++h) {
+            tma_load_3d(sbase + kQ + st * kTileBytes + h * kHalf, &tm_q, bar(bars.q_full[st]), h * 64, un.g * p.G, tok);
+            tma_load_3d(sbase + kDO + st * kTileBytes + h * kHalf, &tm_do, bar(bars.q_full[st]), h * 64, un.g * p.G,
+                        tok);
+          }
+        }
+        ++q_it;
+      }
+      if (!ok) break;
+    }
+    if (!ok && lane == 0) {
+      *abort_flag = 1;
+      atomicOr(&g_error_word, MBE_DEVERR_TIMEOUT);
+      // let the copies already issued land before the CTA can exit
+      const int zero = 0;
+      if (kv_loads >= 1) mbar_wait(bar(bars.kv_full), (kv_loads - 1) & 1, &zero);
+      for (uint32_t n = (q_it >= 2 ? q_it - 2 : 0); n < q_it; ++n) mbar_wait(bar(bars.q_full[n & 1]), (n >> 1) & 1, &zero);
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc_kk = idesc_bf16_f32(kTile, kTile, false, false);  // S^T, dP^T
+      constexpr uint32_t idesc_tb = idesc_bf16_f32(kTile, kD, false, true);      // dV, dK: TMEM A, MN-major B
+      constexpr uint32_t idesc_dq = idesc_bf16_f32(kTile, kD, true, true);       // dQ: MN-major A and B
+      uint32_t u_it = 0, units = 0, q_it = 0, tiles = 0;
+      bool ok = true;
+      for (;;) {
+        const int slot = u_it & 1;
+        if (!mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag)) { ok = false; break; }
+        const Unit un = ring[slot];
+        int n_q = 0;
+        for (int w = 0; w < kMaxQWords; ++w) n_q += __popc(ring_bits[slot][w]);
+        mbar_arrive(bar(bars.u_empty[slot]));
+        ++u_it;
+        if (un.seq < 0) break;
+        if (n_q == 0) continue;
+        if (!mbar_wait(bar(bars.kv_full), units & 1, abort_flag)) { ok = false; break; }
+        tc_fence_after();
+        for (int j = 0; j < n_q; ++j) {
+          const uint32_t st = q_it & 1;
+          if (!mbar_wait(bar(bars.q_full[st]), (q_it >> 1) & 1, abort_flag)) { ok = false; break; }
+          if (tiles >= 1 && !mbar_wait(bar(bars.dq_empty), (tiles - 1) & 1, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t qa = sbase + kQ + st * kTileBytes, da = sbase + kDO + st * kTileBytes;
+#pragma unroll
+          for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const uint32_t off = h * kHalf + k * 32;
+              umma_ss(tmem + kTmS, sdesc_sw128(sbase + kK + off, 16, 1024), sdesc_sw128(qa + off, 16, 1024), idesc_kk,
+                      (h | k) ? 1u : 0u);
+              umma_ss(tmem + kTmDP, sdesc_sw128(sbase + kV + off, 16, 1024), sdesc_sw128(da + off, 16, 1024), idesc_kk,
+                      (h | k) ? 1u : 0u);
+            }
+          umma_commit(bar(bars.s_full));
+          if (!mbar_wait(bar(bars.p_full), tiles & 1, abort_flag)) { ok = false; break; }
+          if (j == 0 && units >= 1 && !mbar_wait(bar(bars.acc_empty), (units - 1) & 1, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+#pragma unroll
+          for (int kk = 0; kk < kTile / 16; ++kk) {
+            const uint32_t acc = (j > 0 || kk > 0) ? 1u : 0u;
+            umma_ts(tmem + kTmDV, tmem + kTmS + kk * 8, sdesc_sw128(da + kk * 16 * 128, kHalf, 1024), idesc_tb, acc);
+            umma_ts(tmem + kTmDK, tmem + kTmDP + kk * 8, sdesc_sw128(qa + kk * 16 * 128, kHalf, 1024), idesc_tb, acc);
+          }
+#pragma unroll
+          for (int kk = 0; kk < kTile / 16; ++kk)
+            umma_ss(tmem + kTmS, sdesc_sw128(sbase + kDS + kk * 16 * 128, kHalf, 1024),
+                    sdesc_sw128(sbase + kK + kk * 16 * 128, kHalf, 1024), idesc_dq, kk > 0 ? 1u : 0u);
+          umma_commit(bar(bars.dq_full));
+          umma_commit(bar(bars.q_empty[st]));
+          ++q_it;
+          ++tiles;
+        }
+        if (!ok) break;
+        umma_commit(bar(bars.acc_full));
+        umma_commit(bar(bars.kv_empty));
+        ++units;
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        atomicOr(&g_error_word, MBE_DEVERR_TIMEOUT);
+      }
+      const int zero = 0;
+      umma_commit(bar(bars.mma_done));
+      mbar_wait(bar(bars.mma_done), 0, &zero);
+    }
+  } else if (warp >= 4) {
+    // ---------------------------------------------------------------- compute warps
+    const int quad = warp & 3;
+    const int r = quad * 32 + lane;  // TMEM lane: key row, or query row for dQ
+    const uint32_t t_lane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+    uint32_t u_it = 0, units = 0, tiles = 0, syncs = 0;
+    bool ok = true;
+    // bounded barrier of the four compute warps (orders the per-tile column data)
+    auto group_sync = [&]() {
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar(bars.group));
+      const bool done = __all_sync(0xffffffffu, mbar_wait(bar(bars.group), syncs & 1, abort_flag));
+      ++syncs;
+      return done;
+    };
+    for (;;) {
+      const int slot = u_it & 1;
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag));
+      if (!ok) break;
+      const Unit un = ring[slot];
+      const volatile uint32_t* bits = ring_bits[slot];
+      ++u_it;
+      auto release = [&]() {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(bars.u_empty[slot]));
+      };
+      if (un.seq < 0) {
+        release();
+        break;
+      }
+      int n_q = 0;
+      for (int w = 0; w < kMaxQWords; ++w) n_q += __popc(bits[w]);
+      const int key = un.kt * kTile + r;
+      const bool key_ok = key < un.len;
+      const int64_t kv_row = (static_cast<int64_t>(un.cu) + key) * p.Hkv + un.g;
+      if (n_q == 0) {  // no query sees these keys: zero gradients
+        release();
+        if (key_ok)
+          for (int d = 0; d < kD; d += 4) {
+            *reinterpret_cast<float4*>(p.dk + kv_row * kD + d) = make_float4(0.f, 0.f, 0.f, 0.f);
+            *reinterpret_cast<float4*>(p.dv + kv_row * kD + d) = make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+        continue;
+      }
+      const int kb = key >> p.block_log2;
+      for (int i = next_bit(bits, -1); i >= 0; i = next_bit(bits, i)) {
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.s_full), tiles & 1, abort_flag));
+        if (!ok) break;
+        tc_fence_after();
+        // per-column data of query tile i: lse (log2 units), delta, query block
+        const int qb0 = ((i * kTile) / p.G) >> p.block_log2;
+        ok = group_sync();  // every warp is done with the previous tile's column data
+        if (!ok) break;
+        {
+          const int R = i * kTile + r;
+          const int tok = R / p.G, head = un.g * p.G + (R - tok * p.G);
+          const bool qv = tok < un.len;
+          const int64_t row = (static_cast<int64_t>(un.cu) + tok) * p.Hq + head;
+          lse2_s[r] = qv ? p.lse[row] * kLog2e : __int_as_float(0x7f800000);  // +inf: P = 0
+          delta_s[r] = qv ? p.delta[row] : 0.f;
+          qrel_s[r] = min((tok >> p.block_log2) - qb0, 31);
+        }
+        ok = group_sync();
+        if (!ok) break;
+        // this key block against the (<= 32) query blocks of the tile
+        uint32_t qvis = 0;
+        const int qb_last = min(qb0 + 31, (min(un.len - 1, ((i + 1) * kTile - 1) / p.G)) >> p.block_log2);
+        if (key_ok)
+          for (int qb = qb0; qb <= qb_last; ++qb)
+            if (mask_bit(p, un.seq, qb, kb)) qvis |= 1u << (qb - qb0);
+#pragma unroll 1
+        for (int c4 = 0; c4 < kTile / 32; ++c4) {
+          uint32_t sv[32], dv[32];
+          tmem_ld32(t_lane + kTmS + 32 * c4, sv);
+          tmem_ld32(t_lane + kTmDP + 32 * c4, dv);
+          uint32_t pw[16], dsw[16];
+#pragma unroll
+          for (int jj = 0; jj < 32; jj += 2) {
+            float pp[2], ds[2];
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+              const int col = 32 * c4 + jj + e;
+              const bool vis = (qvis >> qrel_s[col]) & 1u;
+              const float pr = vis ? ex2f(__uint_as_float(sv[jj + e]) * p.scale_log2 - lse2_s[col]) : 0.f;
+              pp[e] = pr;
+              ds[e] = pr * (__uint_as_float(dv[jj + e]) - delta_s[col]);
+            }
+            pw[jj / 2] = pack_bf16x2(pp[0], pp[1]);
+            dsw[jj / 2] = pack_bf16x2(ds[0], ds[1]);
+          }
+          tmem_st16(t_lane + kTmS + 16 * c4, pw);
+          tmem_st16(t_lane + kTmDP + 16 * c4, dsw);
+          // dS into shared memory as row r of a [key][query row] tile, 128-byte swizzle
+          const int h = c4 >> 1;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const int chunk = ((c4 & 1) * 4 + q) ^ (r & 7);
+            *reinterpret_cast<uint4*>(smem + kDS + h * kHalf + r * 128 + chunk * 16) =
+                make_uint4(dsw[4 * q], dsw[4 * q + 1], dsw[4 * q + 2], dsw[4 * q + 3]);
+          }
+        }
+        tmem_st_wait();
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(bars.p_full));
+        // dQ of this query tile: thread = query row
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.dq_full), tiles & 1, abort_flag));
+        if (!ok) break;
+        tc_fence_after();
+        {
+          const int R = i * kTile + r;
+          const int tok = R / p.G, head = un.g * p.G + (R - tok * p.G);
+          const bool qv = tok < un.len;
+          float* dst = p.dq + ((static_cast<int64_t>(un.cu) + tok) * p.Hq + head) * kD;
+#pragma unroll 1
+          for (int c4 = 0; c4 < kD / 32; ++c4) {
+            uint32_t o[32];
+            tmem_ld32(t_lane + kTmS + 32 * c4, o);
+            if (qv)
+#pragma unroll
+              for (int e = 0; e < 32; e += 4)
+                atomicAdd(reinterpret_cast<float4*>(dst + 32 * c4 + e),
+                          make_float4(__uint_as_float(o[e]) * p.scale, __uint_as_float(o[e + 1]) * p.scale,
+                                      __uint_as_float(o[e + 2]) * p.scale, __uint_as_float(o[e + 3]) * p.scale));
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(bars.dq_empty));
+        ++tiles;
+      }
+      if (!ok) break;
+      release();
+      // dK and dV of the unit's keys: thread = key row
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.acc_full), units & 1, abort_flag));
+      if (!ok) break;
+      tc_fence_after();
+#pragma unroll 1
+      for (int c4 = 0; c4 < kD / 32; ++c4) {
+        uint32_t a[32], b[32];
+        tmem_ld32(t_lane + kTmDK + 32 * c4, a);
+        tmem_ld32(t_lane + kTmDV + 32 * c4, b);
+        if (key_ok)
+#pragma unroll
+          for (int e = 0; e < 32; e += 4) {
+            *reinterpret_cast<float4*>(p.dk + kv_row * kD + 32 * c4 + e) =
+                make_float4(__uint_as_float(a[e]) * p.scale, __uint_as_float(a[e + 1]) * p.scale,
+                            __uint_as_float(a[e + 2]) * p.scale, __uint_as_float(a[e + 3]) * p.scale);
+            *reinterpret_cast<float4*>(p.dv + kv_row * kD + 32 * c4 + e) =
+                make_float4(__uint_as_float(b[e]), __uint_as_float(b[e + 1]), __uint_as_float(b[e + 2]),
+                            __uint_as_float(b[e + 3]));
+          }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar(bars.acc_empty));
+      ++units;
+    }
+    if (!ok && lane == 0) {
+      *abort_flag = 1;
+      atomicOr(&g_error_word, MBE_DEVERR_TIMEOUT);
+    }
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmCols);
+  }
+}
+
+// delta = rowsum(dO o O) per (token, head) (one warp per row), dQ zeroed, unit
+// offsets and the work counter set up by block 0.
+__global__ void __launch_bounds__(256) bwd_prep_kernel(const __nv_bfloat16* __restrict__ out,
+                                                       const __nv_bfloat16* __restrict__ dout, int64_t rows,
+                                                       float* __restrict__ delta, float* __restrict__ dq,
+                                                       const int32_t* __restrict__ seq_len, int batch, int Hkv,
+                                                       int32_t* unit_start, int* counter) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = static_cast<int64_t>(gridDim.x) * (blockDim.x / 32);
+  for (int64_t row = static_cast<int64_t>(blockIdx.x) * (blockDim.x / 32) + threadIdx.x / 32; row < rows;
+       row += warps) {
+    const uint2 a = reinterpret_cast<const uint2*>(out + row * kD)[lane];
+    const uint2 b = reinterpret_cast<const uint2*>(dout + row * kD)[lane];
+    const float2 a0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&a.x));
+    const float2 a1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&a.y));
+    const float2 b0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&b.x));
+    const float2 b1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&b.y));
+    float s = a0.x * b0.x + a0.y * b0.y + a1.x * b1.x + a1.y * b1.y;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    if (lane == 0) delta[row] = s;
+    reinterpret_cast<float4*>(dq + row * kD)[lane] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    int acc = 0;
+    for (int s = 0; s < batch; ++s) {
+      unit_start[s] = acc;
+      const int len = seq_len[s];
+      acc += len > 0 ? Hkv * ((len + kTile - 1) / kTile) : 0;
+    }
+    unit_start[batch] = acc;
+    *counter = 0;
+  }
+}
+
+struct DeviceState {
+  int num_sms = 0;
+  bool attr_set = false;
+};
+
+DeviceState* device_state(int dev) {
+  static DeviceState st[64];
+  static std::mutex mu;
+  if (dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lock(mu);
+  DeviceState& d = st[dev];
+  if (d.num_sms == 0 && cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    d.num_sms = 0;
+  if (d.num_sms > 0 && !d.attr_set &&
+      cudaFuncSetAttribute(bwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) == cudaSuccess)
+    d.attr_set = true;
+  return &d;
+}
+
+}  // namespace bwd
 }  // namespace mbe
+
+extern "C" size_t mbe_block_mask_attention_bwd_workspace_size(int32_t batch, int32_t total_tokens,
+                                                              int32_t num_q_heads) {
+  if (batch < 0 || total_tokens < 0 || num_q_heads < 1) return 0;
+  const size_t head = (static_cast<size_t>(batch) + 1) * sizeof(int32_t) + 16;
+  return ((head + 255) & ~size_t(255)) + static_cast<size_t>(total_tokens) * num_q_heads * sizeof(float);
+}
+
+extern "C" mbe_status mbe_block_mask_attention_bwd(const void* q, const void* k, const void* v, const void* out,
+                                                   const void* dout, const float* lse, const int32_t* seq_len,
+                                                   const int32_t* cu_seqlens, const uint32_t* mask, int32_t mask_rows,
+                                                   int32_t mask_words, int32_t batch, int32_t total_tokens,
+                                                   int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim,
+                                                   int32_t block_size, int32_t max_seq_len, float softmax_scale,
+                                                   float* dq, float* dk, float* dv, void* workspace,
+                                                   size_t workspace_bytes, cudaStream_t stream) {
+  using namespace mbe;
+  using namespace mbe::bwd;
+  if (batch < 0 || total_tokens < 0 || num_q_heads < 1 || num_kv_heads < 1 || num_q_heads % num_kv_heads != 0 ||
+      block_size < 8 || (block_size & (block_size - 1)) != 0 || mask_rows < 1 || mask_words < 1 ||
+      static_cast<int64_t>(mask_words) * 32 < mask_rows || max_seq_len < 0 || !(softmax_scale >= 0.f))
+    return MBE_ERR_INVALID_ARG;
+  if (head_dim != kD) return MBE_ERR_UNSUPPORTED;
+  const int G = num_q_heads / num_kv_heads;
+  if (G > kTile || kTile % G != 0) return MBE_ERR_UNSUPPORTED;
+  if (static_cast<int64_t>(max_seq_len) * G > static_cast<int64_t>(kMaxQWords) * 32 * kTile) return MBE_ERR_UNSUPPORTED;
+  if ((max_seq_len + block_size - 1) / block_size > mask_rows) return MBE_ERR_INVALID_ARG;
+  if (batch == 0 || total_tokens == 0) return MBE_OK;
+  if (!q || !k || !v || !out || !dout || !lse || !seq_len || !cu_seqlens || !mask || !dq || !dk || !dv)
+    return MBE_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out) || !aligned16(dout) || !aligned16(dq) ||
+      !aligned16(dk) || !aligned16(dv))
+    return MBE_ERR_INVALID_ARG;
+  if (!workspace || workspace_bytes < mbe_block_mask_attention_bwd_workspace_size(batch, total_tokens, num_q_heads) ||
+      !aligned16(workspace))
+    return MBE_ERR_WORKSPACE;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) {
+    record_cuda_error(e, "cudaGetDevice");
+    return MBE_ERR_CUDA;
+  }
+  DeviceState* ds = device_state(dev);
+  if (!ds || ds->num_sms <= 0 || !ds->attr_set) {
+    record_cuda_error(cudaGetLastError(), "block-mask backward setup");
+    return MBE_ERR_CUDA;
+  }
+  CUtensorMap tq, tdo, tk, tv;
+  {
+    const cuuint64_t dims[3] = {(cuuint64_t)kD, (cuuint64_t)num_q_heads, (cuuint64_t)total_tokens};
+    const cuuint64_t strides[2] = {(cuuint64_t)kD * 2, (cuuint64_t)num_q_heads * kD * 2};
+    const cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)(kTile / G)};
+    if (!encode_bf16_sw128(&tq, q, 3, dims, strides, box) || !encode_bf16_sw128(&tdo, dout, 3, dims, strides, box))
+      return MBE_ERR_CUDA;
+  }
+  {
+    const cuuint64_t dims[3] = {(cuuint64_t)kD, (cuuint64_t)num_kv_heads, (cuuint64_t)total_tokens};
+    const cuuint64_t strides[2] = {(cuuint64_t)kD * 2, (cuuint64_t)num_kv_heads * kD * 2};
+    const cuuint32_t box[3] = {64, 1, (cuuint32_t)kTile};
+    if (!encode_bf16_sw128(&tk, k, 3, dims, strides, box) || !encode_bf16_sw128(&tv, v, 3, dims, strides, box))
+      return MBE_ERR_CUDA;
+  }
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  int* counter = reinterpret_cast<int*>(ws);
+  int32_t* unit_start = reinterpret_cast<int32_t*>(ws + 16);
+  const size_t head = (static_cast<size_t>(batch) + 1) * sizeof(int32_t) + 16;
+  float* delta = reinterpret_cast<float*>(ws + ((head + 255) & ~size_t(255)));
+  const int64_t rows = static_cast<int64_t>(total_tokens) * num_q_heads;
+  const int64_t prep_blocks = std::min<int64_t>((rows + 7) / 8, 8ll * ds->num_sms);
+  bwd_prep_kernel<<<static_cast<unsigned>(std::max<int64_t>(prep_blocks, 1)), 256, 0, stream>>>(
+      static_cast<const __nv_bfloat16*>(out), static_cast<const __nv_bfloat16*>(dout), rows, delta, dq, seq_len, batch,
+      num_kv_heads, unit_start, counter);
+  mbe_status st = launch_status("bwd_prep_kernel");
+  if (st != MBE_OK) return st;
+  Params p;
+  p.seq_len = seq_len;
+  p.cu = cu_seqlens;
+  p.mask = mask;
+  p.lse = lse;
+  p.delta = delta;
+  p.unit_start = unit_start;
+  p.counter = counter;
+  p.dq = dq;
+  p.dk = dk;
+  p.dv = dv;
+  p.mask_rows = mask_rows;
+  p.mask_words = mask_words;
+  p.block_log2 = 0;
+  while ((1 << p.block_log2) < block_size) ++p.block_log2;
+  p.batch = batch;
+  p.total_tokens = total_tokens;
+  p.Hq = num_q_heads;
+  p.Hkv = num_kv_heads;
+  p.G = G;
+  p.scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(kD));
+  p.scale_log2 = p.scale * kLog2e;
+  bwd_kernel<<<ds->num_sms, kThreads, kSmemBytes, stream>>>(tq, tdo, tk, tv, p);
+  return launch_status("bwd_kernel");
+}
 
 extern "C" mbe_status mbe_sft_block_mask(const int32_t* n_prompt_blocks, const int32_t* n_blocks, int32_t K,
                                          int32_t batch, int32_t mask_rows, int32_t mask_words, uint32_t* mask,

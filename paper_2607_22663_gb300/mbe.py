@@ -87,6 +87,11 @@ def lib(build_if_missing: bool = True):
     L.mbe_block_mask_attention.restype = ctypes.c_int
     L.mbe_block_mask_attention.argtypes = [P, P, P, P, P, P, i32, i32, i32, i32, i32, i32, i32, i32, i32, f32, P, P, P,
                                            sz, P]
+    L.mbe_block_mask_attention_bwd_workspace_size.restype = sz
+    L.mbe_block_mask_attention_bwd_workspace_size.argtypes = [i32, i32, i32]
+    L.mbe_block_mask_attention_bwd.restype = ctypes.c_int
+    L.mbe_block_mask_attention_bwd.argtypes = [P, P, P, P, P, P, P, P, P, i32, i32, i32, i32, i32, i32, i32, i32, i32,
+                                               f32, P, P, P, P, sz, P]
     L.mbe_refresh_plan.restype = ctypes.c_int
     L.mbe_refresh_plan.argtypes = [P, i32, P, P, P, P, i32, i32, i32, i32, i32, P, P, P, P, P, P, P, P]
     L.mbe_gather_rows.restype = ctypes.c_int
@@ -432,6 +437,34 @@ def block_mask_attention(q, k, v, seq_len, cu_seqlens, mask, *, block_size, max_
                                         _stream(stream))
     _check("mbe_block_mask_attention", st)
     return (out, lse) if return_lse else out
+
+
+def block_mask_attention_bwd(q, k, v, out, dout, lse, seq_len, cu_seqlens, mask, *, block_size, max_seq_len,
+                             softmax_scale=0.0, dq=None, dk=None, dv=None, workspace=None, stream=None):
+    """mbe_block_mask_attention_bwd: see include/mbe.h. Returns fp32 (dq, dk, dv)."""
+    for t, n in ((q, "q"), (k, "k"), (v, "v"), (out, "out"), (dout, "dout")):
+        _need(t, n, torch.bfloat16)
+    _need(lse, "lse", torch.float32)
+    for t, n in ((seq_len, "seq_len"), (cu_seqlens, "cu_seqlens"), (mask, "mask")):
+        _need(t, n, torch.int32)
+    T, Hq, D = q.shape
+    Hkv = k.shape[1]
+    batch, mask_rows, mask_words = mask.shape
+    dev = q.device
+    dq = torch.empty((T, Hq, D), dtype=torch.float32, device=dev) if dq is None else dq
+    dk = torch.empty((T, Hkv, D), dtype=torch.float32, device=dev) if dk is None else dk
+    dv = torch.empty((T, Hkv, D), dtype=torch.float32, device=dev) if dv is None else dv
+    for t, n in ((dq, "dq"), (dk, "dk"), (dv, "dv")):
+        _need(t, n, torch.float32)
+    need = int(lib().mbe_block_mask_attention_bwd_workspace_size(batch, T, Hq))
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
+    st = lib().mbe_block_mask_attention_bwd(_ptr(q), _ptr(k), _ptr(v), _ptr(out), _ptr(dout), _ptr(lse),
+                                            _ptr(seq_len), _ptr(cu_seqlens), _ptr(mask), mask_rows, mask_words, batch,
+                                            T, Hq, Hkv, D, block_size, max_seq_len, float(softmax_scale), _ptr(dq),
+                                            _ptr(dk), _ptr(dv), _ptr(workspace), workspace.numel(), _stream(stream))
+    _check("mbe_block_mask_attention_bwd", st)
+    return dq, dk, dv
 
 
 def refresh_plan(block_changed, prefix_len, window_len, cu_window, block_table, *, block_size, max_window,
