@@ -346,6 +346,7 @@ def time_extras(w, a0, dev, stream, peaks, reps=10):
     nv = torch.full((a0.batch,), 3, dtype=torch.int32, device=dev)
     ms_sel = ev_time(lambda: mbe.tail_entropy_select(ent, nv, rho=0.25, k_max=4))
     lm_head = time_lm_head(w, dev, peaks, ev_time)
+    sft = time_sft_attention(dev, peaks, ev_time)
     refresh = time_refresh(w, dev, stream, peaks, ev_time)
     loop = time_pass_loop(w, dev, reps=3)
     st, flags = mbe.get_device_error()
@@ -355,7 +356,7 @@ def time_extras(w, a0, dev, stream, peaks, reps=10):
                                "frac_hbm": round(byts / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"], 4),
                                "rows": R, "vocab": V},
             "tail_entropy_select": {"us": round(ms_sel * 1e3, 2), "sequences": a0.batch, "k_max": 4, "rho": 0.25},
-            "lm_head_edit_decide": lm_head, "refresh": refresh, "pass_loop": loop}
+            "lm_head_edit_decide": lm_head, "sft_attention": sft, "refresh": refresh, "pass_loop": loop}
 
 
 def time_lm_head(w, dev, peaks, ev_time, hidden=4096):
@@ -390,6 +391,48 @@ def time_lm_head(w, dev, peaks, ev_time, hidden=4096):
             "hidden": hidden, "cublas_gemm_ms": round(gemm, 4),
             "cublas_tflops": round(flops / (gemm * 1e-3) / 1e12, 1), "cublas_gemm_plus_edit_decide_ms": round(unf, 4),
             "note": "random bf16 weights; roofline bound: tensor"}
+
+
+def time_sft_attention(dev, peaks, ev_time, batch=4, n_prompt=4, n_blocks=64, K=4, B=32):
+    """Multi-Block Edit SFT attention (Sec. 3) on a seeded training batch: the
+    cross-block mask, the forward and the backward; FLOPs count visible token
+    pairs only (4 D Hq per pair forward, 10 D Hq backward)."""
+    from paper_2607_22663_gb300 import mbe
+    from paper_2607_22663_gb300.workloads import sft_problem
+    prob = sft_problem([n_prompt] * batch, [n_blocks] * batch, 32, 8, 128, B, seed=7, device=dev)
+    mask = mbe.sft_block_mask(prob.n_prompt_blocks, prob.n_blocks, K, prob.mask_rows)
+    T, Hq, D = prob.q.shape
+    Hkv = prob.k.shape[1]
+    nb = n_prompt + 2 * n_blocks
+    bits = mask[0].cpu().numpy().astype("int64") & 0xFFFFFFFF
+    visible = sum(bin(int(w)).count("1") for w in bits[:nb].ravel())
+    pairs = visible * B * B * batch
+    ws = torch.empty(mbe.window_attention_workspace_size(batch, Hq, Hkv, D, prob.max_seq_len, 0), dtype=torch.uint8,
+                     device=dev)
+    out = torch.empty_like(prob.q)
+    lse = torch.empty((T, Hq), dtype=torch.float32, device=dev)
+    bws = torch.empty(int(mbe.lib().mbe_block_mask_attention_bwd_workspace_size(batch, T, Hq)), dtype=torch.uint8,
+                      device=dev)
+    dq = torch.empty((T, Hq, D), dtype=torch.float32, device=dev)
+    dk = torch.empty((T, Hkv, D), dtype=torch.float32, device=dev)
+    dv = torch.empty_like(dk)
+    ms_mask = ev_time(lambda: mbe.sft_block_mask(prob.n_prompt_blocks, prob.n_blocks, K, prob.mask_rows, out=mask))
+    ms_f = ev_time(lambda: mbe.block_mask_attention(prob.q, prob.k, prob.v, prob.seq_len, prob.cu_seqlens, mask,
+                                                    block_size=B, max_seq_len=prob.max_seq_len, out=out, lse=lse,
+                                                    workspace=ws))
+    ms_b = ev_time(lambda: mbe.block_mask_attention_bwd(prob.q, prob.k, prob.v, out, prob.dout, lse, prob.seq_len,
+                                                        prob.cu_seqlens, mask, block_size=B,
+                                                        max_seq_len=prob.max_seq_len, dq=dq, dk=dk, dv=dv,
+                                                        workspace=bws))
+    tf_f = 4.0 * D * Hq * pairs / (ms_f * 1e-3) / 1e12
+    tf_b = 10.0 * D * Hq * pairs / (ms_b * 1e-3) / 1e12
+    return {"batch": batch, "seq_len": prob.max_seq_len, "heads_q_kv": [Hq, Hkv], "head_dim": D, "block_size": B,
+            "K": K, "mask_density": round(visible / (nb * nb), 4), "mask_us": round(ms_mask * 1e3, 2),
+            "fwd_ms": round(ms_f, 4), "fwd_tflops": round(tf_f, 1),
+            "fwd_frac_bf16_peak_burst": round(tf_f / peaks["bf16_tflops"], 4),
+            "bwd_ms": round(ms_b, 4), "bwd_tflops": round(tf_b, 1),
+            "bwd_frac_bf16_peak_burst": round(tf_b / peaks["bf16_tflops"], 4),
+            "note": "FLOPs of visible token pairs only; roofline bound: tensor"}
 
 
 class RefreshBuffers:

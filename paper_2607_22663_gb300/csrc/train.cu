@@ -152,7 +152,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ __align__(8) Bars bars;
   __shared__ Unit ring[2];
   __shared__ uint32_t ring_bits[2][kMaxQWords];
-  __shared__ float lse2_s[kTile], delta_s[kTile];
+  __shared__ float2 col_s[kTile];  // per query row of the tile: (lse in log2 units, delta)
   __shared__ int qrel_s[kTile];
   __shared__ uint32_t tmem_base_s;
   __shared__ int abort_s;
@@ -408,8 +408,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int tok = R / p.G, head = un.g * p.G + (R - tok * p.G);
           const bool qv = tok < un.len;
           const int64_t row = (static_cast<int64_t>(un.cu) + tok) * p.Hq + head;
-          lse2_s[r] = qv ? p.lse[row] * kLog2e : __int_as_float(0x7f800000);  // +inf: P = 0
-          delta_s[r] = qv ? p.delta[row] : 0.f;
+          col_s[r] = make_float2(qv ? p.lse[row] * kLog2e : __int_as_float(0x7f800000),  // +inf: P = 0
+                                 qv ? p.delta[row] : 0.f);
           qrel_s[r] = min((tok >> p.block_log2) - qb0, 31);
         }
         ok = group_sync();
@@ -417,6 +417,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // this key block against the (<= 32) query blocks of the tile
         uint32_t qvis = 0;
         const int qb_last = min(qb0 + 31, (min(un.len - 1, ((i + 1) * kTile - 1) / p.G)) >> p.block_log2);
+        const bool one_qblock = qb_last == qb0;  // every column in the same query block
         if (key_ok)
           for (int qb = qb0; qb <= qb_last; ++qb)
             if (mask_bit(p, un.seq, qb, kb)) qvis |= 1u << (qb - qb0);
@@ -432,10 +433,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
               const int col = 32 * c4 + jj + e;
-              const bool vis = (qvis >> qrel_s[col]) & 1u;
-              const float pr = vis ? ex2f(__uint_as_float(sv[jj + e]) * p.scale_log2 - lse2_s[col]) : 0.f;
+              const bool vis = one_qblock ? (qvis & 1u) : ((qvis >> qrel_s[col]) & 1u);
+              const float2 cd = col_s[col];
+              const float pr = vis ? ex2f(fmaf(__uint_as_float(sv[jj + e]), p.scale_log2, -cd.x)) : 0.f;
               pp[e] = pr;
-              ds[e] = pr * (__uint_as_float(dv[jj + e]) - delta_s[col]);
+              ds[e] = pr * (__uint_as_float(dv[jj + e]) - cd.y);
             }
             pw[jj / 2] = pack_bf16x2(pp[0], pp[1]);
             dsw[jj / 2] = pack_bf16x2(ds[0], ds[1]);
