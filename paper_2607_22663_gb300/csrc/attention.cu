@@ -800,9 +800,36 @@ __global__ void __launch_bounds__(kThreads, 1)
         // The whole S row (128 fp32) comes from TMEM in one load; P is packed to
         // bf16 in place (entry k <- columns 2k, 2k+1) and stored as 64 columns
         // over the start of the same TMEM region.
-        const bool full = __all_sync(0xffffffffu, n_vis == kTileKeys && (!kMask || nib == all_bits));
+        bool full = __all_sync(0xffffffffu, n_vis == kTileKeys && (!kMask || nib == all_bits));
         uint32_t v[128];
         tmem_ld128(tS, v);
+        if constexpr (kMask) {
+          // block-mask mode: invisible columns (other key blocks, past the sequence)
+          // become -inf and the tile takes the packed path (exp2(-inf) = 0)
+          if (!full) {
+            uint32_t cm[4];
+#pragma unroll
+            for (int w = 0; w < 4; ++w) {
+              uint32_t bits;
+              if (p.block_log2 >= 5) {
+                bits = ((nib >> ((32 * w) >> p.block_log2)) & 1u) ? 0xFFFFFFFFu : 0u;
+              } else {  // 8- or 16-token blocks: 32 / B blocks per word
+                const int per = 32 >> p.block_log2, base = (32 * w) >> p.block_log2;
+                const uint32_t run = (1u << (1 << p.block_log2)) - 1u;
+                bits = 0u;
+                for (int b = 0; b < per; ++b)
+                  if ((nib >> (base + b)) & 1u) bits |= run << (b << p.block_log2);
+              }
+              const int lo = 32 * w;
+              bits &= n_vis >= lo + 32 ? 0xFFFFFFFFu : (n_vis <= lo ? 0u : ((1u << (n_vis - lo)) - 1u));
+              cm[w] = bits;
+            }
+#pragma unroll
+            for (int k = 0; k < 128; ++k)
+              if (!((cm[k >> 5] >> (k & 31)) & 1u)) v[k] = 0xFF800000u;
+            full = true;
+          }
+        }
         float mx = neg_inf();
         if (full) {
           float a0 = neg_inf(), a1 = neg_inf();
