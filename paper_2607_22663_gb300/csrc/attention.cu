@@ -241,16 +241,22 @@ __global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p
     }
     atomicAdd(&hist[b], count);
   };
-  // one thread per (sequence, KV head) pair, so that few long sequences still
-  // spread their pieces over many threads
-  for (int sg = tid; sg < p.batch * p.Hkv; sg += blockDim.x) {
+  // one thread per (sequence, KV head, slab group), so that few long sequences
+  // still spread their pieces over many threads; a sequence with at most
+  // kMaxGroupedSlabs slabs forms one group, longer ones one group per slab
+  const int max_slabs = (p.max_window * p.G + kUnitRows - 1) / kUnitRows;
+  const int groups_per_sg = max_slabs > kMaxGroupedSlabs ? max_slabs : 1;
+  for (int64_t it = tid; it < static_cast<int64_t>(p.batch) * p.Hkv * groups_per_sg; it += blockDim.x) {
+    const int sg = static_cast<int>(it / groups_per_sg);
+    const int grp = static_cast<int>(it - static_cast<int64_t>(sg) * groups_per_sg);
     const int s = sg / p.Hkv, g = sg - s * p.Hkv;
     const int P = seq_prefix(p, s), W = p.window_len[s], mode = seq_mode(p, s);
     if (!seq_ok(p, s, P, W, mode)) continue;
     const int slabs = (W * p.G + kUnitRows - 1) / kUnitRows;
     const int ng = slabs <= kMaxGroupedSlabs ? slabs : 1;  // slabs per piece
+    if (grp * ng >= slabs) continue;
     {
-      for (int s0 = 0; s0 < slabs; s0 += ng) {
+      for (int s0 = grp * ng; s0 < min(slabs, (grp + 1) * ng); s0 += ng) {
         const int cnt = min(ng, slabs - s0);
         int T[kMaxGroupedSlabs], n[kMaxGroupedSlabs], slot0[kMaxGroupedSlabs];
         int nmax = 0;
