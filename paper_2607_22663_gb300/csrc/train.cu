@@ -7,21 +7,22 @@
 //
 // bwd_prep_kernel: delta = rowsum(dO o O) per (token, head), dQ zeroed, the
 // work counter armed.
-// bwd_kernel (persistent, one CTA per SM, 256 threads): a work unit is
+// bwd_kernel (persistent, one CTA per SM, 384 threads): a work unit is
 // (sequence, KV head g, 128-key tile); K and V stay in shared memory while the
 // unit walks the 128-row query tiles (packed rows token * G + head of the heads
 // of g) that see any of its key blocks. Per query tile:
-//   warp 0     TMA: Q_i and dO_i into a 2-stage ring (K, V once per unit)
-//   warp 1     MMA: S^T = K Q_i^T and dP^T = V dO_i^T (SS, into TMEM);
-//              then dV += P^T dO_i and dK += dS^T Q_i (TS, P^T and dS^T from
-//              TMEM) and dQ_i = dS K (SS, dS from shared memory)
-//   warps 4-7  thread = key row: P^T = exp(S^T * scale - lse), masked;
-//              dS^T = P^T o (dP^T - delta); P^T and dS^T back to TMEM as bf16,
-//              dS also into shared memory in the layout TMA gives a V tile;
-//              then thread = query row: dQ_i * scale added to dQ (fp32
-//              atomics); at the unit's end, thread = key row: dK * scale and dV
-//              stored (fp32).
-// TMEM: dK, dV, S^T/P^T/dQ and dP^T/dS^T, 128 columns each.
+//   warp 0      TMA: Q_i and dO_i into a 2-stage ring (K, V once per unit)
+//   warp 1      MMA: S^T = K Q_i^T and dP^T = V dO_i^T (SS, into TMEM); then
+//               dV += P^T dO_i (TS, P^T from TMEM), dK += dS^T Q_i and
+//               dQ_i = dS K (SS, dS from shared memory)
+//   warps 4-11  two warps per TMEM lane quadrant, splitting columns 0-63 /
+//               64-127; thread = key row: P^T = exp(S^T * scale - lse),
+//               masked, back to TMEM as bf16; dS^T = P^T o (dP^T - delta)
+//               into shared memory as a [key][query row] tile (K-major for
+//               dK, MN-major for dQ); then thread = query row: dQ_i * scale
+//               added to dQ (fp32 atomics); at the unit's end, thread = key
+//               row: dK * scale and dV stored (fp32).
+// TMEM: dK, dV, S^T/P^T/dQ and dP^T, 128 columns each.
 #include <cuda_bf16.h>
 #include <algorithm>
 #include <cmath>
@@ -79,7 +80,7 @@ namespace bwd {
 
 constexpr int kD = 128;                      // head size of the backward
 constexpr int kTile = 128;                   // keys per key tile = packed rows per query tile
-constexpr int kThreads = 256;
+constexpr int kThreads = 384;              // 4 role warps + 8 compute warps (two per TMEM lane quadrant)
 constexpr int kMaxQWords = 16;               // query-tile bitmask of a unit (<= 512 query tiles)
 constexpr uint32_t kHalf = 128 * 128;        // a 64-column half of a 128-row bf16 tile (16 KB)
 constexpr uint32_t kTileBytes = 2 * kHalf;   // 32 KB
@@ -166,20 +167,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     abort_s = 0;
     for (int i = 0; i < 2; ++i) {
       mbar_init(bar(bars.u_full[i]), 1);
-      mbar_init(bar(bars.u_empty[i]), 5);  // MMA issuer + 4 compute warps
+      mbar_init(bar(bars.u_empty[i]), 9);  // MMA issuer + 8 compute warps
       mbar_init(bar(bars.q_full[i]), 1);
       mbar_init(bar(bars.q_empty[i]), 1);
     }
     mbar_init(bar(bars.kv_full), 1);
     mbar_init(bar(bars.kv_empty), 1);
     mbar_init(bar(bars.s_full), 1);
-    mbar_init(bar(bars.p_full), 4);
+    mbar_init(bar(bars.p_full), 8);
     mbar_init(bar(bars.dq_full), 1);
-    mbar_init(bar(bars.dq_empty), 4);
+    mbar_init(bar(bars.dq_empty), 8);
     mbar_init(bar(bars.acc_full), 1);
-    mbar_init(bar(bars.acc_empty), 4);
+    mbar_init(bar(bars.acc_empty), 8);
     mbar_init(bar(bars.mma_done), 1);
-    mbar_init(bar(bars.group), 4);  // the compute warps among themselves
+    mbar_init(bar(bars.group), 8);  // the compute warps among themselves
     mbar_fence_init();
   }
   if (warp == 1) {
@@ -326,7 +327,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int kk = 0; kk < kTile / 16; ++kk) {
             const uint32_t acc = (j > 0 || kk > 0) ? 1u : 0u;
             umma_ts(tmem + kTmDV, tmem + kTmS + kk * 8, sdesc_sw128(da + kk * 16 * 128, kHalf, 1024), idesc_tb, acc);
-            umma_ts(tmem + kTmDK, tmem + kTmDP + kk * 8, sdesc_sw128(qa + kk * 16 * 128, kHalf, 1024), idesc_tb, acc);
+            // dS^T from shared memory: [key][query row] is K-major for A = dS^T
+            umma_ss(tmem + kTmDK, sdesc_sw128(sbase + kDS + (kk >> 2) * kHalf + (kk & 3) * 32, 16, 1024),
+                    sdesc_sw128(qa + kk * 16 * 128, kHalf, 1024), idesc_tb, acc);
           }
 #pragma unroll
           for (int kk = 0; kk < kTile / 16; ++kk)
@@ -353,11 +356,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp >= 4) {
     // ---------------------------------------------------------------- compute warps
     const int quad = warp & 3;
+    const int hf = (warp - 4) >> 2;  // the pair of warps of a quadrant splits columns 0-63 / 64-127
     const int r = quad * 32 + lane;  // TMEM lane: key row, or query row for dQ
     const uint32_t t_lane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
     uint32_t u_it = 0, units = 0, tiles = 0, syncs = 0;
     bool ok = true;
-    // bounded barrier of the four compute warps (orders the per-tile column data)
+    // bounded barrier of the eight compute warps
     auto group_sync = [&]() {
       __syncwarp();
       if (lane == 0) mbar_arrive(bar(bars.group));
@@ -385,13 +389,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int key = un.kt * kTile + r;
       const bool key_ok = key < un.len;
       const int64_t kv_row = (static_cast<int64_t>(un.cu) + key) * p.Hkv + un.g;
-      if (n_q == 0) {  // no query sees these keys: zero gradients
+      if (n_q == 0) {  // no query sees these keys: zero gradients (dK by one half, dV by the other)
         release();
+        float* dst = (hf == 0 ? p.dk : p.dv) + kv_row * kD;
         if (key_ok)
-          for (int d = 0; d < kD; d += 4) {
-            *reinterpret_cast<float4*>(p.dk + kv_row * kD + d) = make_float4(0.f, 0.f, 0.f, 0.f);
-            *reinterpret_cast<float4*>(p.dv + kv_row * kD + d) = make_float4(0.f, 0.f, 0.f, 0.f);
-          }
+          for (int d = 0; d < kD; d += 4) *reinterpret_cast<float4*>(dst + d) = make_float4(0.f, 0.f, 0.f, 0.f);
         continue;
       }
       const int kb = key >> p.block_log2;
@@ -403,7 +405,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int qb0 = ((i * kTile) / p.G) >> p.block_log2;
         ok = group_sync();  // every warp is done with the previous tile's column data
         if (!ok) break;
-        {
+        if (hf == 0) {
           const int R = i * kTile + r;
           const int tok = R / p.G, head = un.g * p.G + (R - tok * p.G);
           const bool qv = tok < un.len;
@@ -421,35 +423,47 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (key_ok)
           for (int qb = qb0; qb <= qb_last; ++qb)
             if (mask_bit(p, un.seq, qb, kb)) qvis |= 1u << (qb - qb0);
-#pragma unroll 1
-        for (int c4 = 0; c4 < kTile / 32; ++c4) {
-          uint32_t sv[32], dv[32];
-          tmem_ld32(t_lane + kTmS + 32 * c4, sv);
-          tmem_ld32(t_lane + kTmDP + 32 * c4, dv);
-          uint32_t pw[16], dsw[16];
+        // P^T of this warp's 64 columns, packed to bf16 pairs
+        uint32_t pw[32];
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          uint32_t sv[32];
+          tmem_ld32(t_lane + kTmS + 64 * hf + 32 * c, sv);
 #pragma unroll
           for (int jj = 0; jj < 32; jj += 2) {
-            float pp[2], ds[2];
+            float pp[2];
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
-              const int col = 32 * c4 + jj + e;
+              const int col = 64 * hf + 32 * c + jj + e;
               const bool vis = one_qblock ? (qvis & 1u) : ((qvis >> qrel_s[col]) & 1u);
-              const float2 cd = col_s[col];
-              const float pr = vis ? ex2f(fmaf(__uint_as_float(sv[jj + e]), p.scale_log2, -cd.x)) : 0.f;
-              pp[e] = pr;
-              ds[e] = pr * (__uint_as_float(dv[jj + e]) - cd.y);
+              pp[e] = vis ? ex2f(fmaf(__uint_as_float(sv[jj + e]), p.scale_log2, -col_s[col].x)) : 0.f;
             }
-            pw[jj / 2] = pack_bf16x2(pp[0], pp[1]);
-            dsw[jj / 2] = pack_bf16x2(ds[0], ds[1]);
+            pw[16 * c + jj / 2] = pack_bf16x2(pp[0], pp[1]);
           }
-          tmem_st16(t_lane + kTmS + 16 * c4, pw);
-          tmem_st16(t_lane + kTmDP + 16 * c4, dsw);
-          // dS into shared memory as row r of a [key][query row] tile, 128-byte swizzle
-          const int h = c4 >> 1;
+        }
+        // P^T overwrites S^T columns 32 hf .. 32 hf + 31, which the other half of the
+        // pair reads: store only once every warp has loaded its S^T columns
+        ok = group_sync();
+        if (!ok) break;
+        tmem_st32(t_lane + kTmS + 32 * hf, pw);
+        // dS^T = P^T o (dP^T - delta) into shared memory: row r of a [key][query row] tile
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          uint32_t dv[32];
+          tmem_ld32(t_lane + kTmDP + 64 * hf + 32 * c, dv);
+          uint32_t dsw[16];
+#pragma unroll
+          for (int jj = 0; jj < 32; jj += 2) {
+            const uint32_t pk = pw[16 * c + jj / 2];
+            const float p0 = __uint_as_float(pk << 16), p1 = __uint_as_float(pk & 0xFFFF0000u);
+            const int col = 64 * hf + 32 * c + jj;
+            dsw[jj / 2] = pack_bf16x2(p0 * (__uint_as_float(dv[jj]) - col_s[col].y),
+                                      p1 * (__uint_as_float(dv[jj + 1]) - col_s[col + 1].y));
+          }
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
-            const int chunk = ((c4 & 1) * 4 + q) ^ (r & 7);
-            *reinterpret_cast<uint4*>(smem + kDS + h * kHalf + r * 128 + chunk * 16) =
+            const int chunk = (c * 4 + q) ^ (r & 7);
+            *reinterpret_cast<uint4*>(smem + kDS + hf * kHalf + r * 128 + chunk * 16) =
                 make_uint4(dsw[4 * q], dsw[4 * q + 1], dsw[4 * q + 2], dsw[4 * q + 3]);
           }
         }
@@ -458,7 +472,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(bar(bars.p_full));
-        // dQ of this query tile: thread = query row
+        // dQ of this query tile: thread = query row, the pair splits the head dimension
         ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.dq_full), tiles & 1, abort_flag));
         if (!ok) break;
         tc_fence_after();
@@ -466,15 +480,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int R = i * kTile + r;
           const int tok = R / p.G, head = un.g * p.G + (R - tok * p.G);
           const bool qv = tok < un.len;
-          float* dst = p.dq + ((static_cast<int64_t>(un.cu) + tok) * p.Hq + head) * kD;
+          float* dst = p.dq + ((static_cast<int64_t>(un.cu) + tok) * p.Hq + head) * kD + 64 * hf;
 #pragma unroll 1
-          for (int c4 = 0; c4 < kD / 32; ++c4) {
+          for (int c = 0; c < 2; ++c) {
             uint32_t o[32];
-            tmem_ld32(t_lane + kTmS + 32 * c4, o);
+            tmem_ld32(t_lane + kTmS + 64 * hf + 32 * c, o);
             if (qv)
 #pragma unroll
               for (int e = 0; e < 32; e += 4)
-                atomicAdd(reinterpret_cast<float4*>(dst + 32 * c4 + e),
+                atomicAdd(reinterpret_cast<float4*>(dst + 32 * c + e),
                           make_float4(__uint_as_float(o[e]) * p.scale, __uint_as_float(o[e + 1]) * p.scale,
                                       __uint_as_float(o[e + 2]) * p.scale, __uint_as_float(o[e + 3]) * p.scale));
           }
@@ -486,25 +500,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (!ok) break;
       release();
-      // dK and dV of the unit's keys: thread = key row
+      // dK (first half of the pair) and dV (second half) of the unit's keys: thread = key row
       ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.acc_full), units & 1, abort_flag));
       if (!ok) break;
       tc_fence_after();
+      {
+        const uint32_t src = hf == 0 ? kTmDK : kTmDV;
+        const float mul = hf == 0 ? p.scale : 1.f;
+        float* dst = (hf == 0 ? p.dk : p.dv) + kv_row * kD;
 #pragma unroll 1
-      for (int c4 = 0; c4 < kD / 32; ++c4) {
-        uint32_t a[32], b[32];
-        tmem_ld32(t_lane + kTmDK + 32 * c4, a);
-        tmem_ld32(t_lane + kTmDV + 32 * c4, b);
-        if (key_ok)
+        for (int c4 = 0; c4 < kD / 32; ++c4) {
+          uint32_t a[32];
+          tmem_ld32(t_lane + src + 32 * c4, a);
+          if (key_ok)
 #pragma unroll
-          for (int e = 0; e < 32; e += 4) {
-            *reinterpret_cast<float4*>(p.dk + kv_row * kD + 32 * c4 + e) =
-                make_float4(__uint_as_float(a[e]) * p.scale, __uint_as_float(a[e + 1]) * p.scale,
-                            __uint_as_float(a[e + 2]) * p.scale, __uint_as_float(a[e + 3]) * p.scale);
-            *reinterpret_cast<float4*>(p.dv + kv_row * kD + 32 * c4 + e) =
-                make_float4(__uint_as_float(b[e]), __uint_as_float(b[e + 1]), __uint_as_float(b[e + 2]),
-                            __uint_as_float(b[e + 3]));
-          }
+            for (int e = 0; e < 32; e += 4)
+              *reinterpret_cast<float4*>(dst + 32 * c4 + e) =
+                  make_float4(__uint_as_float(a[e]) * mul, __uint_as_float(a[e + 1]) * mul,
+                              __uint_as_float(a[e + 2]) * mul, __uint_as_float(a[e + 3]) * mul);
+        }
       }
       tc_fence_before();
       __syncwarp();
