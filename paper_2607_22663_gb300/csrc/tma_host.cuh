@@ -1,6 +1,6 @@
 // Host side of the TMA tensor maps: cuTensorMapEncodeTiled reached through the
-// runtime's driver entry point (no link against libcuda), for bf16 tensors
-// with 128-byte swizzle, the layout the tcgen05 operand descriptors expect.
+// runtime's driver entry point (no link against libcuda), for bf16 and fp32
+// tensors with 128-byte swizzle, the layout the tcgen05 operand descriptors expect.
 #pragma once
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -28,14 +28,23 @@ inline EncodeTiledFn encode_fn() {
 
 // dims/strides/box in the driver's order (innermost first); strides[i] is the
 // byte stride of dimension i + 1. Out-of-range elements of a box read as zero.
-inline bool encode_bf16_sw128(CUtensorMap* tm, const void* base, int rank, const cuuint64_t* dims,
-                              const cuuint64_t* strides, const cuuint32_t* box) {
+inline bool encode_sw128(CUtensorMap* tm, CUtensorMapDataType type, const void* base, int rank,
+                         const cuuint64_t* dims, const cuuint64_t* strides, const cuuint32_t* box) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint32_t es[5] = {1, 1, 1, 1, 1};
-  return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+  return fn(tm, type, rank, const_cast<void*>(base), dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+inline bool encode_bf16_sw128(CUtensorMap* tm, const void* base, int rank, const cuuint64_t* dims,
+                              const cuuint64_t* strides, const cuuint32_t* box) {
+  return encode_sw128(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, base, rank, dims, strides, box);
+}
+// fp32 tensors (the inner box extent is then at most 32 elements: 128 bytes)
+inline bool encode_f32_sw128(CUtensorMap* tm, const void* base, int rank, const cuuint64_t* dims,
+                             const cuuint64_t* strides, const cuuint32_t* box) {
+  return encode_sw128(tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, base, rank, dims, strides, box);
 }
 
 }  // namespace mbe

@@ -10,19 +10,24 @@
 // bwd_kernel (persistent, one CTA per SM, 384 threads): a work unit is
 // (sequence, KV head g, 128-key tile); K and V stay in shared memory while the
 // unit walks the 128-row query tiles (packed rows token * G + head of the heads
-// of g) that see any of its key blocks. Per query tile:
-//   warp 0      TMA: Q_i and dO_i into a 2-stage ring (K, V once per unit)
-//   warp 1      MMA: S^T = K Q_i^T and dP^T = V dO_i^T (SS, into TMEM); then
-//               dV += P^T dO_i (TS, P^T from TMEM), dK += dS^T Q_i and
-//               dQ_i = dS K (SS, dS from shared memory)
+// of g) that see any of its key blocks. Per query tile i:
+//   warp 0      TMA: Q_i and dO_i into a 2-stage ring (K, V once per unit);
+//               the tile's column data (lse, delta, which query blocks see
+//               each key block of the unit) into shared memory
+//   warp 1      MMA: S^T = K Q_i^T (SS, into TMEM); dP^T = V dO_i^T once the
+//               dQ of tile i-1 has left TMEM; then dV += P^T dO_i (TS, P^T
+//               from TMEM), dK += dS^T Q_i and dQ_i = dS K (SS, dS from
+//               shared memory). S^T of tile i+1 follows dQ_i at once, so it
+//               runs while the compute warps read dQ_i out.
 //   warps 4-11  two warps per TMEM lane quadrant, splitting columns 0-63 /
 //               64-127; thread = key row: P^T = exp(S^T * scale - lse),
-//               masked, back to TMEM as bf16; dS^T = P^T o (dP^T - delta)
-//               into shared memory as a [key][query row] tile (K-major for
-//               dK, MN-major for dQ); then thread = query row: dQ_i * scale
-//               added to dQ (fp32 atomics); at the unit's end, thread = key
-//               row: dK * scale and dV stored (fp32).
-// TMEM: dK, dV, S^T/P^T/dQ and dP^T, 128 columns each.
+//               masked, back to TMEM as bf16 over the warp's own S^T columns;
+//               dS^T = P^T o (dP^T - delta) into shared memory as a [key][query
+//               row] tile (K-major for dK, MN-major for dQ); then thread =
+//               query row: dQ_i * scale into the stage Q_i and dO_i came in,
+//               as 32 x 32 fp32 boxes that TMA adds into dQ in L2; at the
+//               unit's end, thread = key row: dK * scale and dV stored (fp32).
+// TMEM: dK, dV, S^T/P^T and dP^T/dQ, 128 columns each.
 #include <cuda_bf16.h>
 #include <algorithm>
 #include <cmath>
@@ -80,12 +85,15 @@ namespace bwd {
 
 constexpr int kD = 128;                      // head size of the backward
 constexpr int kTile = 128;                   // keys per key tile = packed rows per query tile
-constexpr int kThreads = 384;              // 4 role warps + 8 compute warps (two per TMEM lane quadrant)
+constexpr int kThreads = 384;                // 4 role warps + 8 compute warps (two per TMEM lane quadrant)
 constexpr int kMaxQWords = 16;               // query-tile bitmask of a unit (<= 512 query tiles)
+constexpr int kMaxKeyBlocks = 16;            // key blocks of a 128-key tile (block size >= 8)
 constexpr uint32_t kHalf = 128 * 128;        // a 64-column half of a 128-row bf16 tile (16 KB)
 constexpr uint32_t kTileBytes = 2 * kHalf;   // 32 KB
-constexpr uint32_t kK = 0, kV = kTileBytes, kQ = 2 * kTileBytes, kDO = 4 * kTileBytes, kDS = 6 * kTileBytes;
-constexpr uint32_t kSmemBytes = 7 * kTileBytes + 1024;
+constexpr uint32_t kStageBytes = 2 * kTileBytes;  // Q_i and dO_i, then the fp32 dQ_i of the same tile
+constexpr uint32_t kBoxBytes = 32 * 128;     // a dQ box: 32 rows x 32 fp32 (one 128-byte row each)
+constexpr uint32_t kK = 0, kV = kTileBytes, kStage = 2 * kTileBytes, kDS = kStage + 2 * kStageBytes;
+constexpr uint32_t kSmemBytes = kDS + kTileBytes + 1024;  // + 1024-byte alignment slack
 constexpr uint32_t kTmDK = 0, kTmDV = 128, kTmS = 256, kTmDP = 384, kTmCols = 512;
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -97,11 +105,10 @@ struct Params {
   const float* delta;
   const int32_t* unit_start;  // [batch + 1]: first work unit of each sequence
   int* counter;
-  float* dq;
   float* dk;
   float* dv;
   int mask_rows, mask_words, block_log2;
-  int batch, total_tokens, Hq, Hkv, G;
+  int batch, total_tokens, Hq, Hkv, G, lgG;
   float scale, scale_log2;
 };
 
@@ -110,8 +117,8 @@ struct Unit {
 };
 
 struct Bars {
-  uint64_t u_full[2], u_empty[2], q_full[2], q_empty[2], kv_full, kv_empty, s_full, p_full, dq_full, dq_empty,
-      acc_full, acc_empty, mma_done, group;
+  uint64_t u_full[2], u_empty[2], q_full[2], q_empty[2], kv_full, kv_empty, col_full, col_empty, s_full, dp_full,
+      p_full, dq_full, dq_empty, acc_full, acc_empty, mma_done;
 };
 
 __device__ __forceinline__ float ex2f(float x) {
@@ -127,7 +134,7 @@ __device__ __forceinline__ bool mask_bit(const Params& p, int seq, int qb, int k
 
 // Does any query block of query tile i see a key block of key tile kt?
 __device__ __forceinline__ bool qtile_visible(const Params& p, const Unit& u, int i) {
-  const int q0 = (i * kTile) / p.G, q1 = min(u.len, ((i + 1) * kTile) / p.G) - 1;
+  const int q0 = (i * kTile) >> p.lgG, q1 = min(u.len, ((i + 1) * kTile) >> p.lgG) - 1;
   const int k0 = u.kt * kTile, k1 = min(u.len, k0 + kTile) - 1;
   if (q1 < q0 || k1 < k0) return false;
   for (int qb = q0 >> p.block_log2; qb <= (q1 >> p.block_log2); ++qb)
@@ -145,16 +152,26 @@ __device__ __forceinline__ int next_bit(const volatile uint32_t* bits, int i) {
   return -1;
 }
 
+// First and (capped) last query block of query tile i.
+__device__ __forceinline__ int qblock0(const Params& p, int i) { return ((i * kTile) >> p.lgG) >> p.block_log2; }
+__device__ __forceinline__ int qblock_count(const Params& p, const Unit& u, int i) {
+  const int last = min(u.len - 1, ((i + 1) * kTile - 1) >> p.lgG) >> p.block_log2;
+  return min(32, last - qblock0(p, i) + 1);
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     bwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_do,
-               const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v, const Params p) {
+               const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+               const __grid_constant__ CUtensorMap tm_dq, const Params p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   __shared__ __align__(8) Bars bars;
   __shared__ Unit ring[2];
   __shared__ uint32_t ring_bits[2][kMaxQWords];
-  __shared__ float2 col_s[kTile];  // per query row of the tile: (lse in log2 units, delta)
-  __shared__ int qrel_s[kTile];
+  // column data of the current query tile, written by the producer warp
+  __shared__ __align__(16) float col_lse[kTile];    // lse in log2 units; +inf past the sequence (P = 0)
+  __shared__ __align__(16) float col_delta[kTile];  // rowsum(dO o O)
+  __shared__ uint32_t col_kvis[kMaxKeyBlocks];      // per key block of the unit: bit b = query block qb0 + b sees it
   __shared__ uint32_t tmem_base_s;
   __shared__ int abort_s;
   volatile int* abort_flag = &abort_s;
@@ -169,18 +186,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(bar(bars.u_full[i]), 1);
       mbar_init(bar(bars.u_empty[i]), 9);  // MMA issuer + 8 compute warps
       mbar_init(bar(bars.q_full[i]), 1);
-      mbar_init(bar(bars.q_empty[i]), 1);
+      mbar_init(bar(bars.q_empty[i]), 8);  // each compute warp once its dQ boxes have been read
     }
     mbar_init(bar(bars.kv_full), 1);
     mbar_init(bar(bars.kv_empty), 1);
+    mbar_init(bar(bars.col_full), 1);
+    mbar_init(bar(bars.col_empty), 8);
     mbar_init(bar(bars.s_full), 1);
+    mbar_init(bar(bars.dp_full), 1);
     mbar_init(bar(bars.p_full), 8);
     mbar_init(bar(bars.dq_full), 1);
     mbar_init(bar(bars.dq_empty), 8);
     mbar_init(bar(bars.acc_full), 1);
     mbar_init(bar(bars.acc_empty), 8);
     mbar_init(bar(bars.mma_done), 1);
-    mbar_init(bar(bars.group), 8);  // the compute warps among themselves
     mbar_fence_init();
   }
   if (warp == 1) {
@@ -200,7 +219,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tm_k);
       tma_prefetch_desc(&tm_v);
     }
-    uint32_t u_it = 0, kv_loads = 0, q_it = 0;
+    uint32_t u_it = 0, kv_loads = 0, q_loads = 0, cols = 0;
     bool ok = true;
     for (;;) {
       int uidx = 0;
@@ -223,7 +242,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int tiles = (len + kTile - 1) / kTile;
         const int r = uidx - p.unit_start[lo];
         un = Unit{lo, r / max(tiles, 1), r % max(tiles, 1), len, p.cu[lo]};
-        const int n_qt = (len * p.G + kTile - 1) / kTile;
+        const int n_qt = ((len << p.lgG) + kTile - 1) / kTile;
         for (int w = 0; w < kMaxQWords; ++w) {
           const int i = 32 * w + lane;
           const uint32_t word = __ballot_sync(kAll, i < n_qt && qtile_visible(p, un, i));
@@ -253,22 +272,54 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       ++kv_loads;
+      const int kb_first = (un.kt * kTile) >> p.block_log2;
+      const int kb_last = (min(un.len, (un.kt + 1) * kTile) - 1) >> p.block_log2;
       for (int i = next_bit(bits, -1); i >= 0 && ok; i = next_bit(bits, i)) {
-        const uint32_t st = q_it & 1;
-        if (q_it >= 2) {
-          ok = __all_sync(kAll, mbar_wait(bar(bars.q_empty[st]), ((q_it >> 1) - 1) & 1, abort_flag));
+        const uint32_t st = q_loads & 1;
+        if (q_loads >= 2) {
+          ok = __all_sync(kAll, mbar_wait(bar(bars.q_empty[st]), ((q_loads >> 1) - 1) & 1, abort_flag));
           if (!ok) break;
         }
         if (lane == 0) {
-          mbar_arrive_expect_tx(bar(bars.q_full[st]), 2 * kTileBytes);
-          const int tok = un.cu + (i * kTile) / p.G;
+          const uint32_t qa = sbase + kStage + st * kStageBytes;
+          mbar_arrive_expect_tx(bar(bars.q_full[st]), kStageBytes);
+          const int tok = un.cu + ((i * kTile) >> p.lgG);
           for (int h = 0; h < 2; ++h) {
-            tma_load_3d(sbase + kQ + st * kTileBytes + h * kHalf, &tm_q, bar(bars.q_full[st]), h * 64, un.g * p.G, tok);
-            tma_load_3d(sbase + kDO + st * kTileBytes + h * kHalf, &tm_do, bar(bars.q_full[st]), h * 64, un.g * p.G,
-                        tok);
+            tma_load_3d(qa + h * kHalf, &tm_q, bar(bars.q_full[st]), h * 64, un.g * p.G, tok);
+            tma_load_3d(qa + kTileBytes + h * kHalf, &tm_do, bar(bars.q_full[st]), h * 64, un.g * p.G, tok);
           }
         }
-        ++q_it;
+        ++q_loads;
+        // column data of tile i, fetched before waiting for the compute warps to
+        // finish with the previous tile's
+        float lse_r[4], dl_r[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int R = i * kTile + lane + 32 * e;
+          const int tok = R >> p.lgG, head = un.g * p.G + (R & (p.G - 1));
+          const bool qv = tok < un.len;
+          const int64_t row = (static_cast<int64_t>(un.cu) + tok) * p.Hq + head;
+          lse_r[e] = qv ? p.lse[row] * kLog2e : __int_as_float(0x7f800000);
+          dl_r[e] = qv ? p.delta[row] : 0.f;
+        }
+        const int qb0 = qblock0(p, i), nqb = qblock_count(p, un, i);
+        uint32_t kvis = 0;
+        if (lane < kMaxKeyBlocks && kb_first + lane <= kb_last)
+          for (int b = 0; b < nqb; ++b)
+            if (mask_bit(p, un.seq, qb0 + b, kb_first + lane)) kvis |= 1u << b;
+        if (cols >= 1) {
+          ok = __all_sync(kAll, mbar_wait(bar(bars.col_empty), (cols - 1) & 1, abort_flag));
+          if (!ok) break;
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          col_lse[lane + 32 * e] = lse_r[e];
+          col_delta[lane + 32 * e] = dl_r[e];
+        }
+        if (lane < kMaxKeyBlocks) col_kvis[lane] = kvis;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(bars.col_full));
+        ++cols;
       }
       if (!ok) break;
     }
@@ -278,15 +329,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       // let the copies already issued land before the CTA can exit
       const int zero = 0;
       if (kv_loads >= 1) mbar_wait(bar(bars.kv_full), (kv_loads - 1) & 1, &zero);
-      for (uint32_t n = (q_it >= 2 ? q_it - 2 : 0); n < q_it; ++n) mbar_wait(bar(bars.q_full[n & 1]), (n >> 1) & 1, &zero);
+      for (uint32_t n = (q_loads >= 2 ? q_loads - 2 : 0); n < q_loads; ++n)
+        mbar_wait(bar(bars.q_full[n & 1]), (n >> 1) & 1, &zero);
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc_kk = idesc_bf16_f32(kTile, kTile, false, false);  // S^T, dP^T
-      constexpr uint32_t idesc_tb = idesc_bf16_f32(kTile, kD, false, true);      // dV, dK: TMEM A, MN-major B
+      constexpr uint32_t idesc_tb = idesc_bf16_f32(kTile, kD, false, true);      // dV, dK: MN-major B
       constexpr uint32_t idesc_dq = idesc_bf16_f32(kTile, kD, true, true);       // dQ: MN-major A and B
-      uint32_t u_it = 0, units = 0, q_it = 0, tiles = 0;
+      uint32_t u_it = 0, units = 0, tiles = 0;
       bool ok = true;
       for (;;) {
         const int slot = u_it & 1;
@@ -299,13 +351,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (un.seq < 0) break;
         if (n_q == 0) continue;
         if (!mbar_wait(bar(bars.kv_full), units & 1, abort_flag)) { ok = false; break; }
-        tc_fence_after();
-        for (int j = 0; j < n_q; ++j) {
-          const uint32_t st = q_it & 1;
-          if (!mbar_wait(bar(bars.q_full[st]), (q_it >> 1) & 1, abort_flag)) { ok = false; break; }
-          if (tiles >= 1 && !mbar_wait(bar(bars.dq_empty), (tiles - 1) & 1, abort_flag)) { ok = false; break; }
+        for (int j = 0; j < n_q; ++j, ++tiles) {
+          const uint32_t st = tiles & 1;
+          if (!mbar_wait(bar(bars.q_full[st]), (tiles >> 1) & 1, abort_flag)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t qa = sbase + kQ + st * kTileBytes, da = sbase + kDO + st * kTileBytes;
+          const uint32_t qa = sbase + kStage + st * kStageBytes, da = qa + kTileBytes;
+          // S^T = K Q_i^T over the previous tile's P^T (read by MMAs issued before)
 #pragma unroll
           for (int h = 0; h < 2; ++h)
 #pragma unroll
@@ -313,10 +364,20 @@ __global__ void __launch_bounds__(kThreads, 1)
               const uint32_t off = h * kHalf + k * 32;
               umma_ss(tmem + kTmS, sdesc_sw128(sbase + kK + off, 16, 1024), sdesc_sw128(qa + off, 16, 1024), idesc_kk,
                       (h | k) ? 1u : 0u);
-              umma_ss(tmem + kTmDP, sdesc_sw128(sbase + kV + off, 16, 1024), sdesc_sw128(da + off, 16, 1024), idesc_kk,
-                      (h | k) ? 1u : 0u);
             }
           umma_commit(bar(bars.s_full));
+          // dP^T = V dO_i^T, once the previous tile's dQ has been read out of the region
+          if (tiles >= 1 && !mbar_wait(bar(bars.dq_empty), (tiles - 1) & 1, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+#pragma unroll
+          for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const uint32_t off = h * kHalf + k * 32;
+              umma_ss(tmem + kTmDP, sdesc_sw128(sbase + kV + off, 16, 1024), sdesc_sw128(da + off, 16, 1024),
+                      idesc_kk, (h | k) ? 1u : 0u);
+            }
+          umma_commit(bar(bars.dp_full));
           if (!mbar_wait(bar(bars.p_full), tiles & 1, abort_flag)) { ok = false; break; }
           if (j == 0 && units >= 1 && !mbar_wait(bar(bars.acc_empty), (units - 1) & 1, abort_flag)) {
             ok = false;
@@ -326,19 +387,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int kk = 0; kk < kTile / 16; ++kk) {
             const uint32_t acc = (j > 0 || kk > 0) ? 1u : 0u;
-            umma_ts(tmem + kTmDV, tmem + kTmS + kk * 8, sdesc_sw128(da + kk * 16 * 128, kHalf, 1024), idesc_tb, acc);
+            // P^T of query columns 64 h .. 64 h + 63 sits packed at S region columns 64 h .. 64 h + 31
+            umma_ts(tmem + kTmDV, tmem + kTmS + (kk >> 2) * 64 + (kk & 3) * 8,
+                    sdesc_sw128(da + kk * 16 * 128, kHalf, 1024), idesc_tb, acc);
             // dS^T from shared memory: [key][query row] is K-major for A = dS^T
             umma_ss(tmem + kTmDK, sdesc_sw128(sbase + kDS + (kk >> 2) * kHalf + (kk & 3) * 32, 16, 1024),
                     sdesc_sw128(qa + kk * 16 * 128, kHalf, 1024), idesc_tb, acc);
           }
+          // dQ_i = dS K (the same tile as MN-major A) into the dP region
 #pragma unroll
           for (int kk = 0; kk < kTile / 16; ++kk)
-            umma_ss(tmem + kTmS, sdesc_sw128(sbase + kDS + kk * 16 * 128, kHalf, 1024),
+            umma_ss(tmem + kTmDP, sdesc_sw128(sbase + kDS + kk * 16 * 128, kHalf, 1024),
                     sdesc_sw128(sbase + kK + kk * 16 * 128, kHalf, 1024), idesc_dq, kk > 0 ? 1u : 0u);
           umma_commit(bar(bars.dq_full));
-          umma_commit(bar(bars.q_empty[st]));
-          ++q_it;
-          ++tiles;
         }
         if (!ok) break;
         umma_commit(bar(bars.acc_full));
@@ -359,16 +420,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int hf = (warp - 4) >> 2;  // the pair of warps of a quadrant splits columns 0-63 / 64-127
     const int r = quad * 32 + lane;  // TMEM lane: key row, or query row for dQ
     const uint32_t t_lane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
-    uint32_t u_it = 0, units = 0, tiles = 0, syncs = 0;
+    const int sh = p.lgG + p.block_log2;  // packed row -> query block
+    uint32_t u_it = 0, units = 0, tiles = 0;
     bool ok = true;
-    // bounded barrier of the eight compute warps
-    auto group_sync = [&]() {
-      __syncwarp();
-      if (lane == 0) mbar_arrive(bar(bars.group));
-      const bool done = __all_sync(0xffffffffu, mbar_wait(bar(bars.group), syncs & 1, abort_flag));
-      ++syncs;
-      return done;
-    };
     for (;;) {
       const int slot = u_it & 1;
       ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag));
@@ -396,69 +450,74 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int d = 0; d < kD; d += 4) *reinterpret_cast<float4*>(dst + d) = make_float4(0.f, 0.f, 0.f, 0.f);
         continue;
       }
-      const int kb = key >> p.block_log2;
-      for (int i = next_bit(bits, -1); i >= 0; i = next_bit(bits, i)) {
+      const int kb_rel = (key >> p.block_log2) - ((un.kt * kTile) >> p.block_log2);
+      for (int i = next_bit(bits, -1); i >= 0; i = next_bit(bits, i), ++tiles) {
+        const uint32_t st = tiles & 1;
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.col_full), tiles & 1, abort_flag));
+        if (!ok) break;
         ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.s_full), tiles & 1, abort_flag));
         if (!ok) break;
         tc_fence_after();
-        // per-column data of query tile i: lse (log2 units), delta, query block
-        const int qb0 = ((i * kTile) / p.G) >> p.block_log2;
-        ok = group_sync();  // every warp is done with the previous tile's column data
-        if (!ok) break;
-        if (hf == 0) {
-          const int R = i * kTile + r;
-          const int tok = R / p.G, head = un.g * p.G + (R - tok * p.G);
-          const bool qv = tok < un.len;
-          const int64_t row = (static_cast<int64_t>(un.cu) + tok) * p.Hq + head;
-          col_s[r] = make_float2(qv ? p.lse[row] * kLog2e : __int_as_float(0x7f800000),  // +inf: P = 0
-                                 qv ? p.delta[row] : 0.f);
-          qrel_s[r] = min((tok >> p.block_log2) - qb0, 31);
-        }
-        ok = group_sync();
-        if (!ok) break;
-        // this key block against the (<= 32) query blocks of the tile
-        uint32_t qvis = 0;
-        const int qb_last = min(qb0 + 31, (min(un.len - 1, ((i + 1) * kTile - 1) / p.G)) >> p.block_log2);
-        const bool one_qblock = qb_last == qb0;  // every column in the same query block
-        if (key_ok)
-          for (int qb = qb0; qb <= qb_last; ++qb)
-            if (mask_bit(p, un.seq, qb, kb)) qvis |= 1u << (qb - qb0);
+        const int qb0 = qblock0(p, i), nqb = qblock_count(p, un, i);
+        const uint32_t all = nqb >= 32 ? 0xFFFFFFFFu : ((1u << nqb) - 1u);
+        // query blocks of this tile that see this key row's block
+        const uint32_t qvis = key_ok ? (col_kvis[kb_rel] & all) : 0u;
+        // TMEM loads are warp-wide: the warp skips them only if no lane needs them
+        const bool any_vis = __any_sync(0xffffffffu, qvis != 0u);
+        const bool every = __all_sync(0xffffffffu, qvis == all);
         // P^T of this warp's 64 columns, packed to bf16 pairs
         uint32_t pw[32];
+        if (!any_vis) {
 #pragma unroll
-        for (int c = 0; c < 2; ++c) {
-          uint32_t sv[32];
-          tmem_ld32(t_lane + kTmS + 64 * hf + 32 * c, sv);
+          for (int m = 0; m < 32; ++m) pw[m] = 0u;
+        } else {
 #pragma unroll
-          for (int jj = 0; jj < 32; jj += 2) {
-            float pp[2];
+          for (int c = 0; c < 2; ++c) {
+            uint32_t sv[32];
+            tmem_ld32(t_lane + kTmS + 64 * hf + 32 * c, sv);
 #pragma unroll
-            for (int e = 0; e < 2; ++e) {
-              const int col = 64 * hf + 32 * c + jj + e;
-              const bool vis = one_qblock ? (qvis & 1u) : ((qvis >> qrel_s[col]) & 1u);
-              pp[e] = vis ? ex2f(fmaf(__uint_as_float(sv[jj + e]), p.scale_log2, -col_s[col].x)) : 0.f;
+            for (int jj = 0; jj < 32; jj += 4) {
+              const int col = 64 * hf + 32 * c + jj;
+              const float4 l4 = *reinterpret_cast<const float4*>(&col_lse[col]);
+              float x[4] = {fmaf(__uint_as_float(sv[jj]), p.scale_log2, -l4.x),
+                            fmaf(__uint_as_float(sv[jj + 1]), p.scale_log2, -l4.y),
+                            fmaf(__uint_as_float(sv[jj + 2]), p.scale_log2, -l4.z),
+                            fmaf(__uint_as_float(sv[jj + 3]), p.scale_log2, -l4.w)};
+              if (!every) {
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                  if (!((qvis >> (((i * kTile + col + e) >> sh) - qb0)) & 1u)) x[e] = __int_as_float(0xff800000);
+              }
+              pw[16 * c + jj / 2] = pack_bf16x2(ex2f(x[0]), ex2f(x[1]));
+              pw[16 * c + jj / 2 + 1] = pack_bf16x2(ex2f(x[2]), ex2f(x[3]));
             }
-            pw[16 * c + jj / 2] = pack_bf16x2(pp[0], pp[1]);
           }
         }
-        // P^T overwrites S^T columns 32 hf .. 32 hf + 31, which the other half of the
-        // pair reads: store only once every warp has loaded its S^T columns
-        ok = group_sync();
+        // P^T over S^T columns this warp has already read: 64 hf .. 64 hf + 31
+        tmem_st32(t_lane + kTmS + 64 * hf, pw);
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.dp_full), tiles & 1, abort_flag));
         if (!ok) break;
-        tmem_st32(t_lane + kTmS + 32 * hf, pw);
+        tc_fence_after();
         // dS^T = P^T o (dP^T - delta) into shared memory: row r of a [key][query row] tile
 #pragma unroll
         for (int c = 0; c < 2; ++c) {
-          uint32_t dv[32];
-          tmem_ld32(t_lane + kTmDP + 64 * hf + 32 * c, dv);
           uint32_t dsw[16];
+          if (!any_vis) {
 #pragma unroll
-          for (int jj = 0; jj < 32; jj += 2) {
-            const uint32_t pk = pw[16 * c + jj / 2];
-            const float p0 = __uint_as_float(pk << 16), p1 = __uint_as_float(pk & 0xFFFF0000u);
-            const int col = 64 * hf + 32 * c + jj;
-            dsw[jj / 2] = pack_bf16x2(p0 * (__uint_as_float(dv[jj]) - col_s[col].y),
-                                      p1 * (__uint_as_float(dv[jj + 1]) - col_s[col + 1].y));
+            for (int m = 0; m < 16; ++m) dsw[m] = 0u;
+          } else {
+            uint32_t dv[32];
+            tmem_ld32(t_lane + kTmDP + 64 * hf + 32 * c, dv);
+#pragma unroll
+            for (int jj = 0; jj < 32; jj += 4) {
+              const int col = 64 * hf + 32 * c + jj;
+              const float4 d4 = *reinterpret_cast<const float4*>(&col_delta[col]);
+              const uint32_t pa = pw[16 * c + jj / 2], pb = pw[16 * c + jj / 2 + 1];
+              dsw[jj / 2] = pack_bf16x2(__uint_as_float(pa << 16) * (__uint_as_float(dv[jj]) - d4.x),
+                                        __uint_as_float(pa & 0xFFFF0000u) * (__uint_as_float(dv[jj + 1]) - d4.y));
+              dsw[jj / 2 + 1] = pack_bf16x2(__uint_as_float(pb << 16) * (__uint_as_float(dv[jj + 2]) - d4.z),
+                                            __uint_as_float(pb & 0xFFFF0000u) * (__uint_as_float(dv[jj + 3]) - d4.w));
+            }
           }
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
@@ -471,32 +530,45 @@ __global__ void __launch_bounds__(kThreads, 1)
         fence_proxy_async_smem();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(bar(bars.p_full));
-        // dQ of this query tile: thread = query row, the pair splits the head dimension
+        if (lane == 0) {
+          mbar_arrive(bar(bars.p_full));
+          mbar_arrive(bar(bars.col_empty));
+        }
+        // dQ_i: thread = query row r of the tile, this warp's half of the head dimension
         ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.dq_full), tiles & 1, abort_flag));
         if (!ok) break;
         tc_fence_after();
-        {
-          const int R = i * kTile + r;
-          const int tok = R / p.G, head = un.g * p.G + (R - tok * p.G);
-          const bool qv = tok < un.len;
-          float* dst = p.dq + ((static_cast<int64_t>(un.cu) + tok) * p.Hq + head) * kD + 64 * hf;
-#pragma unroll 1
-          for (int c = 0; c < 2; ++c) {
-            uint32_t o[32];
-            tmem_ld32(t_lane + kTmS + 64 * hf + 32 * c, o);
-            if (qv)
-#pragma unroll
-              for (int e = 0; e < 32; e += 4)
-                atomicAdd(reinterpret_cast<float4*>(dst + 32 * c + e),
-                          make_float4(__uint_as_float(o[e]) * p.scale, __uint_as_float(o[e + 1]) * p.scale,
-                                      __uint_as_float(o[e + 2]) * p.scale, __uint_as_float(o[e + 3]) * p.scale));
-          }
-        }
+        uint32_t o0[32], o1[32];
+        tmem_ld32(t_lane + kTmDP + 64 * hf, o0);
+        tmem_ld32(t_lane + kTmDP + 64 * hf + 32, o1);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(bar(bars.dq_empty));
-        ++tiles;
+        // The tile's MMAs are done with Q_i and dO_i: their stage takes dQ_i * scale as
+        // two boxes of this warp (32 rows x 32 fp32, 128-byte swizzle) that TMA adds into dQ.
+        // Rows past the sequence are exact zeros (P = 0 there).
+        const uint32_t box = kStage + st * kStageBytes + (quad * 4 + hf * 2) * kBoxBytes;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const uint32_t at = lane * 128 + ((q ^ (lane & 7)) * 16);
+          *reinterpret_cast<float4*>(smem + box + at) =
+              make_float4(__uint_as_float(o0[4 * q]) * p.scale, __uint_as_float(o0[4 * q + 1]) * p.scale,
+                          __uint_as_float(o0[4 * q + 2]) * p.scale, __uint_as_float(o0[4 * q + 3]) * p.scale);
+          *reinterpret_cast<float4*>(smem + box + kBoxBytes + at) =
+              make_float4(__uint_as_float(o1[4 * q]) * p.scale, __uint_as_float(o1[4 * q + 1]) * p.scale,
+                          __uint_as_float(o1[4 * q + 2]) * p.scale, __uint_as_float(o1[4 * q + 3]) * p.scale);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          const int tok = un.cu + ((i * kTile + quad * 32) >> p.lgG);
+          tma_reduce_add_3d(&tm_dq, sbase + box, 64 * hf, un.g * p.G, tok);
+          tma_reduce_add_3d(&tm_dq, sbase + box + kBoxBytes, 64 * hf + 32, un.g * p.G, tok);
+          bulk_commit_group();
+          bulk_wait_group_read0();  // the stage may be refilled once TMA has read the boxes
+          mbar_arrive(bar(bars.q_empty[st]));
+        }
+        __syncwarp();
       }
       if (!ok) break;
       release();
@@ -525,6 +597,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) mbar_arrive(bar(bars.acc_empty));
       ++units;
     }
+    if (lane == 0) bulk_wait_group0();  // every dQ addition of this warp done before the CTA exits
     if (!ok && lane == 0) {
       *abort_flag = 1;
       atomicOr(&g_error_word, MBE_DEVERR_TIMEOUT);
@@ -617,7 +690,7 @@ extern "C" mbe_status mbe_block_mask_attention_bwd(const void* q, const void* k,
     return MBE_ERR_INVALID_ARG;
   if (head_dim != kD) return MBE_ERR_UNSUPPORTED;
   const int G = num_q_heads / num_kv_heads;
-  if (G > kTile || kTile % G != 0) return MBE_ERR_UNSUPPORTED;
+  if (G > 32 || 32 % G != 0) return MBE_ERR_UNSUPPORTED;  // a warp's 32 query rows are whole tokens
   if (static_cast<int64_t>(max_seq_len) * G > static_cast<int64_t>(kMaxQWords) * 32 * kTile) return MBE_ERR_UNSUPPORTED;
   if ((max_seq_len + block_size - 1) / block_size > mask_rows) return MBE_ERR_INVALID_ARG;
   if (batch == 0 || total_tokens == 0) return MBE_OK;
@@ -655,6 +728,13 @@ extern "C" mbe_status mbe_block_mask_attention_bwd(const void* q, const void* k,
     if (!encode_bf16_sw128(&tk, k, 3, dims, strides, box) || !encode_bf16_sw128(&tv, v, 3, dims, strides, box))
       return MBE_ERR_CUDA;
   }
+  CUtensorMap tdq;  // fp32 dQ, added into by 32-row x 32-column boxes
+  {
+    const cuuint64_t dims[3] = {(cuuint64_t)kD, (cuuint64_t)num_q_heads, (cuuint64_t)total_tokens};
+    const cuuint64_t strides[2] = {(cuuint64_t)kD * 4, (cuuint64_t)num_q_heads * kD * 4};
+    const cuuint32_t box[3] = {32, (cuuint32_t)G, (cuuint32_t)(32 / G)};
+    if (!encode_f32_sw128(&tdq, dq, 3, dims, strides, box)) return MBE_ERR_CUDA;
+  }
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   int* counter = reinterpret_cast<int*>(ws);
   int32_t* unit_start = reinterpret_cast<int32_t*>(ws + 16);
@@ -675,7 +755,6 @@ extern "C" mbe_status mbe_block_mask_attention_bwd(const void* q, const void* k,
   p.delta = delta;
   p.unit_start = unit_start;
   p.counter = counter;
-  p.dq = dq;
   p.dk = dk;
   p.dv = dv;
   p.mask_rows = mask_rows;
@@ -687,9 +766,11 @@ extern "C" mbe_status mbe_block_mask_attention_bwd(const void* q, const void* k,
   p.Hq = num_q_heads;
   p.Hkv = num_kv_heads;
   p.G = G;
+  p.lgG = 0;
+  while ((1 << p.lgG) < G) ++p.lgG;
   p.scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(kD));
   p.scale_log2 = p.scale * kLog2e;
-  bwd_kernel<<<ds->num_sms, kThreads, kSmemBytes, stream>>>(tq, tdo, tk, tv, p);
+  bwd_kernel<<<ds->num_sms, kThreads, kSmemBytes, stream>>>(tq, tdo, tk, tv, tdq, p);
   return launch_status("bwd_kernel");
 }
 

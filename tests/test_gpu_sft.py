@@ -180,7 +180,9 @@ def _fwd_bwd(prob, mask):
 
 
 @pytest.mark.parametrize("G,B,K,Np,N,trim", [(4, 32, 3, [1, 0], [6, 3], [0, 7]), (1, 16, 2, [2], [5], [3]),
-                                             (8, 64, 1, [1], [3], [0]), (2, 32, 4, [1, 3], [9, 4], [31, 0])])
+                                             (8, 64, 1, [1], [3], [0]), (2, 32, 4, [1, 3], [9, 4], [31, 0]),
+                                             (4, 8, 2, [1], [9], [5]), (16, 32, 2, [1], [3], [9]),
+                                             (32, 16, 3, [1, 2], [2, 3], [0, 4])])
 def test_backward_matches_oracle(G, B, K, Np, N, trim):
     prob = sft_problem(Np, N, 2 * G, 2, 128, B, seed=100 + G + B + K, trim=trim)
     mask = _gpu_mask(prob, K)
@@ -210,3 +212,14 @@ def test_backward_long_sequence():
     mask = _gpu_mask(prob, 3)
     out, grads = _fwd_bwd(prob, mask)
     _check_bwd(prob, mask.cpu().numpy().view(np.uint32), out, grads)
+
+
+def test_backward_argument_errors():
+    # 64 query heads per KV head: a warp's 32 query rows would not be whole tokens
+    prob = sft_problem([1], [2], 64, 1, 128, 32, seed=5)
+    mask = _gpu_mask(prob, 2)
+    d = {k: getattr(prob, k).to(DEV) for k in ("q", "k", "v", "dout", "seq_len", "cu_seqlens")}
+    lse = torch.zeros(d["q"].shape[:2], dtype=torch.float32, device=DEV)
+    with pytest.raises(mbe.MbeError):
+        mbe.block_mask_attention_bwd(d["q"], d["k"], d["v"], d["q"], d["dout"], lse, d["seq_len"], d["cu_seqlens"],
+                                     mask, block_size=32, max_seq_len=prob.max_seq_len)
