@@ -104,7 +104,11 @@ struct Params {
   const float* lse;
   const float* delta;
   const int32_t* unit_start;  // [batch + 1]: first work unit of each sequence
-  int* counter;
+  int* counter;               // [0] work queue, [1] plan blocks done, [2] work units planned
+  int* unit_nq;               // [max_units]: visible query tiles of each unit
+  int* unit_order;            // [max_units]: units by descending visible query tiles
+  uint32_t* unit_bits;        // [max_units][kMaxQWords]: the visible query tiles
+  int max_units;
   float* dk;
   float* dv;
   int mask_rows, mask_words, block_log2;
@@ -152,6 +156,19 @@ __device__ __forceinline__ int next_bit(const volatile uint32_t* bits, int i) {
   return -1;
 }
 
+// Work unit u: (sequence, KV head, key tile), key tiles fastest.
+__device__ __forceinline__ Unit decode_unit(const Params& p, int u) {
+  int lo = 0, hi = p.batch - 1;  // the sequence whose unit range holds u
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.unit_start[mid] <= u) lo = mid; else hi = mid - 1;
+  }
+  const int len = p.seq_len[lo];
+  const int tiles = max((len + kTile - 1) / kTile, 1);
+  const int r = u - p.unit_start[lo];
+  return Unit{lo, r / tiles, r % tiles, len, p.cu[lo]};
+}
+
 // First and (capped) last query block of query tile i.
 __device__ __forceinline__ int qblock0(const Params& p, int i) { return ((i * kTile) >> p.lgG) >> p.block_log2; }
 __device__ __forceinline__ int qblock_count(const Params& p, const Unit& u, int i) {
@@ -178,7 +195,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t sbase = smem_u32(smem);
   auto bar = [](uint64_t& b) { return smem_u32(&b); };
-  const int n_units = p.unit_start[p.batch];
+  const int n_units = p.counter[2];
 
   if (tid == 0) {
     abort_s = 0;
@@ -233,22 +250,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       Unit un{-1, 0, 0, 0, 0};
       if (!done) {
-        int lo = 0, hi = p.batch - 1;  // the sequence whose unit range holds uidx
-        while (lo < hi) {
-          const int mid = (lo + hi + 1) >> 1;
-          if (p.unit_start[mid] <= uidx) lo = mid; else hi = mid - 1;
-        }
-        const int len = p.seq_len[lo];
-        const int tiles = (len + kTile - 1) / kTile;
-        const int r = uidx - p.unit_start[lo];
-        un = Unit{lo, r / max(tiles, 1), r % max(tiles, 1), len, p.cu[lo]};
-        const int n_qt = ((len << p.lgG) + kTile - 1) / kTile;
-        for (int w = 0; w < kMaxQWords; ++w) {
-          const int i = 32 * w + lane;
-          const uint32_t word = __ballot_sync(kAll, i < n_qt && qtile_visible(p, un, i));
-          if (lane == 0) ring_bits[slot][w] = word;
-        }
+        // units in the planned order: most visible query tiles first
+        const int u = p.unit_order[uidx];
+        un = decode_unit(p, u);
+        if (lane < kMaxQWords) ring_bits[slot][lane] = p.unit_bits[static_cast<int64_t>(u) * kMaxQWords + lane];
       }
+      __syncwarp();
       if (lane == 0) {
         ring[slot] = un;
         mbar_arrive(bar(bars.u_full[slot]));
@@ -610,8 +617,69 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// The backward's work list: one warp per unit finds the query tiles that see
+// its key tile; the last block to finish orders the units by descending count
+// (a counting sort), so the persistent kernel takes the longest units first.
+__global__ void __launch_bounds__(256) bwd_plan_kernel(const Params p) {
+  constexpr int kBins = kMaxQWords * 32 + 1;
+  __shared__ int hist[kBins];
+  __shared__ int last_s;
+  const int lane = threadIdx.x & 31;
+  const int n_all = p.unit_start[p.batch];
+  const int n_units = min(n_all, min(p.max_units, static_cast<int>(gridDim.x) * 8));
+  const int u = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (u < n_units) {
+    const Unit un = decode_unit(p, u);
+    const int n_qt = ((un.len << p.lgG) + kTile - 1) / kTile;
+    int n_q = 0;
+    for (int w = 0; w < kMaxQWords; ++w) {
+      const int i = 32 * w + lane;
+      const uint32_t word = __ballot_sync(0xffffffffu, i < n_qt && qtile_visible(p, un, i));
+      if (lane == 0) p.unit_bits[static_cast<int64_t>(u) * kMaxQWords + w] = word;
+      n_q += __popc(word);
+    }
+    if (lane == 0) p.unit_nq[u] = n_q;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    last_s = atomicAdd(&p.counter[1], 1) == static_cast<int>(gridDim.x) - 1;
+  }
+  __syncthreads();
+  if (!last_s) return;
+  __threadfence();
+  for (int b = threadIdx.x; b < kBins; b += blockDim.x) hist[b] = 0;
+  __syncthreads();
+  for (int v = threadIdx.x; v < n_units; v += blockDim.x) atomicAdd(&hist[__ldcg(&p.unit_nq[v])], 1);
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    // exclusive prefix over the bins taken from the top: lane l owns 17 bins
+    constexpr int kPer = (kBins + 31) / 32;
+    int sum = 0;
+    for (int j = lane * kPer; j < min(kBins, (lane + 1) * kPer); ++j) sum += hist[kBins - 1 - j];
+    int incl = sum;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += y;
+    }
+    int acc = incl - sum;
+    for (int j = lane * kPer; j < min(kBins, (lane + 1) * kPer); ++j) {
+      const int c = hist[kBins - 1 - j];
+      hist[kBins - 1 - j] = acc;
+      acc += c;
+    }
+  }
+  __syncthreads();
+  for (int v = threadIdx.x; v < n_units; v += blockDim.x) p.unit_order[atomicAdd(&hist[__ldcg(&p.unit_nq[v])], 1)] = v;
+  if (threadIdx.x == 0) {
+    p.counter[2] = n_units;
+    if (n_units < n_all) atomicOr(&g_error_word, MBE_DEVERR_LENGTH);
+  }
+}
+
 // delta = rowsum(dO o O) per (token, head) (one warp per row), dQ zeroed, unit
-// offsets and the work counter set up by block 0.
+// offsets and the work counters set up by block 0.
 __global__ void __launch_bounds__(256) bwd_prep_kernel(const __nv_bfloat16* __restrict__ out,
                                                        const __nv_bfloat16* __restrict__ dout, int64_t rows,
                                                        float* __restrict__ delta, float* __restrict__ dq,
@@ -641,8 +709,28 @@ __global__ void __launch_bounds__(256) bwd_prep_kernel(const __nv_bfloat16* __re
       acc += len > 0 ? Hkv * ((len + kTile - 1) / kTile) : 0;
     }
     unit_start[batch] = acc;
-    *counter = 0;
+    counter[0] = 0;
+    counter[1] = 0;
   }
+}
+
+// Workspace: work counters and unit offsets, delta, then the work-unit plan
+// (sized for at most num_q_heads KV heads).
+struct WsLayout {
+  size_t delta, nq, order, bits, total;
+  int64_t max_units;
+};
+
+inline WsLayout ws_layout(int64_t batch, int64_t total_tokens, int64_t num_q_heads) {
+  auto up = [](size_t x) { return (x + 255) & ~size_t(255); };
+  WsLayout L;
+  L.max_units = std::min<int64_t>(num_q_heads * ((total_tokens + kTile - 1) / kTile + batch), 1 << 30);
+  L.delta = up(16 + static_cast<size_t>(batch + 1) * sizeof(int32_t));
+  L.nq = up(L.delta + static_cast<size_t>(total_tokens) * num_q_heads * sizeof(float));
+  L.order = up(L.nq + static_cast<size_t>(L.max_units) * sizeof(int32_t));
+  L.bits = up(L.order + static_cast<size_t>(L.max_units) * sizeof(int32_t));
+  L.total = L.bits + static_cast<size_t>(L.max_units) * kMaxQWords * sizeof(uint32_t);
+  return L;
 }
 
 struct DeviceState {
@@ -670,8 +758,7 @@ DeviceState* device_state(int dev) {
 extern "C" size_t mbe_block_mask_attention_bwd_workspace_size(int32_t batch, int32_t total_tokens,
                                                               int32_t num_q_heads) {
   if (batch < 0 || total_tokens < 0 || num_q_heads < 1) return 0;
-  const size_t head = (static_cast<size_t>(batch) + 1) * sizeof(int32_t) + 16;
-  return ((head + 255) & ~size_t(255)) + static_cast<size_t>(total_tokens) * num_q_heads * sizeof(float);
+  return mbe::bwd::ws_layout(batch, total_tokens, num_q_heads).total;
 }
 
 extern "C" mbe_status mbe_block_mask_attention_bwd(const void* q, const void* k, const void* v, const void* out,
@@ -736,10 +823,10 @@ extern "C" mbe_status mbe_block_mask_attention_bwd(const void* q, const void* k,
     if (!encode_f32_sw128(&tdq, dq, 3, dims, strides, box)) return MBE_ERR_CUDA;
   }
   uint8_t* ws = static_cast<uint8_t*>(workspace);
+  const WsLayout L = ws_layout(batch, total_tokens, num_q_heads);
   int* counter = reinterpret_cast<int*>(ws);
   int32_t* unit_start = reinterpret_cast<int32_t*>(ws + 16);
-  const size_t head = (static_cast<size_t>(batch) + 1) * sizeof(int32_t) + 16;
-  float* delta = reinterpret_cast<float*>(ws + ((head + 255) & ~size_t(255)));
+  float* delta = reinterpret_cast<float*>(ws + L.delta);
   const int64_t rows = static_cast<int64_t>(total_tokens) * num_q_heads;
   const int64_t prep_blocks = std::min<int64_t>((rows + 7) / 8, 8ll * ds->num_sms);
   bwd_prep_kernel<<<static_cast<unsigned>(std::max<int64_t>(prep_blocks, 1)), 256, 0, stream>>>(
@@ -755,6 +842,10 @@ extern "C" mbe_status mbe_block_mask_attention_bwd(const void* q, const void* k,
   p.delta = delta;
   p.unit_start = unit_start;
   p.counter = counter;
+  p.unit_nq = reinterpret_cast<int*>(ws + L.nq);
+  p.unit_order = reinterpret_cast<int*>(ws + L.order);
+  p.unit_bits = reinterpret_cast<uint32_t*>(ws + L.bits);
+  p.max_units = static_cast<int>(L.max_units);
   p.dk = dk;
   p.dv = dv;
   p.mask_rows = mask_rows;
@@ -770,6 +861,11 @@ extern "C" mbe_status mbe_block_mask_attention_bwd(const void* q, const void* k,
   while ((1 << p.lgG) < G) ++p.lgG;
   p.scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(kD));
   p.scale_log2 = p.scale * kLog2e;
+  const int64_t launch_units =
+      std::min<int64_t>(L.max_units, static_cast<int64_t>(num_kv_heads) * batch * ((max_seq_len + kTile - 1) / kTile));
+  bwd_plan_kernel<<<static_cast<unsigned>(std::max<int64_t>((launch_units + 7) / 8, 1)), 256, 0, stream>>>(p);
+  st = launch_status("bwd_plan_kernel");
+  if (st != MBE_OK) return st;
   bwd_kernel<<<ds->num_sms, kThreads, kSmemBytes, stream>>>(tq, tdo, tk, tv, tdq, p);
   return launch_status("bwd_kernel");
 }
