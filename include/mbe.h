@@ -384,9 +384,8 @@ mbe_status mbe_block_mask_attention(const void* q, const void* k, const void* v,
  * rounded to bf16 before their products (tensor cores), as in the forward's P.
  * workspace: mbe_block_mask_attention_bwd_workspace_size(batch, total_tokens,
  * num_q_heads) bytes, 16-byte aligned. head_dim must be 128; num_q_heads /
- * num_kv_heads must divide 32; max_seq_len * that ratio <= 65536. dq is
- * zeroed by this call and then accumulated in place (TMA additions), so it
- * must not overlap another argument.
+ * num_kv_heads must divide 32; max_seq_len * that ratio <= 65536. Rows past
+ * cu_seqlens[batch] are not written.
  * Errors: MBE_ERR_INVALID_ARG, MBE_ERR_UNSUPPORTED, MBE_ERR_WORKSPACE,
  * MBE_ERR_CUDA; a bounded wait that expires sets MBE_DEVERR_TIMEOUT.
  */
