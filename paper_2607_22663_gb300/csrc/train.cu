@@ -94,10 +94,11 @@ constexpr int kMaxWords = 16;                // tile bitmask of a unit (<= 512 t
 constexpr int kMaxKeyBlocks = 16;            // key blocks of a 128-key tile (block size >= 8)
 constexpr uint32_t kHalf = 128 * 128;        // a 64-column half of a 128-row bf16 tile (16 KB)
 constexpr uint32_t kTileBytes = 2 * kHalf;   // 32 KB
-constexpr uint32_t kStageBytes = 2 * kTileBytes;  // two tiles: Q_i and dO_i, or K_j and V_j
-// shared memory of both kernels: two fixed tiles and a 2-stage ring of tile pairs
-constexpr uint32_t kFix0 = 0, kFix1 = kTileBytes, kRing = 2 * kTileBytes;
-constexpr uint32_t kSmemBytes = kRing + 2 * kStageBytes + 1024;  // + 1024-byte alignment slack
+// shared memory of both kernels: two tiles held for the whole unit, a 3-stage
+// ring of the streamed tile the step's first MMA reads (Q, or K) and a 2-stage
+// ring of the other streamed tile (dO, or V)
+constexpr uint32_t kFix0 = 0, kFix1 = kTileBytes, kRingA = 2 * kTileBytes, kRingB = kRingA + 3 * kTileBytes;
+constexpr uint32_t kSmemBytes = kRingB + 2 * kTileBytes + 1024;  // + 1024-byte alignment slack
 constexpr float kLog2e = 1.4426950408889634f;
 
 // Work units of one kind: (sequence, KV head g, tile t), t fastest.
@@ -216,8 +217,8 @@ __device__ __forceinline__ int popc_bits(const volatile uint32_t* bits) {
 constexpr uint32_t kTmDK = 0, kTmDV = 128, kTmS = 256, kTmDP = 384, kTmCols = 512;
 
 struct KvBars {
-  uint64_t u_full[2], u_empty[2], q_full[2], q_empty[2], kv_full, kv_empty, col_full, col_empty, s_full, s_free,
-      dp_full, p_full, acc_full, acc_empty, mma_done;
+  uint64_t u_full[2], u_empty[2], q_full[3], q_empty[3], do_full[2], do_empty[2], kv_full, kv_empty, col_full,
+      col_empty, s_full, pt_full, dp_full, ds_full, acc_full, acc_empty, mma_done;
 };
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -246,6 +247,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0; i < 2; ++i) {
       mbar_init(bar(bars.u_full[i]), 1);
       mbar_init(bar(bars.u_empty[i]), 9);  // MMA issuer + 8 compute warps
+      mbar_init(bar(bars.do_full[i]), 1);
+      mbar_init(bar(bars.do_empty[i]), 1);
+    }
+    for (int i = 0; i < 3; ++i) {
       mbar_init(bar(bars.q_full[i]), 1);
       mbar_init(bar(bars.q_empty[i]), 1);
     }
@@ -254,9 +259,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(bar(bars.col_full), 1);
     mbar_init(bar(bars.col_empty), 8);
     mbar_init(bar(bars.s_full), 1);
-    mbar_init(bar(bars.s_free), 8);
+    mbar_init(bar(bars.pt_full), 8);
     mbar_init(bar(bars.dp_full), 1);
-    mbar_init(bar(bars.p_full), 8);
+    mbar_init(bar(bars.ds_full), 8);
     mbar_init(bar(bars.acc_full), 1);
     mbar_init(bar(bars.acc_empty), 8);
     mbar_init(bar(bars.mma_done), 1);
@@ -279,7 +284,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tm_k);
       tma_prefetch_desc(&tm_v);
     }
-    uint32_t u_it = 0, kv_loads = 0, q_loads = 0, cols = 0;
+    uint32_t u_it = 0, kv_loads = 0, q_loads = 0, do_loads = 0, cols = 0;
     bool ok = true;
     for (;;) {
       const int slot = u_it & 1;
@@ -309,21 +314,30 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int kb_first = (un.t * kTile) >> p.block_log2;
       const int kb_last = (min(un.len, (un.t + 1) * kTile) - 1) >> p.block_log2;
       for (int i = next_bit(bits, -1); i >= 0 && ok; i = next_bit(bits, i)) {
-        const uint32_t st = q_loads & 1;
-        if (q_loads >= 2) {
-          ok = __all_sync(kAll, mbar_wait(bar(bars.q_empty[st]), ((q_loads >> 1) - 1) & 1, abort_flag));
+        const int tok = un.cu + ((i * kTile) >> p.lgG);
+        const uint32_t sq = q_loads % 3, sd = do_loads & 1;
+        if (q_loads >= 3) {
+          ok = __all_sync(kAll, mbar_wait(bar(bars.q_empty[sq]), ((q_loads / 3) - 1) & 1, abort_flag));
           if (!ok) break;
         }
         if (lane == 0) {
-          const uint32_t qa = sbase + kRing + st * kStageBytes;
-          mbar_arrive_expect_tx(bar(bars.q_full[st]), kStageBytes);
-          const int tok = un.cu + ((i * kTile) >> p.lgG);
-          for (int h = 0; h < 2; ++h) {
-            tma_load_3d(qa + h * kHalf, &tm_q, bar(bars.q_full[st]), h * 64, un.g * p.G, tok);
-            tma_load_3d(qa + kTileBytes + h * kHalf, &tm_do, bar(bars.q_full[st]), h * 64, un.g * p.G, tok);
-          }
+          mbar_arrive_expect_tx(bar(bars.q_full[sq]), kTileBytes);
+          for (int h = 0; h < 2; ++h)
+            tma_load_3d(sbase + kRingA + sq * kTileBytes + h * kHalf, &tm_q, bar(bars.q_full[sq]), h * 64,
+                        un.g * p.G, tok);
         }
         ++q_loads;
+        if (do_loads >= 2) {
+          ok = __all_sync(kAll, mbar_wait(bar(bars.do_empty[sd]), ((do_loads >> 1) - 1) & 1, abort_flag));
+          if (!ok) break;
+        }
+        if (lane == 0) {
+          mbar_arrive_expect_tx(bar(bars.do_full[sd]), kTileBytes);
+          for (int h = 0; h < 2; ++h)
+            tma_load_3d(sbase + kRingB + sd * kTileBytes + h * kHalf, &tm_do, bar(bars.do_full[sd]), h * 64,
+                        un.g * p.G, tok);
+        }
+        ++do_loads;
         // column data of tile i, fetched before waiting for the compute warps to
         // finish with the previous tile's
         float lse_r[4], dl_r[4];
@@ -363,8 +377,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       // let the copies already issued land before the CTA can exit
       const int zero = 0;
       if (kv_loads >= 1) mbar_wait(bar(bars.kv_full), (kv_loads - 1) & 1, &zero);
-      for (uint32_t n = (q_loads >= 2 ? q_loads - 2 : 0); n < q_loads; ++n)
-        mbar_wait(bar(bars.q_full[n & 1]), (n >> 1) & 1, &zero);
+      for (uint32_t n = (q_loads >= 3 ? q_loads - 3 : 0); n < q_loads; ++n)
+        mbar_wait(bar(bars.q_full[n % 3]), (n / 3) & 1, &zero);
+      for (uint32_t n = (do_loads >= 2 ? do_loads - 2 : 0); n < do_loads; ++n)
+        mbar_wait(bar(bars.do_full[n & 1]), (n >> 1) & 1, &zero);
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
@@ -373,12 +389,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t idesc_tb = idesc_bf16_f32(kTile, kD, false, true);      // dV, dK: MN-major B
       uint32_t u_it = 0, units = 0, tiles = 0;
       bool ok = true;
-      // S^T = K Q_t^T into the S region once the compute warps have read S^T of tile t - 1
+      // S^T = K Q_t^T into the S region (issued after dV of tile t - 1, the last reader there)
       auto issue_s = [&](uint32_t t) {
-        if (!mbar_wait(bar(bars.q_full[t & 1]), (t >> 1) & 1, abort_flag)) return false;
-        if (t >= 1 && !mbar_wait(bar(bars.s_free), (t - 1) & 1, abort_flag)) return false;
+        if (!mbar_wait(bar(bars.q_full[t % 3]), (t / 3) & 1, abort_flag)) return false;
         tc_fence_after();
-        const uint32_t qa = sbase + kRing + (t & 1) * kStageBytes;
+        const uint32_t qa = sbase + kRingA + (t % 3) * kTileBytes;
 #pragma unroll
         for (int h = 0; h < 2; ++h)
 #pragma unroll
@@ -390,9 +405,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         umma_commit(bar(bars.s_full));
         return true;
       };
-      // dP^T = V dO_t^T into the dP region (after the MMAs that read P^T of tile t - 1 there)
+      // dP^T = V dO_t^T into the dP region (issued after dK of tile t - 1, the last reader there)
       auto issue_dp = [&](uint32_t t) {
-        const uint32_t da = sbase + kRing + (t & 1) * kStageBytes + kTileBytes;
+        if (!mbar_wait(bar(bars.do_full[t & 1]), (t >> 1) & 1, abort_flag)) return false;
+        tc_fence_after();
+        const uint32_t da = sbase + kRingB + (t & 1) * kTileBytes;
 #pragma unroll
         for (int h = 0; h < 2; ++h)
 #pragma unroll
@@ -402,6 +419,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     (h | k) ? 1u : 0u);
           }
         umma_commit(bar(bars.dp_full));
+        return true;
       };
       for (;;) {
         const int slot = u_it & 1;
@@ -413,31 +431,34 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (un.seq < 0) break;
         if (n_q == 0) continue;
         if (!mbar_wait(bar(bars.kv_full), units & 1, abort_flag)) { ok = false; break; }
-        if (!issue_s(tiles)) { ok = false; break; }
-        issue_dp(tiles);
+        if (!issue_s(tiles) || !issue_dp(tiles)) { ok = false; break; }
         for (int j = 0; j < n_q; ++j) {
           const uint32_t t = tiles + j;
-          // the next tile's S^T runs while the compute warps work on this tile
-          if (j + 1 < n_q && !issue_s(t + 1)) { ok = false; break; }
-          if (!mbar_wait(bar(bars.p_full), t & 1, abort_flag)) { ok = false; break; }
+          const uint32_t qa = sbase + kRingA + (t % 3) * kTileBytes, da = sbase + kRingB + (t & 1) * kTileBytes;
+          // dV as soon as P^T is in TMEM (over S^T), then the next tile's S^T; both run
+          // while the compute warps form dS^T
+          if (!mbar_wait(bar(bars.pt_full), t & 1, abort_flag)) { ok = false; break; }
           if (j == 0 && units >= 1 && !mbar_wait(bar(bars.acc_empty), (units - 1) & 1, abort_flag)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t qa = sbase + kRing + (t & 1) * kStageBytes, da = qa + kTileBytes;
 #pragma unroll
-          for (int kk = 0; kk < kTile / 16; ++kk) {
-            const uint32_t acc = (j > 0 || kk > 0) ? 1u : 0u;
-            // P^T of query columns 64 h .. 64 h + 63 sits packed at dP region columns 64 h .. 64 h + 31
-            umma_ts(tmem + kTmDV, tmem + kTmDP + (kk >> 2) * 64 + (kk & 3) * 8,
-                    sdesc_sw128(da + kk * 16 * 128, kHalf, 1024), idesc_tb, acc);
-            // dS^T of the same columns at dP region columns 64 h + 32 .. 64 h + 63 (A of dK)
-            umma_ts(tmem + kTmDK, tmem + kTmDP + 32 + (kk >> 2) * 64 + (kk & 3) * 8,
-                    sdesc_sw128(qa + kk * 16 * 128, kHalf, 1024), idesc_tb, acc);
-          }
-          umma_commit(bar(bars.q_empty[t & 1]));
-          if (j + 1 < n_q) issue_dp(t + 1);
+          for (int kk = 0; kk < kTile / 16; ++kk)
+            // P^T of query columns 64 h .. 64 h + 63 sits packed at S region columns 64 h .. 64 h + 31
+            umma_ts(tmem + kTmDV, tmem + kTmS + (kk >> 2) * 64 + (kk & 3) * 8,
+                    sdesc_sw128(da + kk * 16 * 128, kHalf, 1024), idesc_tb, (j > 0 || kk > 0) ? 1u : 0u);
+          umma_commit(bar(bars.do_empty[t & 1]));
+          if (j + 1 < n_q && !issue_s(t + 1)) { ok = false; break; }
+          // dK once dS^T is in TMEM (over dP^T), then the next tile's dP^T
+          if (!mbar_wait(bar(bars.ds_full), t & 1, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+#pragma unroll
+          for (int kk = 0; kk < kTile / 16; ++kk)
+            umma_ts(tmem + kTmDK, tmem + kTmDP + (kk >> 2) * 64 + (kk & 3) * 8,
+                    sdesc_sw128(qa + kk * 16 * 128, kHalf, 1024), idesc_tb, (j > 0 || kk > 0) ? 1u : 0u);
+          umma_commit(bar(bars.q_empty[t % 3]));
+          if (j + 1 < n_q && !issue_dp(t + 1)) { ok = false; break; }
         }
         if (!ok) break;
         tiles += n_q;
@@ -503,14 +524,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!ok) break;
         tc_fence_after();
         uint32_t sv[64];
-        if (any_vis) {
-          tmem_ld32(t_lane + kTmS + 64 * hf, *reinterpret_cast<uint32_t(*)[32]>(sv));
-          tmem_ld32(t_lane + kTmS + 64 * hf + 32, *reinterpret_cast<uint32_t(*)[32]>(sv + 32));
-        }
-        // S^T read: the next tile's S^T may overwrite it
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar(bars.s_free));
+        if (any_vis) tmem_ld64(t_lane + kTmS + 64 * hf, sv);
         // P^T of this warp's 64 columns, packed to bf16 pairs; a query block spans at
         // least 8 packed rows, so visibility is decided per group of 8 columns
         uint32_t pw[32];
@@ -537,12 +551,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             pw[4 * g8 + 3] = pack_bf16x2(ex2f(x3.x), ex2f(x3.y)) & keep;
           }
         }
-        // dP^T of this tile (the MMAs of the previous tile have read P^T and dS^T)
+        // P^T over the S^T columns this warp has read (A of dV)
+        tmem_st32(t_lane + kTmS + 64 * hf, pw);
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(bars.pt_full));
+        // dP^T of this tile
         ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.dp_full), tiles & 1, abort_flag));
         if (!ok) break;
         tc_fence_after();
         // dS^T = P^T o (dP^T - delta), packed to bf16 pairs
         uint32_t dsa[32];
+        uint32_t dvv[64];
+        if (any_vis) tmem_ld64(t_lane + kTmDP + 64 * hf, dvv);
 #pragma unroll
         for (int c = 0; c < 2; ++c) {
           uint32_t* dsw = dsa + 16 * c;
@@ -550,8 +572,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int m = 0; m < 16; ++m) dsw[m] = 0u;
           } else {
-            uint32_t dv[32];
-            tmem_ld32(t_lane + kTmDP + 64 * hf + 32 * c, dv);
+            const uint32_t* dv = dvv + 32 * c;
 #pragma unroll
             for (int jj = 0; jj < 32; jj += 4) {
               const int col = 64 * hf + 32 * c + jj;
@@ -568,15 +589,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
         }
-        // over the dP^T columns this warp has read: P^T at 64 hf .. 64 hf + 31 (A of
-        // dV), dS^T at 64 hf + 32 .. 64 hf + 63 (A of dK)
-        tmem_st32(t_lane + kTmDP + 64 * hf, pw);
-        tmem_st32(t_lane + kTmDP + 64 * hf + 32, dsa);
+        // dS^T over the dP^T columns this warp has read (A of dK)
+        tmem_st32(t_lane + kTmDP + 64 * hf, dsa);
         tmem_st_wait();
         tc_fence_before();
         __syncwarp();
         if (lane == 0) {
-          mbar_arrive(bar(bars.p_full));
+          mbar_arrive(bar(bars.ds_full));
           mbar_arrive(bar(bars.col_empty));
         }
       }
@@ -626,8 +645,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 constexpr uint32_t kTmQS = 0, kTmQDP = 256, kTmQDQ = 384;
 
 struct QBars {
-  uint64_t u_full[2], u_empty[2], qd_full, qd_empty, kv_full[2], kv_empty[2], s_full[2], dp_full, dp_free, ds_full,
-      acc_full, acc_empty, mma_done;
+  uint64_t u_full[2], u_empty[2], qd_full, qd_empty, k_full[3], k_empty[3], v_full[2], v_empty[2], s_full[2],
+      dp_full, dp_free, ds_full, acc_full, acc_empty, mma_done;
 };
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -652,9 +671,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0; i < 2; ++i) {
       mbar_init(bar(bars.u_full[i]), 1);
       mbar_init(bar(bars.u_empty[i]), 9);  // MMA issuer + 8 compute warps
-      mbar_init(bar(bars.kv_full[i]), 1);
-      mbar_init(bar(bars.kv_empty[i]), 1);
+      mbar_init(bar(bars.v_full[i]), 1);
+      mbar_init(bar(bars.v_empty[i]), 1);
       mbar_init(bar(bars.s_full[i]), 1);
+    }
+    for (int i = 0; i < 3; ++i) {
+      mbar_init(bar(bars.k_full[i]), 1);
+      mbar_init(bar(bars.k_empty[i]), 1);
     }
     mbar_init(bar(bars.qd_full), 1);
     mbar_init(bar(bars.qd_empty), 1);
@@ -683,7 +706,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tm_k);
       tma_prefetch_desc(&tm_v);
     }
-    uint32_t u_it = 0, qd_loads = 0, kv_loads = 0;
+    uint32_t u_it = 0, qd_loads = 0, k_loads = 0, v_loads = 0;
     bool ok = true;
     for (;;) {
       const int slot = u_it & 1;
@@ -712,20 +735,29 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       ++qd_loads;
       for (int j = next_bit(bits, -1); j >= 0 && ok; j = next_bit(bits, j)) {
-        const uint32_t st = kv_loads & 1;
-        if (kv_loads >= 2) {
-          ok = __all_sync(kAll, mbar_wait(bar(bars.kv_empty[st]), ((kv_loads >> 1) - 1) & 1, abort_flag));
+        const uint32_t sk = k_loads % 3, sv = v_loads & 1;
+        if (k_loads >= 3) {
+          ok = __all_sync(kAll, mbar_wait(bar(bars.k_empty[sk]), ((k_loads / 3) - 1) & 1, abort_flag));
           if (!ok) break;
         }
         if (lane == 0) {
-          const uint32_t ka = sbase + kRing + st * kStageBytes;
-          mbar_arrive_expect_tx(bar(bars.kv_full[st]), kStageBytes);
-          for (int h = 0; h < 2; ++h) {
-            tma_load_3d(ka + h * kHalf, &tm_k, bar(bars.kv_full[st]), h * 64, un.g, un.cu + j * kTile);
-            tma_load_3d(ka + kTileBytes + h * kHalf, &tm_v, bar(bars.kv_full[st]), h * 64, un.g, un.cu + j * kTile);
-          }
+          mbar_arrive_expect_tx(bar(bars.k_full[sk]), kTileBytes);
+          for (int h = 0; h < 2; ++h)
+            tma_load_3d(sbase + kRingA + sk * kTileBytes + h * kHalf, &tm_k, bar(bars.k_full[sk]), h * 64, un.g,
+                        un.cu + j * kTile);
         }
-        ++kv_loads;
+        ++k_loads;
+        if (v_loads >= 2) {
+          ok = __all_sync(kAll, mbar_wait(bar(bars.v_empty[sv]), ((v_loads >> 1) - 1) & 1, abort_flag));
+          if (!ok) break;
+        }
+        if (lane == 0) {
+          mbar_arrive_expect_tx(bar(bars.v_full[sv]), kTileBytes);
+          for (int h = 0; h < 2; ++h)
+            tma_load_3d(sbase + kRingB + sv * kTileBytes + h * kHalf, &tm_v, bar(bars.v_full[sv]), h * 64, un.g,
+                        un.cu + j * kTile);
+        }
+        ++v_loads;
       }
       if (!ok) break;
     }
@@ -734,8 +766,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       atomicOr(&g_error_word, MBE_DEVERR_TIMEOUT);
       const int zero = 0;
       if (qd_loads >= 1) mbar_wait(bar(bars.qd_full), (qd_loads - 1) & 1, &zero);
-      for (uint32_t n = (kv_loads >= 2 ? kv_loads - 2 : 0); n < kv_loads; ++n)
-        mbar_wait(bar(bars.kv_full[n & 1]), (n >> 1) & 1, &zero);
+      for (uint32_t n = (k_loads >= 3 ? k_loads - 3 : 0); n < k_loads; ++n)
+        mbar_wait(bar(bars.k_full[n % 3]), (n / 3) & 1, &zero);
+      for (uint32_t n = (v_loads >= 2 ? v_loads - 2 : 0); n < v_loads; ++n)
+        mbar_wait(bar(bars.v_full[n & 1]), (n >> 1) & 1, &zero);
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
@@ -747,9 +781,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       // S = Q K_t^T into S buffer t & 1 (issued after dQ of tile t - 2, which read dS there)
       auto issue_s = [&](uint32_t t) {
         const uint32_t b = t & 1;
-        if (!mbar_wait(bar(bars.kv_full[b]), (t >> 1) & 1, abort_flag)) return false;
+        if (!mbar_wait(bar(bars.k_full[t % 3]), (t / 3) & 1, abort_flag)) return false;
         tc_fence_after();
-        const uint32_t ka = sbase + kRing + b * kStageBytes;
+        const uint32_t ka = sbase + kRingA + (t % 3) * kTileBytes;
 #pragma unroll
         for (int h = 0; h < 2; ++h)
 #pragma unroll
@@ -764,8 +798,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       // dP = dO V_t^T once the compute warps have read dP of tile t - 1
       auto issue_dp = [&](uint32_t t) {
         if (t >= 1 && !mbar_wait(bar(bars.dp_free), (t - 1) & 1, abort_flag)) return false;
+        if (!mbar_wait(bar(bars.v_full[t & 1]), (t >> 1) & 1, abort_flag)) return false;
         tc_fence_after();
-        const uint32_t va = sbase + kRing + (t & 1) * kStageBytes + kTileBytes;
+        const uint32_t va = sbase + kRingB + (t & 1) * kTileBytes;
 #pragma unroll
         for (int h = 0; h < 2; ++h)
 #pragma unroll
@@ -775,6 +810,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     idesc_kk, (h | k) ? 1u : 0u);
           }
         umma_commit(bar(bars.dp_full));
+        umma_commit(bar(bars.v_empty[t & 1]));
         return true;
       };
       for (;;) {
@@ -787,25 +823,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (un.seq < 0) break;
         if (n_k == 0) continue;
         if (!mbar_wait(bar(bars.qd_full), units & 1, abort_flag)) { ok = false; break; }
-        if (!issue_s(tiles) || !issue_dp(tiles)) { ok = false; break; }
+        // S two tiles ahead: it runs while the compute warps form dS of the tile before
+        if (!issue_s(tiles) || !issue_dp(tiles) || (n_k >= 2 && !issue_s(tiles + 1))) { ok = false; break; }
         for (int j = 0; j < n_k; ++j) {
           const uint32_t t = tiles + j;
-          if (j + 1 < n_k && !issue_s(t + 1)) { ok = false; break; }
           if (!mbar_wait(bar(bars.ds_full), t & 1, abort_flag)) { ok = false; break; }
+          // the next tile's dP first: the compute warps wait for it, and its region was
+          // read before ds_full
+          if (j + 1 < n_k && !issue_dp(t + 1)) { ok = false; break; }
           if (j == 0 && units >= 1 && !mbar_wait(bar(bars.acc_empty), (units - 1) & 1, abort_flag)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t ka = sbase + kRing + (t & 1) * kStageBytes;
+          const uint32_t ka = sbase + kRingA + (t % 3) * kTileBytes;
           // dQ += dS K_t: dS of key columns 64 h .. 64 h + 63 sits packed at S buffer columns
           // 64 h .. 64 h + 31 (A from TMEM); K_t [key][d] is an MN-major B
 #pragma unroll
           for (int kk = 0; kk < kTile / 16; ++kk)
             umma_ts(tmem + kTmQDQ, tmem + kTmQS + 128 * (t & 1) + (kk >> 2) * 64 + (kk & 3) * 8,
                     sdesc_sw128(ka + kk * 16 * 128, kHalf, 1024), idesc_dq, (j > 0 || kk > 0) ? 1u : 0u);
-          umma_commit(bar(bars.kv_empty[t & 1]));
-          if (j + 1 < n_k && !issue_dp(t + 1)) { ok = false; break; }
+          umma_commit(bar(bars.k_empty[t % 3]));
+          if (j + 2 < n_k && !issue_s(t + 2)) { ok = false; break; }
         }
         if (!ok) break;
         tiles += n_k;
@@ -877,10 +916,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!ok) break;
         tc_fence_after();
         uint32_t sv[64];
-        if (any_vis) {
-          tmem_ld32(t_lane + kTmQS + 128 * b + 64 * hf, *reinterpret_cast<uint32_t(*)[32]>(sv));
-          tmem_ld32(t_lane + kTmQS + 128 * b + 64 * hf + 32, *reinterpret_cast<uint32_t(*)[32]>(sv + 32));
-        }
+        if (any_vis) tmem_ld64(t_lane + kTmQS + 128 * b + 64 * hf, sv);
         // P of this warp's 64 key columns, packed to bf16 pairs; a key block spans at
         // least 8 columns, so visibility is decided per group of 8
         uint32_t pw[32];
@@ -922,8 +958,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int m = 0; m < 32; ++m) dsa[m] = 0u;
         } else {
           uint32_t dv[64];
-          tmem_ld32(t_lane + kTmQDP + 64 * hf, *reinterpret_cast<uint32_t(*)[32]>(dv));
-          tmem_ld32(t_lane + kTmQDP + 64 * hf + 32, *reinterpret_cast<uint32_t(*)[32]>(dv + 32));
+          tmem_ld64(t_lane + kTmQDP + 64 * hf, dv);
           const float2 nd2 = make_float2(-dl, -dl);
 #pragma unroll
           for (int jj = 0; jj < 64; jj += 2) {
