@@ -152,6 +152,8 @@ def _check_bwd(prob, mask_bits, out_gpu, grads):
     nb = mask_bits.shape[1]
     for s in range(len(prob.seq_host)):
         a, b = cu[s], cu[s + 1]
+        if a == b:
+            continue
         q, k, v, do = prob.q[a:b], prob.k[a:b], prob.v[a:b], prob.dout[a:b]
         ref = oracle.block_mask_attention_bwd(bf16_bits(q), bf16_bits(k), bf16_bits(v), bf16_bits(do),
                                               prob.block_size, mask_bits[s])
@@ -223,3 +225,11 @@ def test_backward_argument_errors():
     with pytest.raises(mbe.MbeError):
         mbe.block_mask_attention_bwd(d["q"], d["k"], d["v"], d["q"], d["dout"], lse, d["seq_len"], d["cu_seqlens"],
                                      mask, block_size=32, max_seq_len=prob.max_seq_len)
+
+
+def test_backward_with_an_empty_sequence_in_the_batch():
+    # the middle sequence has no tokens: no work units, nothing written for it
+    prob = sft_problem([1, 0, 2], [3, 0, 4], 8, 2, 128, 32, seed=21, trim=[5, 0, 0])
+    mask = _gpu_mask(prob, 2)
+    out, grads = _fwd_bwd(prob, mask)
+    _check_bwd(prob, mask.cpu().numpy().view(np.uint32), out, grads)
