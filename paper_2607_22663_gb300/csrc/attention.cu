@@ -1010,20 +1010,18 @@ __device__ __forceinline__ void merge_row_warp(const MergeParams& p, const Merge
   const float* lse = p.part_lse + static_cast<int64_t>(grp.slot_base) * kUnitRows + r;  // split k at k * kUnitRows
   const float* part = p.part_o + (static_cast<int64_t>(grp.slot_base) * kUnitRows + r) * D + lane * kPer;
   const int n = grp.n_splits;
-  // the row's largest log-sum-exp: lanes read the splits' values in parallel
-  float M = neg_inf();
-  for (int k = lane; k < n; k += 32) M = fmaxf(M, lse[static_cast<int64_t>(k) * kUnitRows]);
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-  float wsum = 0.f;
+  // Online merge: eight splits per step, all their loads issued before any is
+  // used; the running maximum M of the splits' log-sum-exps rescales what has
+  // been summed so far when it grows (one pass over the partials).
+  constexpr int kBatch = 8;
+  float M = neg_inf(), wsum = 0.f;
   float acc[kPer];
 #pragma unroll
   for (int d = 0; d < kPer; ++d) acc[d] = 0.f;
-  // four splits per step, their loads issued before any is used
-  for (int k0 = 0; k0 < n; k0 += 4) {
-    float lk[4], v[4][kPer];
+  for (int k0 = 0; k0 < n; k0 += kBatch) {
+    float lk[kBatch], v[kBatch][kPer];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < kBatch; ++u) {
       const int k = k0 + u;
       lk[u] = neg_inf();
 #pragma unroll
@@ -1040,8 +1038,18 @@ __device__ __forceinline__ void merge_row_warp(const MergeParams& p, const Merge
         }
       }
     }
+    float mb = lk[0];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 1; u < kBatch; ++u) mb = fmaxf(mb, lk[u]);
+    if (mb > M) {
+      const float c = (M == neg_inf()) ? 0.f : ex2f(M - mb);
+      wsum *= c;
+#pragma unroll
+      for (int d = 0; d < kPer; ++d) acc[d] *= c;
+      M = mb;
+    }
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
       const float w = (lk[u] == neg_inf()) ? 0.f : ex2f(lk[u] - M);
       wsum += w;
 #pragma unroll
