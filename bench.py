@@ -75,7 +75,7 @@ def edit_bytes(rows, vocab, elem):
 # a changed kernel gets no traffic figure until it is measured again. Source:
 # profiles/attn_dram_serving128.md.
 MEASURED_TRAFFIC = {
-    "ecdb41c61a34af40": {"serving128": 4442425600 + 60212992 + 11264},
+    "a79788f3811471c0": {"serving128": 4442590720 + 59869440 + 8704},
 }
 
 
