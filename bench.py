@@ -462,7 +462,7 @@ def refresh_pass(attn, changed, rb, stream=None):
     p = rb.plan
     for i, a in enumerate(attn):
         for src, dst in ((a.q, rb.q), (a.k_win, rb.k), (a.v_win, rb.v)):
-            mbe.gather_rows(src, p["src_row"], out=dst, stream=stream)
+            mbe.gather_rows(src, p["src_row"], out=dst, rows_used=p["count"][1:], stream=stream)
         mbe.kv_window_write(rb.k, rb.v, a.k_cache, a.v_cache, p["block_table"], p["prefix_len"], p["window_len"],
                             p["cu_window"], block_size=B, max_window=B, stream=stream)
         fn = mbe.window_attention if i == 0 else mbe.window_attention_run

@@ -478,12 +478,15 @@ mbe_status mbe_refresh_plan(const uint8_t* block_changed, int32_t max_blocks_per
  * (k < rows): the compaction of per-row inputs (token ids, hidden states,
  * Q/K/V) for the refresh batch of mbe_refresh_plan. A negative src_row[k]
  * gives a zero row; src_row[k] >= src_rows gives a zero row and sets
- * MBE_DEVERR_LENGTH. src and dst are device buffers that must not overlap;
- * 16-byte rows and alignment give vectorised copies.
+ * MBE_DEVERR_LENGTH. rows_used_or_null (device int32, e.g. &r_count[1] of
+ * mbe_refresh_plan) limits the copy to rows k < min(rows, *rows_used): the rows
+ * after it are left as they are, so a refresh batch only costs its changed rows.
+ * src and dst are device buffers that must not overlap; 16-byte rows and
+ * alignment give vectorised copies.
  * Errors: MBE_ERR_INVALID_ARG, MBE_ERR_CUDA.
  */
 mbe_status mbe_gather_rows(const void* src, int64_t src_rows, int64_t row_bytes, const int32_t* src_row,
-                           int64_t rows, void* dst, cudaStream_t stream);
+                           int64_t rows, const int32_t* rows_used_or_null, void* dst, cudaStream_t stream);
 
 /*
  * Editing-pass loop on the device. Paper: Sec. 4.1 (the window is edited by

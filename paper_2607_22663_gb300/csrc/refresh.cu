@@ -116,11 +116,14 @@ __global__ void __launch_bounds__(kScanThreads) refresh_plan_kernel(
 }
 
 // dst row k = src row map[k]; zeros where map[k] < 0; zeros and a device flag
-// where map[k] >= src_rows. V is the copy width (16, 4 or 1 bytes).
+// where map[k] >= src_rows; rows from *rows_used on (if given) untouched. V is
+// the copy width (16, 4 or 1 bytes).
 template <typename V>
 __global__ void __launch_bounds__(256) gather_rows_kernel(const V* __restrict__ src, int64_t src_rows,
                                                           int64_t row_elems, const int32_t* __restrict__ map,
-                                                          int64_t rows, V* __restrict__ dst) {
+                                                          int64_t rows, const int32_t* __restrict__ rows_used,
+                                                          V* __restrict__ dst) {
+  if (rows_used) rows = min(rows, static_cast<int64_t>(max(*rows_used, 0)));
   const int64_t total = rows * row_elems;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < total; i += stride) {
@@ -197,7 +200,8 @@ extern "C" mbe_status mbe_refresh_plan(const uint8_t* block_changed, int32_t max
 }
 
 extern "C" mbe_status mbe_gather_rows(const void* src, int64_t src_rows, int64_t row_bytes, const int32_t* src_row,
-                                      int64_t rows, void* dst, cudaStream_t stream) {
+                                      int64_t rows, const int32_t* rows_used_or_null, void* dst,
+                                      cudaStream_t stream) {
   using namespace mbe;
   if (src_rows < 0 || row_bytes < 1 || rows < 0) return MBE_ERR_INVALID_ARG;
   if (rows == 0) return MBE_OK;
@@ -215,13 +219,14 @@ extern "C" mbe_status mbe_gather_rows(const void* src, int64_t src_rows, int64_t
   const unsigned g = static_cast<unsigned>(ctas);
   if (width == 16)
     gather_rows_kernel<uint4><<<g, 256, 0, stream>>>(static_cast<const uint4*>(src), src_rows, row_bytes / 16,
-                                                     src_row, rows, static_cast<uint4*>(dst));
+                                                     src_row, rows, rows_used_or_null, static_cast<uint4*>(dst));
   else if (width == 4)
     gather_rows_kernel<uint32_t><<<g, 256, 0, stream>>>(static_cast<const uint32_t*>(src), src_rows, row_bytes / 4,
-                                                        src_row, rows, static_cast<uint32_t*>(dst));
+                                                        src_row, rows, rows_used_or_null,
+                                                        static_cast<uint32_t*>(dst));
   else
     gather_rows_kernel<uint8_t><<<g, 256, 0, stream>>>(static_cast<const uint8_t*>(src), src_rows, row_bytes,
-                                                       src_row, rows, static_cast<uint8_t*>(dst));
+                                                       src_row, rows, rows_used_or_null, static_cast<uint8_t*>(dst));
   return launch_status("gather_rows_kernel");
 }
 

@@ -95,7 +95,7 @@ def lib(build_if_missing: bool = True):
     L.mbe_refresh_plan.restype = ctypes.c_int
     L.mbe_refresh_plan.argtypes = [P, i32, P, P, P, P, i32, i32, i32, i32, i32, P, P, P, P, P, P, P, P]
     L.mbe_gather_rows.restype = ctypes.c_int
-    L.mbe_gather_rows.argtypes = [P, i64, i64, P, i64, P, P]
+    L.mbe_gather_rows.argtypes = [P, i64, i64, P, i64, P, P, P]
     L.mbe_pass_loop_begin.restype = ctypes.c_int
     L.mbe_pass_loop_begin.argtypes = [i32, P, P, ctypes.POINTER(ctypes.c_void_p)]
     L.mbe_pass_loop_until_stable.restype = ctypes.c_int
@@ -509,8 +509,10 @@ def refresh_plan(block_changed, prefix_len, window_len, cu_window, block_table, 
     return out
 
 
-def gather_rows(src, src_row, out=None, stream=None):
-    """mbe_gather_rows: out[k] = src[src_row[k]] (zero rows where src_row[k] < 0)."""
+def gather_rows(src, src_row, out=None, rows_used=None, stream=None):
+    """mbe_gather_rows: out[k] = src[src_row[k]] (zero rows where src_row[k] < 0);
+    with rows_used (a device int32 tensor, e.g. plan["count"][1:]) only rows
+    k < rows_used[0] are written."""
     _need(src, "src", None)
     _need(src_row, "src_row", torch.int32)
     rows = src_row.numel()
@@ -520,7 +522,10 @@ def gather_rows(src, src_row, out=None, stream=None):
     if tuple(out.shape[1:]) != tuple(src.shape[1:]) or out.shape[0] != rows:
         raise ValueError("out must be [len(src_row)] + src.shape[1:]")
     row_bytes = (src[0].numel() if src.shape[0] else out[0].numel() if rows else 1) * src.element_size()
-    st = lib().mbe_gather_rows(_ptr(src), src.shape[0], row_bytes, _ptr(src_row), rows, _ptr(out), _stream(stream))
+    if rows_used is not None:
+        _need(rows_used, "rows_used", torch.int32)
+    st = lib().mbe_gather_rows(_ptr(src), src.shape[0], row_bytes, _ptr(src_row), rows,
+                               _ptr(rows_used) if rows_used is not None else None, _ptr(out), _stream(stream))
     _check("mbe_gather_rows", st)
     return out
 

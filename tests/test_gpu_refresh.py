@@ -90,6 +90,17 @@ def test_gather_rows(shape, dtype):
     assert not got[3].any()
     st, flags = mbe.get_device_error()
     assert flags == mbe.DEVERR_LENGTH
+    # a device row count: rows from it on keep what the output held
+    fill = torch.full((70,) + shape[1:], 9, dtype=dtype, device=DEV)
+    n = torch.tensor([41], dtype=torch.int32, device=DEV)
+    idx[3] = 0
+    got = mbe.gather_rows(src.to(DEV), idx.to(DEV), out=fill, rows_used=n).cpu()
+    ref[3] = src[0]
+    assert torch.equal(got[:41], ref[:41]) and (got[41:] == 9).all()
+    n.fill_(-3)
+    got = mbe.gather_rows(src.to(DEV), idx.to(DEV), out=fill, rows_used=n).cpu()
+    assert torch.equal(got[:41], ref[:41]) and (got[41:] == 9).all()
+    assert mbe.get_device_error() == (0, 0)
 
 
 def _refresh_problem(seed):
@@ -144,7 +155,8 @@ def _gpu_refresh(prob, old, changed, B, stream=None, bufs=None):
                             max_window=mw, total_rows=T, out=bufs["plan"], stream=stream)
     bufs["plan"] = plan
     for src, dst in ((d.q, bufs["q"]), (d.k_win, bufs["k"]), (d.v_win, bufs["v"])):
-        mbe.gather_rows(src, plan["src_row"], out=dst, stream=stream)
+        # only the refresh rows are gathered; the rest of the buffers are never read
+        mbe.gather_rows(src, plan["src_row"], out=dst, rows_used=plan["count"][1:], stream=stream)
     mbe.kv_window_write(bufs["k"], bufs["v"], d.k_cache, d.v_cache, plan["block_table"], plan["prefix_len"],
                         plan["window_len"], plan["cu_window"], block_size=B, max_window=B, stream=stream)
     mbe.window_attention(bufs["q"], bufs["k"], bufs["v"], d.k_cache, d.v_cache, plan["block_table"],
