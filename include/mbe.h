@@ -102,7 +102,8 @@ typedef enum { MBE_F32 = 0, MBE_BF16 = 1 } mbe_dtype;
  *              MBE_DEVERR_PAGE.
  *   prefix_len, window_len int32 [batch]; cu_window int32 [batch + 1] with
  *              cu_window[0] = 0, cu_window[s+1] = cu_window[s] + window_len[s],
- *              cu_window[batch] = total_q_tokens.
+ *              cu_window[batch] <= total_q_tokens (rows past it are not
+ *              attended to, and those of out are not written).
  *   mask_mode  uint8 [batch], values of mbe_mask_mode (per sequence, so mixed
  *              standard and editing passes run in one launch).
  *   max_window, max_prefix  host upper bounds of window_len[] and prefix_len[]
@@ -117,7 +118,8 @@ typedef enum { MBE_F32 = 0, MBE_BF16 = 1 } mbe_dtype;
  *              concurrent calls.
  * Supported: head_dim in {64, 128}; num_q_heads / num_kv_heads a power of two
  * <= 128; page_size a power of two >= 8; block_size >= 1. Rows of k_win/v_win
- * for all total_q_tokens tokens must hold finite values.
+ * outside every window, and cache rows past a prefix, may hold any bits (NaN
+ * included): they never reach out.
  * Errors: MBE_ERR_INVALID_ARG, MBE_ERR_UNSUPPORTED, MBE_ERR_WORKSPACE,
  * MBE_ERR_CUDA (launch failure).
  */

@@ -898,12 +898,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         tmem_st_wait();
-        if (wg == 0 && t == nP - 1 && (P % kTileKeys) != 0) {
-          // stale cache rows past the prefix end: zero them in V so that 0 * V stays 0
+        // Rows past the end of the last prefix tile (stale cache rows) or of the
+        // last window tile (whatever follows the window in k_win / v_win, even
+        // NaN) are masked in S but still enter P V as 0 * V: zero them in V.
+        const int v0 = (t == nP - 1) ? P % kTileKeys : (t - nP == (W - 1) / kTileKeys ? W % kTileKeys : 0);
+        if (wg == 0 && v0 != 0) {
           const uint32_t nv = 2 * ki + 1;  // the V item of this tile
           ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.full[nv % S::kSlots]), (nv / S::kSlots) & 1, abort_flag));
           if (!ok) break;
-          const int v0 = P % kTileKeys;
           uint8_t* vt = smem + S::kRing + (nv % S::kSlots) * S::kItem;
           const int per_row = S::kHalves * 8;  // 16-byte chunks per key row
           for (int idx = r; idx < (kTileKeys - v0) * per_row; idx += kTileRows) {

@@ -116,6 +116,22 @@ def test_stale_cache_rows_past_prefix_do_not_leak():
     assert torch.equal(out, ref) and torch.equal(lse, ref_lse)
 
 
+@pytest.mark.parametrize("mode", [BIDIRECTIONAL, BLOCK_CAUSAL])
+def test_rows_past_the_last_window_do_not_leak(mode):
+    """q / k_win / v_win rows after cu_window[batch] hold NaN: the last key tile
+    reads them, and neither out nor lse may see them."""
+    prob = attention_problem([45, 300], [32, 72], [mode, mode], 8, 2, 128, 32, 32, seed=14, device=DEV)
+    ref, ref_lse = run_attention(prob)
+    T = int(prob.cu_window[-1])
+
+    def pad(x):
+        return torch.cat([x, torch.full((200,) + tuple(x.shape[1:]), float("nan"), dtype=x.dtype, device=DEV)])
+    out, lse = run_attention(AttnProblem(**{**prob.__dict__, "q": pad(prob.q), "k_win": pad(prob.k_win),
+                                            "v_win": pad(prob.v_win)}))
+    assert torch.isfinite(out[:T].float()).all()
+    assert torch.equal(out[:T], ref) and torch.equal(lse[:T], ref_lse)
+
+
 def test_empty_windows_and_zero_prefix():
     prob = attention_problem([100, 0, 64, 0], [0, 32, 0, 64], [BIDIRECTIONAL, BLOCK_CAUSAL, BIDIRECTIONAL,
                                                                BIDIRECTIONAL], 8, 2, 128, 32, 32, seed=2, device=DEV)

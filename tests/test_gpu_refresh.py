@@ -144,8 +144,10 @@ def _gpu_refresh(prob, old, changed, B, stream=None, bufs=None):
     E = prob.batch * changed.shape[1]
     if bufs is None:
         bufs = {"prob": d, "old_k": old.k_win.to(DEV), "old_v": old.v_win.to(DEV), "changed": changed.to(DEV),
-                "plan": None, "q": torch.empty_like(d.q), "k": torch.empty_like(d.k_win),
-                "v": torch.empty_like(d.k_win), "out": torch.zeros_like(d.q),
+                # NaN rows: only the refresh rows are gathered, and the rows after
+                # them (read in the last key tile) must never reach the output
+                "plan": None, "q": torch.full_like(d.q, float("nan")), "k": torch.full_like(d.k_win, float("nan")),
+                "v": torch.full_like(d.k_win, float("nan")), "out": torch.zeros_like(d.q),
                 "ws": torch.empty(mbe.window_attention_workspace_size(E, 8, 2, 128, B, _refresh_max_prefix(prob)),
                                   dtype=torch.uint8, device=DEV)}
     mw = max(prob.window_host)
@@ -178,8 +180,8 @@ def test_refresh_attention_and_cache_match_oracle():
     assert np.abs(got - out_ref).max() <= ATTN_ATOL
     np.testing.assert_array_equal(bf16_bits(bufs["prob"].k_cache.cpu()), kc_ref)
     np.testing.assert_array_equal(bf16_bits(bufs["prob"].v_cache.cpu()), vc_ref)
-    # rows past the refresh rows gathered as zeros
-    assert not bufs["q"][n:].any()
+    # rows past the refresh rows are left as they were
+    assert bufs["q"][n:].isnan().all() and bufs["v"][n:].isnan().all()
 
 
 def test_refresh_in_a_captured_graph_matches_eager():
