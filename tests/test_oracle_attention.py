@@ -185,6 +185,31 @@ def test_gqa_equals_replicated_kv_heads():
     np.testing.assert_array_equal(out, out_r)
 
 
+@pytest.mark.parametrize("mode", [BIDIRECTIONAL, BLOCK_CAUSAL])
+def test_split_invariance_prefix_and_window_merge_by_lse(mode):
+    """Attention over prefix + window equals the log-sum-exp merge of attention
+    over the prefix alone and over the window alone (the identity split-KV
+    merging relies on). With P = W the prefix-only part is the oracle itself,
+    run with no prefix on a window made of the prefix rows (bidirectional)."""
+    P = W = 48
+    prob = attention_problem([P], [W], [mode], 4, 2, 16, 16, 16, seed=21)
+    full, full_lse = oracle_attention(prob)
+    no_prefix = {"prefix_len": torch.tensor([0], dtype=torch.int32), "prefix_host": [0]}
+    ow, lw = oracle_attention(AttnProblem(**{**prob.__dict__, **no_prefix}))
+    pos = torch.arange(P)
+    pages = prob.block_table[0][pos // prob.page_size].long()
+    kp = prob.k_cache[pages, :, pos % prob.page_size]          # [P, Hkv, D], rows in logical order
+    vp = prob.v_cache[pages, :, pos % prob.page_size]
+    op, lp = oracle_attention(AttnProblem(**{**prob.__dict__, **no_prefix, "k_win": kp, "v_win": vp,
+                                             "mask_mode": torch.tensor([BIDIRECTIONAL], dtype=torch.uint8),
+                                             "mode_host": [BIDIRECTIONAL]}))
+    m = np.maximum(lp, lw)
+    wp, ww = np.exp(lp - m), np.exp(lw - m)
+    merged = (wp[..., None] * op + ww[..., None] * ow) / (wp + ww)[..., None]
+    np.testing.assert_allclose(full, merged, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(full_lse, m + np.log(wp + ww), rtol=0, atol=1e-12)
+
+
 def test_units_subset_matches_full():
     prob = attention_problem([60, 33], [32, 64], [BIDIRECTIONAL, BLOCK_CAUSAL], 4, 2, 16, 32, 16, seed=12)
     out, lse = oracle_attention(prob)
