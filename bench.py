@@ -296,7 +296,7 @@ def run_gpu(args, rank, world):
                               "ms": round(edit_ms, 4), "bytes": eb,
                               "edit_rate": round(float(mask_t.float().mean().item()), 5)}
     res["roofline"] = {"bound": "hbm", "achieved": round(attn_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                       "frac": round(attn_gbs / peaks["hbm_gbs"], 4), "traffic": measured_traffic(args.workload),
+                       "frac": round(attn_gbs / peaks["hbm_gbs"], 4), "traffic": measured_traffic(args.workload) if args.batch in (None, 128) else None,
                        "kernel": "mbe_window_attention per layer (attn_kernel + split merge; one plan per pass)",
                        "peak_source": f"{peak_src} hbm_gbs"}
     res["clocks"] = clocks

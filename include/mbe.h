@@ -362,7 +362,9 @@ mbe_status mbe_sft_block_mask(const int32_t* n_prompt_blocks, const int32_t* n_b
  * 1/sqrt(head_dim). Key tiles of 128 keys that no row of a 256-row work unit
  * sees are skipped. block_size must be a power of two >= 8 and max_seq_len <=
  * 65536; workspace as for mbe_window_attention_workspace_size(batch,
- * num_q_heads, num_kv_heads, head_dim, max_seq_len, 0).
+ * num_q_heads, num_kv_heads, head_dim, max_seq_len, 0). Rows of q, k and v
+ * after cu_seqlens[batch] may hold any bits (NaN included): they never reach
+ * out.
  * Errors as mbe_window_attention.
  */
 mbe_status mbe_block_mask_attention(const void* q, const void* k, const void* v, const int32_t* seq_len,
@@ -387,7 +389,10 @@ mbe_status mbe_block_mask_attention(const void* q, const void* k, const void* v,
  * workspace: mbe_block_mask_attention_bwd_workspace_size(batch, total_tokens,
  * num_q_heads) bytes, 16-byte aligned. head_dim must be 128; num_q_heads /
  * num_kv_heads must divide 32; max_seq_len * that ratio <= 65536. Rows past
- * cu_seqlens[batch] are not written.
+ * cu_seqlens[batch] are not written; where total_tokens exceeds
+ * cu_seqlens[batch], those rows of q, k, v, out and dout must hold finite
+ * values (the last tiles of the last sequence read them, and masked products
+ * still multiply them by zero).
  * Errors: MBE_ERR_INVALID_ARG, MBE_ERR_UNSUPPORTED, MBE_ERR_WORKSPACE,
  * MBE_ERR_CUDA; a bounded wait that expires sets MBE_DEVERR_TIMEOUT.
  */

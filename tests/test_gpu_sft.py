@@ -11,6 +11,8 @@ is formed from the bf16 forward output, |O_bf16 - O| <= u |O|, which moves dS
 by at most P u sum_d |dO||O| and adds scale (P u sum_d |dO||O|)^T |Q| to dK and
 the same against |K| to dQ. Every gradient also stays within 1e-2 relative in
 the Frobenius norm."""
+import dataclasses
+
 import numpy as np
 import pytest
 import torch
@@ -91,6 +93,22 @@ def test_forward_with_a_hand_mask_and_an_empty_row():
     out, lse = _run(prob, mask)
     _check(prob, bits, out, lse)
     assert np.isneginf(lse[32:64]).all()
+
+
+def test_forward_rows_after_the_last_sequence_do_not_leak():
+    """q / k / v rows after cu_seqlens[batch] hold NaN: the last key tile of the
+    last sequence reads them, and the output must not see them."""
+    prob = sft_problem([1, 0], [3, 4], 8, 2, 128, 32, seed=13, trim=[0, 9])
+    mask = _gpu_mask(prob, 2)
+    ref, ref_lse = _run(prob, mask)
+    T = int(prob.cu_seqlens[-1])
+    pad = lambda x: torch.cat([x, torch.full((100,) + tuple(x.shape[1:]), float("nan"), dtype=x.dtype)])
+    padded = dataclasses.replace(prob, q=pad(prob.q), k=pad(prob.k), v=pad(prob.v))
+    out, lse = _run(padded, mask)
+    assert np.isfinite(out[:T]).all()
+    np.testing.assert_array_equal(out[:T], ref)
+    np.testing.assert_array_equal(lse[:T], ref_lse)
+    _check(prob, mask.cpu().numpy().view(np.uint32), out[:T], lse[:T])
 
 
 def test_longer_sequences_with_split_pieces():
