@@ -838,13 +838,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         float mx = neg_inf();
         if (full) {
-          float a0 = neg_inf(), a1 = neg_inf();
+          // eight independent accumulators: the maximum does not depend on the order,
+          // and short dependency chains keep the softmax latency down
+          float acc[8];
 #pragma unroll
-          for (int k = 0; k < 128; k += 4) {
-            a0 = fmax3(a0, __uint_as_float(v[k]), __uint_as_float(v[k + 1]));
-            a1 = fmax3(a1, __uint_as_float(v[k + 2]), __uint_as_float(v[k + 3]));
-          }
-          mx = fmaxf(a0, a1);
+          for (int a = 0; a < 8; ++a) acc[a] = neg_inf();
+#pragma unroll
+          for (int k = 0; k < 128; k += 16)
+#pragma unroll
+            for (int a = 0; a < 8; ++a)
+              acc[a] = fmax3(acc[a], __uint_as_float(v[k + 2 * a]), __uint_as_float(v[k + 2 * a + 1]));
+          mx = fmaxf(fmax3(acc[0], acc[1], acc[2]), fmax3(acc[3], fmax3(acc[4], acc[5], acc[6]), acc[7]));
         } else {
 #pragma unroll
           for (int k = 0; k < 128; ++k)
