@@ -52,6 +52,7 @@ constexpr int kMaxGroupedSlabs = 8; // slabs of one (sequence, KV head) kept adj
 constexpr float kUnitStartTiles = 2.f;  // start-up cost of a work unit, in key tiles (scheduler estimate)
 constexpr int kBuckets = 1024;      // counting-sort buckets for unit cost
 constexpr float kRescaleLog2 = 8.0f;  // rescale O only when the max grows by > 2^8
+constexpr float kSpeculateSum = 128.f; // a tile's row sum below 2^7 proves no value reached 2^8
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kTmemS = 256;    // S/P of tile i at columns 256 + 128 i; O_i at i * D
 
@@ -836,36 +837,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             full = true;
           }
         }
-        float mx = neg_inf();
-        if (full) {
-          // eight independent accumulators: the maximum does not depend on the order,
-          // and short dependency chains keep the softmax latency down
-          float acc[8];
-#pragma unroll
-          for (int a = 0; a < 8; ++a) acc[a] = neg_inf();
-#pragma unroll
-          for (int k = 0; k < 128; k += 16)
-#pragma unroll
-            for (int a = 0; a < 8; ++a)
-              acc[a] = fmax3(acc[a], __uint_as_float(v[k + 2 * a]), __uint_as_float(v[k + 2 * a + 1]));
-          mx = fmaxf(fmax3(acc[0], acc[1], acc[2]), fmax3(acc[3], fmax3(acc[4], acc[5], acc[6]), acc[7]));
-        } else {
-#pragma unroll
-          for (int k = 0; k < 128; ++k)
-            if (visible(k)) mx = fmaxf(mx, __uint_as_float(v[k]));
-        }
-        // Lazy rescaling: the reference max m only moves when the tile's max
-        // exceeds it by more than 2^8; P, l and O then all use the new m.
-        const float m_new = fmaxf(m, mx * p.scale_log2);
-        const bool rescale = __any_sync(0xffffffffu, m_new > m + kRescaleLog2);
-        float alpha = 1.f;
-        if (rescale) {
-          alpha = (m_new == neg_inf()) ? 1.f : ex2f(m - m_new);
-          m = m_new;
-        }
-        const float neg_mu = (m == neg_inf()) ? 0.f : -m;
-        float l0 = 0.f, l1 = 0.f;
-        if (full) {
+        // exponentials of a fully visible tile against the reference max: P (bf16
+        // pairs) replaces the first half of v, (l0, l1) are its row sums
+        auto exp_full = [&](float neg_mu, float& l0, float& l1) {
           const float2 sl2 = make_float2(p.scale_log2, p.scale_log2), nm2 = make_float2(neg_mu, neg_mu);
           float2 la = make_float2(0.f, 0.f), lb = make_float2(0.f, 0.f);
 #pragma unroll
@@ -878,14 +852,57 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float2 ls = fadd2(la, lb);
           l0 = ls.x;
           l1 = ls.y;
-        } else {
+        };
+        // Lazy rescaling: the reference max m only moves when the tile's max
+        // exceeds it by more than 2^8; P, l and O then all use the new m. A fully
+        // visible tile with a finite m first takes its exponentials against m as it
+        // stands: if no row's sum exceeds 2^7, no value reached 2^8, m would not move
+        // and P is final (the values the max-first order gives). Otherwise S is read
+        // again and the row max decides, as for every other tile.
+        float l0 = 0.f, l1 = 0.f, alpha = 1.f;
+        bool rescale = false, done = false;
+        if (full && __all_sync(0xffffffffu, m != neg_inf())) {
+          exp_full(-m, l0, l1);
+          done = !__any_sync(0xffffffffu, !(l0 + l1 <= kSpeculateSum));
+          if (!done) tmem_ld128(tS, v);
+        }
+        if (!done) {
+          float mx = neg_inf();
+          if (full) {
+            // eight independent accumulators: the maximum does not depend on the order,
+            // and short dependency chains keep the softmax latency down
+            float acc[8];
 #pragma unroll
-          for (int k = 0; k < 64; ++k) {
-            const float p0 = visible(2 * k) ? ex2f(fmaf(__uint_as_float(v[2 * k]), p.scale_log2, neg_mu)) : 0.f;
-            const float p1 = visible(2 * k + 1) ? ex2f(fmaf(__uint_as_float(v[2 * k + 1]), p.scale_log2, neg_mu)) : 0.f;
-            l0 += p0;
-            l1 += p1;
-            v[k] = pack_bf16x2(p0, p1);
+            for (int a = 0; a < 8; ++a) acc[a] = neg_inf();
+#pragma unroll
+            for (int k = 0; k < 128; k += 16)
+#pragma unroll
+              for (int a = 0; a < 8; ++a)
+                acc[a] = fmax3(acc[a], __uint_as_float(v[k + 2 * a]), __uint_as_float(v[k + 2 * a + 1]));
+            mx = fmaxf(fmax3(acc[0], acc[1], acc[2]), fmax3(acc[3], fmax3(acc[4], acc[5], acc[6]), acc[7]));
+          } else {
+#pragma unroll
+            for (int k = 0; k < 128; ++k)
+              if (visible(k)) mx = fmaxf(mx, __uint_as_float(v[k]));
+          }
+          const float m_new = fmaxf(m, mx * p.scale_log2);
+          rescale = __any_sync(0xffffffffu, m_new > m + kRescaleLog2);
+          if (rescale) {
+            alpha = (m_new == neg_inf()) ? 1.f : ex2f(m - m_new);
+            m = m_new;
+          }
+          const float neg_mu = (m == neg_inf()) ? 0.f : -m;
+          if (full) {
+            exp_full(neg_mu, l0, l1);
+          } else {
+#pragma unroll
+            for (int k = 0; k < 64; ++k) {
+              const float p0 = visible(2 * k) ? ex2f(fmaf(__uint_as_float(v[2 * k]), p.scale_log2, neg_mu)) : 0.f;
+              const float p1 = visible(2 * k + 1) ? ex2f(fmaf(__uint_as_float(v[2 * k + 1]), p.scale_log2, neg_mu)) : 0.f;
+              l0 += p0;
+              l1 += p1;
+              v[k] = pack_bf16x2(p0, p1);
+            }
           }
         }
         tmem_st64(tS, v);
