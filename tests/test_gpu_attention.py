@@ -61,6 +61,29 @@ def test_sharp_attention_outputs_order_one():
     assert out.float().abs().max().item() > 1.0
 
 
+def test_scores_rising_across_key_tiles_rescale_every_tile():
+    """Every query is aligned with one direction and the prefix keys grow along
+    it, so each key tile's scores exceed the previous tile's by about 20 (log2
+    units): the exponentials taken against the running maximum overflow their
+    2^7 check on every tile, the kernel falls back to the max-first order and
+    rescales O each time. The result must still match the oracle."""
+    P, W, D = 1000, 64, 128
+    prob = attention_problem([P], [W], [BIDIRECTIONAL], 8, 2, D, 32, 64, seed=17)
+    g = torch.Generator().manual_seed(17)
+    u = torch.randn(D, generator=g)
+    u /= u.norm()
+    q = (8.0 * u).expand_as(prob.q).to(torch.bfloat16)
+    kc = prob.k_cache.clone()
+    for j in range(P):
+        page = int(prob.block_table[0, j // prob.page_size])
+        kc[page, :, j % prob.page_size] = (20.0 * j / 128.0 * u).to(torch.bfloat16)
+    steep = AttnProblem(**{**prob.__dict__, "q": q, "k_cache": kc})
+    out, lse = run_attention(steep.to(DEV))
+    compare_attention(steep, out, lse)
+    # the softmax is concentrated on the last prefix keys: lse grows with the last score
+    assert lse.float().min().item() > 100.0
+
+
 def test_probability_probe_on_gpu_output():
     """V = one-hot key positions: the GPU output row is the probability row;
     masked keys must get exactly 0 and rows must sum to 1."""
