@@ -15,8 +15,9 @@
 //       warp 1      MMA issuer: S_i = Q_i K^T (SS form) and O_i += P_i V
 //                   (TS form, P read from TMEM), tcgen05, accumulators in TMEM
 //       warps 4-11  two softmax warpgroups, one per 128-row query tile: TMEM
-//                   load of S, row max, exp2, P written back to TMEM as bf16,
-//                   lazy rescaling of O, epilogue
+//                   load of S, exp2 against the running max (the row max is
+//                   taken first only where the max may have moved by 2^8),
+//                   P written back to TMEM as bf16, lazy rescaling of O, epilogue
 //     GQA: the G query heads sharing a KV head are packed into the rows of a
 //     tile (row = token * G + head), so every K/V tile feeds 256 query rows.
 //     The mask is applied per row as a visible-column count: every prefix key
