@@ -808,14 +808,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         // The whole S row (128 fp32) comes from TMEM in one load; P is packed to
         // bf16 in place (entry k <- columns 2k, 2k+1) and stored as 64 columns
         // over the start of the same TMEM region.
-        bool full = __all_sync(0xffffffffu, n_vis == kTileKeys && (!kMask || nib == all_bits));
+        const bool all_vis = __all_sync(0xffffffffu, n_vis == kTileKeys && (!kMask || nib == all_bits));
+        bool full = all_vis;
         uint32_t v[128];
         tmem_ld128(tS, v);
+        // block-mask mode: invisible columns (other key blocks, past the sequence)
+        // become -inf and the tile takes the packed path (exp2(-inf) = 0); cm holds
+        // this row's visible columns so that S read again is masked the same way
+        uint32_t cm[4] = {0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu};
+        auto mask_invisible = [&]() {
+#pragma unroll
+          for (int k = 0; k < 128; ++k)
+            if (!((cm[k >> 5] >> (k & 31)) & 1u)) v[k] = 0xFF800000u;
+        };
         if constexpr (kMask) {
-          // block-mask mode: invisible columns (other key blocks, past the sequence)
-          // become -inf and the tile takes the packed path (exp2(-inf) = 0)
-          if (!full) {
-            uint32_t cm[4];
+          if (!all_vis) {
 #pragma unroll
             for (int w = 0; w < 4; ++w) {
               uint32_t bits;
@@ -832,9 +839,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               bits &= n_vis >= lo + 32 ? 0xFFFFFFFFu : (n_vis <= lo ? 0u : ((1u << (n_vis - lo)) - 1u));
               cm[w] = bits;
             }
-#pragma unroll
-            for (int k = 0; k < 128; ++k)
-              if (!((cm[k >> 5] >> (k & 31)) & 1u)) v[k] = 0xFF800000u;
+            mask_invisible();
             full = true;
           }
         }
@@ -865,7 +870,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (full && __all_sync(0xffffffffu, m != neg_inf())) {
           exp_full(-m, l0, l1);
           done = !__any_sync(0xffffffffu, !(l0 + l1 <= kSpeculateSum));
-          if (!done) tmem_ld128(tS, v);
+          if (!done) {
+            tmem_ld128(tS, v);
+            if (kMask && !all_vis) mask_invisible();
+          }
         }
         if (!done) {
           float mx = neg_inf();

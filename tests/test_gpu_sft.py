@@ -111,6 +111,29 @@ def test_forward_rows_after_the_last_sequence_do_not_leak():
     _check(prob, mask.cpu().numpy().view(np.uint32), out[:T], lse[:T])
 
 
+def test_forward_rising_scores_under_a_partial_mask():
+    """Keys grow along the queries' direction, so every key tile's scores exceed
+    the running maximum by about 2^20 and the kernel falls back from the
+    speculated exponentials to the max-first order; the mask hides every odd key
+    block, so those tiles are partially visible and the fallback (which reads S
+    again) must keep the hidden columns, which hold the larger scores, out."""
+    B = 32
+    prob = sft_problem([0], [16], 4, 1, 128, B, seed=23)  # 32 blocks, 1024 tokens
+    T = prob.seq_host[0]
+    nb = T // B
+    g = torch.Generator().manual_seed(23)
+    u = torch.randn(128, generator=g)
+    u /= u.norm()
+    q = (8.0 * u).expand_as(prob.q).to(torch.bfloat16).contiguous()
+    k = torch.stack([20.0 * j / 128.0 * u for j in range(T)])[:, None, :].expand_as(prob.k)
+    steep = dataclasses.replace(prob, q=q, k=k.to(torch.bfloat16).contiguous())
+    bits = np.zeros((1, nb, 1), np.uint32)
+    bits[0, :, 0] = sum(1 << kb for kb in range(0, nb, 2))  # even key blocks only
+    mask = torch.from_numpy(bits.view(np.int32)).to(DEV)
+    out, lse = _run(steep, mask)
+    _check(steep, bits, out, lse)
+
+
 def test_longer_sequences_with_split_pieces():
     # few long sequences: the scheduler splits the key range; the merge combines pieces
     prob = sft_problem([2, 1], [40, 25], 8, 2, 128, 32, seed=11)  # 2624 and 1632 tokens
