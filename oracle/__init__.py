@@ -44,7 +44,8 @@ _BUILD = _HERE / "_build"
 _LIB_PATH = _BUILD / "libmbe_oracle.so"
 _lib = None
 
-STATUS = {0: "ok", 1: "bad argument", 2: "page id out of range", 3: "non-finite logit", 4: "out of memory"}
+STATUS = {0: "ok", 1: "bad argument", 2: "page id out of range", 3: "rows without a softmax", 4: "out of memory"}
+UNDECIDABLE = 3  # completed; some logit rows had no softmax (NaN / +inf, or every logit -inf)
 
 
 def build(force: bool = False) -> Path:
@@ -159,7 +160,10 @@ def edit_decide(logits, committed, tau=0.0, tau_per_row=None, editable=None, row
 
     logits: float32 [R, V], float64 [R, V] or uint16 bf16 bits [R, V] (set is_bf16).
     Returns dict of new_tokens int32, edit_mask uint8, confidence float64,
-    argmax int32 (all [R]; rows not in `rows` are left as -1 / 0 / NaN).
+    argmax int32 (all [R]; rows not in `rows` are left as -1 / 0 / NaN) and
+    "undecidable": True if some computed row had no softmax (a NaN or +inf
+    logit, or every logit -inf); such a row keeps its token, with argmax -1 and
+    confidence NaN.
     """
     lib = _load()
     logits = np.ascontiguousarray(logits)
@@ -178,14 +182,17 @@ def edit_decide(logits, committed, tau=0.0, tau_per_row=None, editable=None, row
     rc = lib.oracle_edit_decide(_ptr(logits), dtype, V, R, V, _ptr(committed), _ptr(tpr), float(tau), _ptr(ed),
                                 -1 if sel is None else sel.shape[0], _ptr(sel), _ptr(new), _ptr(mask), _ptr(conf),
                                 _ptr(am))
-    _check(rc)
-    return {"new_tokens": new, "edit_mask": mask, "confidence": conf, "argmax": am}
+    if rc != UNDECIDABLE:
+        _check(rc)
+    return {"new_tokens": new, "edit_mask": mask, "confidence": conf, "argmax": am, "undecidable": rc == UNDECIDABLE}
 
 
 def denoise_update(logits, tokens, cu_rows, block_size, mask_id, omega_mask, omega_edit, editable=None,
                    max_blocks=None, is_bf16=False):
     """Full Eq. 2 update (Gamma_t, forced unmasking, Delta_t) with entropies,
-    changed-block flags and per-sequence change counts, in float64."""
+    changed-block flags and per-sequence change counts, in float64.
+    "undecidable" is True if some row had no softmax (it keeps its token, with
+    argmax -1 and confidence / entropy NaN, and is never force-unmasked)."""
     lib = _load()
     dtype = _logit_dtype(logits, is_bf16)
     logits = np.ascontiguousarray(logits) if dtype else np.ascontiguousarray(logits, dtype=np.float32)
@@ -203,7 +210,9 @@ def denoise_update(logits, tokens, cu_rows, block_size, mask_id, omega_mask, ome
                                    _ptr(_c(editable, np.uint8)), _ptr(out["new_tokens"]), _ptr(out["kind"]),
                                    _ptr(out["confidence"]), _ptr(out["argmax"]), _ptr(out["entropy"]),
                                    _ptr(out["block_changed"]), _ptr(out["seq_changes"]))
-    _check(rc)
+    if rc != UNDECIDABLE:
+        _check(rc)
+    out["undecidable"] = rc == UNDECIDABLE
     return out
 
 

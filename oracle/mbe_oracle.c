@@ -33,7 +33,7 @@
 #define ORC_OK 0
 #define ORC_BAD_ARG 1
 #define ORC_BAD_PAGE 2
-#define ORC_NONFINITE 3
+#define ORC_UNDECIDABLE 3 /* completed; some rows had no softmax (see row_softmax) */
 #define ORC_NOMEM 4
 
 /* bf16 bit pattern -> exact double */
@@ -49,6 +49,37 @@ static double load_logit(const void* logits, int32_t dtype, int64_t idx) {
   if (dtype == 0) return (double)((const float*)logits)[idx];
   if (dtype == 1) return bf16_to_double(((const uint16_t*)logits)[idx]);
   return ((const double*)logits)[idx];
+}
+
+/*
+ * Softmax statistics of logit row `off` (vocab entries): the maximum m, its
+ * lowest index x_hat and S = sum_v exp(l_v - m). The row has a softmax only if
+ * none of its logits is NaN or +inf and at least one is finite; a -inf logit
+ * is a token of probability 0 (a vocabulary mask). Returns 0, with x_hat = -1,
+ * for a row without a softmax: Eq. 2 cannot decide on it ("undecidable").
+ */
+static int row_softmax(const void* logits, int32_t dtype, int64_t off, int32_t vocab, double* m_out,
+                       int32_t* xh_out, double* s_out) {
+  double m = -INFINITY;
+  int32_t xh = -1;
+  for (int32_t v = 0; v < vocab; ++v) {
+    const double x = load_logit(logits, dtype, off + v);
+    if (isnan(x) || x == INFINITY) {
+      *xh_out = -1;
+      return 0;
+    }
+    if (x > m) {
+      m = x;
+      xh = v;
+    }
+  }
+  *xh_out = xh;
+  if (xh < 0) return 0; /* every logit is -inf */
+  double ssum = 0.0;
+  for (int32_t v = 0; v < vocab; ++v) ssum += exp(load_logit(logits, dtype, off + v) - m);
+  *m_out = m;
+  *s_out = ssum;
+  return 1;
 }
 
 int oracle_num_threads(void) {
@@ -202,7 +233,9 @@ int oracle_window_attention(const uint16_t* q, const uint16_t* k_win, const uint
  * tau_r is tau_per_row[r] when given, else tau. The comparison c > tau_r is
  * taken on c rounded to float, the precision of tau. editable == NULL means
  * every row is editable (the caller restricts edits to the historical part of
- * the window, Sec. 4.1).
+ * the window, Sec. 4.1). A row without a softmax (a NaN or +inf logit, or
+ * every logit -inf; see row_softmax) keeps its token: edit 0, x_hat -1, c NaN,
+ * and the call returns ORC_UNDECIDABLE after finishing every row.
  * dtype 0: float32 logits, 1: bf16 logits, 2: float64 logits (the LM-head
  * projection of oracle_lm_head_logits). If n_sel >= 0 only rows
  * sel_rows[0..n_sel-1] are computed; outputs are indexed by row.
@@ -213,35 +246,25 @@ int oracle_edit_decide(const void* logits, int32_t dtype, int64_t row_stride, in
                        double* confidence, int32_t* argmax_out) {
   if (rows < 0 || vocab <= 0 || dtype < 0 || dtype > 2 || row_stride < vocab) return ORC_BAD_ARG;
   const int64_t total = n_sel >= 0 ? n_sel : rows;
-  int status = ORC_OK;
+  int bad_arg = 0, undecidable = 0;
 #pragma omp parallel for schedule(static)
   for (int64_t u = 0; u < total; ++u) {
     const int32_t r = n_sel >= 0 ? sel_rows[u] : (int32_t)u;
     if (r < 0 || r >= rows) {
 #pragma omp atomic write
-      status = ORC_BAD_ARG;
+      bad_arg = 1;
       continue;
     }
-    double m = -INFINITY;
+    double m = 0.0, ssum = 0.0;
     int32_t xh = -1;
-    int finite = 1;
-    for (int32_t v = 0; v < vocab; ++v) {
-      const double x = load_logit(logits, dtype, (int64_t)r * row_stride + v);
-      if (!isfinite(x)) finite = 0;
-      if (x > m) {
-        m = x;
-        xh = v;
-      }
-    }
-    if (!finite) {
+    if (!row_softmax(logits, dtype, (int64_t)r * row_stride, vocab, &m, &xh, &ssum)) {
 #pragma omp atomic write
-      status = ORC_NONFINITE;
+      undecidable = 1;
+      if (new_tokens) new_tokens[r] = committed[r];
+      if (edit_mask) edit_mask[r] = 0;
+      if (confidence) confidence[r] = NAN;
+      if (argmax_out) argmax_out[r] = -1;
       continue;
-    }
-    double ssum = 0.0;
-    for (int32_t v = 0; v < vocab; ++v) {
-      const double x = load_logit(logits, dtype, (int64_t)r * row_stride + v);
-      ssum += exp(x - m);
     }
     const double c = 1.0 / ssum;
     const float tr = tau_per_row ? tau_per_row[r] : tau;
@@ -251,7 +274,8 @@ int oracle_edit_decide(const void* logits, int32_t dtype, int64_t row_stride, in
     if (confidence) confidence[r] = c;
     if (argmax_out) argmax_out[r] = xh;
   }
-  return status;
+  if (bad_arg) return ORC_BAD_ARG;
+  return undecidable ? ORC_UNDECIDABLE : ORC_OK;
 }
 
 /*
@@ -304,6 +328,10 @@ int oracle_kv_window_write(const uint16_t* k_win, const uint16_t* v_win, uint16_
  * Then, per block: if the block has masked rows and none of them was unmasked,
  * its masked row of highest confidence (lowest row on equal confidence) is
  * unmasked anyway (kind 2). Confidence comparisons use c rounded to float.
+ * A row without a softmax (see row_softmax) keeps its token (kind 0) with
+ * x_hat -1 and c, H NaN; it is never the forced row, so a block whose masked
+ * rows all lack a softmax unmasks none. The call then returns ORC_UNDECIDABLE
+ * after finishing every row and block.
  * block_changed[s][b] = 1 iff some row of block b got a new token (new != x);
  * seq_changes[s] = number of rows of s whose token changed.
  */
@@ -315,40 +343,27 @@ int oracle_denoise_update(const void* logits, int32_t dtype, int64_t row_stride,
   if (num_seqs < 0 || vocab <= 0 || block_size <= 0 || dtype < 0 || dtype > 2 || row_stride < vocab)
     return ORC_BAD_ARG;
   const int32_t rows = num_seqs > 0 ? cu_rows[num_seqs] : 0;
-  int status = ORC_OK;
+  int undecidable = 0;
 #pragma omp parallel for schedule(static)
   for (int32_t r = 0; r < rows; ++r) {
-    double* x = (double*)malloc(sizeof(double) * (size_t)vocab);
-    if (!x) {
-#pragma omp atomic write
-      status = ORC_NOMEM;
-      continue;
-    }
-    double m = -INFINITY;
+    const int64_t off = (int64_t)r * row_stride;
+    double m = 0.0, ssum = 0.0;
     int32_t xh = -1;
-    int finite = 1;
-    for (int32_t v = 0; v < vocab; ++v) {
-      x[v] = load_logit(logits, dtype, (int64_t)r * row_stride + v);
-      if (!isfinite(x[v])) finite = 0;
-      if (x[v] > m) {
-        m = x[v];
-        xh = v;
-      }
-    }
-    if (!finite) {
-      free(x);
+    if (!row_softmax(logits, dtype, off, vocab, &m, &xh, &ssum)) {
 #pragma omp atomic write
-      status = ORC_NONFINITE;
+      undecidable = 1;
+      confidence[r] = NAN;
+      argmax_out[r] = -1;
+      if (entropy) entropy[r] = NAN;
+      kind[r] = 0;
+      new_tokens[r] = tokens[r];
       continue;
     }
-    double ssum = 0.0;
-    for (int32_t v = 0; v < vocab; ++v) ssum += exp(x[v] - m);
     double h = 0.0;
     for (int32_t v = 0; v < vocab; ++v) {
-      const double pv = exp(x[v] - m) / ssum;
+      const double pv = exp(load_logit(logits, dtype, off + v) - m) / ssum;
       if (pv > 0.0) h -= pv * log(pv);
     }
-    free(x);
     const double c = 1.0 / ssum;
     confidence[r] = c;
     argmax_out[r] = xh;
@@ -363,7 +378,6 @@ int oracle_denoise_update(const void* logits, int32_t dtype, int64_t row_stride,
     kind[r] = k;
     new_tokens[r] = k ? xh : cur;
   }
-  if (status != ORC_OK) return status;
   for (int32_t s = 0; s < num_seqs; ++s) {
     const int32_t r0 = cu_rows[s], r1 = cu_rows[s + 1];
     const int32_t nblocks = (r1 - r0 + block_size - 1) / block_size;
@@ -377,12 +391,13 @@ int oracle_denoise_update(const void* logits, int32_t dtype, int64_t row_stride,
         if (tokens[r] != mask_id) continue;
         any_masked = 1;
         if (kind[r] == 1) any_unmasked = 1;
+        if (argmax_out[r] < 0) continue; /* no softmax: never forced */
         if (best < 0 || (float)confidence[r] > best_c) {
           best = r;
           best_c = (float)confidence[r];
         }
       }
-      if (any_masked && !any_unmasked) {
+      if (any_masked && !any_unmasked && best >= 0) {
         kind[best] = 2;
         new_tokens[best] = argmax_out[best];
       }
@@ -398,7 +413,7 @@ int oracle_denoise_update(const void* logits, int32_t dtype, int64_t row_stride,
       for (int32_t b = nblocks; b < max_blocks; ++b) block_changed[(int64_t)s * max_blocks + b] = 0;
     if (seq_changes) seq_changes[s] = changes;
   }
-  return ORC_OK;
+  return undecidable ? ORC_UNDECIDABLE : ORC_OK;
 }
 
 static int cmp_desc(const void* a, const void* b) {

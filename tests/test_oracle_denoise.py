@@ -151,3 +151,59 @@ def test_forced_unmask_tie_takes_lowest_row():
     res = oracle.denoise_update(logits, [7, 7, 7, 7], [0, 4], 4, 7, 0.9, 0.0)
     assert res["kind"].tolist() == [2, 0, 0, 0]
     assert res["new_tokens"].tolist() == [1, 7, 7, 7]
+
+
+@pytest.mark.parametrize("bad", ["nan", "all_neginf"])
+def test_block_whose_masked_rows_lack_a_softmax_unmasks_nothing(bad):
+    """Forced unmasking (Sec. 2.3) picks the most confident masked row of a
+    block; a row without a softmax has no confidence, so it is never picked,
+    and a block whose masked rows all lack one unmasks none. Rows of the other
+    blocks are decided as without them."""
+    mask_id, B = 63, 8
+    logits, tokens = _random_step(24, 64, 11, 0.0, mask_id)
+    logits[:, mask_id] = -30.0                 # no row predicts [MASK]
+    masked = [9, 12, 14]                       # block 1 (rows 8..15): only these rows are masked
+    tokens[masked] = mask_id
+    for r in masked:
+        if bad == "nan":
+            logits[r, 5] = np.nan
+        else:
+            logits[r, :] = -np.inf
+    tokens[20] = mask_id                       # block 2: one masked row with a softmax
+    res = oracle.denoise_update(logits, tokens, [0, 24], B, mask_id, 2.0, 2.0)
+    assert res["undecidable"]
+    for r in masked:
+        assert res["kind"][r] == 0 and res["new_tokens"][r] == mask_id
+        assert res["argmax"][r] == -1 and np.isnan(res["confidence"][r]) and np.isnan(res["entropy"][r])
+    assert res["block_changed"][0, 1] == 0
+    assert res["kind"][20] == 2                # forced in its own block (omega_mask 2 admits nothing)
+    others = np.array([r for r in range(24) if r not in masked])
+    np.testing.assert_array_equal(res["argmax"][others], np.argmax(logits[others], axis=1))
+
+
+def test_forced_unmask_skips_rows_without_softmax():
+    """A block with one masked row that has a softmax and others that do not
+    force-unmasks that row, whatever the others' logits."""
+    mask_id, B = 63, 8
+    logits, tokens = _random_step(8, 64, 12, 0.0, mask_id)
+    logits[:, mask_id] = -30.0
+    tokens[[1, 2, 6]] = mask_id
+    logits[1, :] = -np.inf
+    logits[6, 0] = np.inf
+    res = oracle.denoise_update(logits, tokens, [0, 8], B, mask_id, 2.0, 2.0)
+    assert res["kind"].tolist() == [0, 0, 2, 0, 0, 0, 0, 0]
+    assert res["new_tokens"][2] == np.argmax(logits[2])
+
+
+def test_entropy_with_neginf_logits_equals_reduced_row():
+    """-inf logits are tokens of probability 0: the entropy equals that of the
+    row without them (torch's categorical entropy of the finite entries)."""
+    logits, tokens = _random_step(6, 200, 13, 0.0, -1)
+    hidden = np.random.default_rng(1).random(logits.shape) < 0.5
+    logits[hidden] = -np.inf
+    res = oracle.denoise_update(logits, tokens, [0, 6], 8, -1, 0.5, 0.0)
+    assert not res["undecidable"]
+    for r in range(6):
+        keep = torch.from_numpy(logits[r, ~hidden[r]]).double()
+        ref = torch.distributions.Categorical(logits=keep).entropy().item()
+        np.testing.assert_allclose(res["entropy"][r], ref, rtol=1e-12)

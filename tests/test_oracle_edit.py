@@ -109,14 +109,60 @@ def test_bf16_path_equals_float_path_on_rounded_values():
         np.testing.assert_array_equal(rb[k], rf[k])
 
 
-def test_row_subset_and_nonfinite_rejected():
+def test_row_subset_matches_full():
     prob = edit_problem(16, 50, torch.float32, seed=8)
     full = oracle.edit_decide(prob.logits.numpy(), prob.committed.numpy(), tau=0.1)
     sub = oracle.edit_decide(prob.logits.numpy(), prob.committed.numpy(), tau=0.1, rows=[3, 9])
     for r in (3, 9):
         assert sub["argmax"][r] == full["argmax"][r]
         assert sub["confidence"][r] == full["confidence"][r]
-    bad = prob.logits.numpy().copy()
-    bad[2, 7] = np.inf
-    with pytest.raises(RuntimeError, match="non-finite"):
-        oracle.edit_decide(bad, prob.committed.numpy(), tau=0.1)
+    assert not full["undecidable"] and not sub["undecidable"]
+
+
+@pytest.mark.parametrize("bad", ["nan", "posinf", "all_neginf"])
+def test_row_without_softmax_keeps_its_token(bad):
+    """Eq. 2 needs the softmax of the row. A row with a NaN or +inf logit, or
+    with every logit -inf, has none: its token stays (no edit, even at tau < 0),
+    its argmax is -1 and its confidence NaN, and every other row is decided as
+    if that row were absent."""
+    prob = edit_problem(12, 40, torch.float32, seed=9, peak_frac=1.0, peak_lo=30.0, peak_hi=40.0)
+    logits = prob.logits.numpy().copy()
+    committed = (prob.logits.argmax(dim=1).numpy() + 1) % 40   # every decidable row edits at tau < 0
+    if bad == "nan":
+        logits[5, 17] = np.nan
+    elif bad == "posinf":
+        logits[5, 3] = np.inf
+    else:
+        logits[5, :] = -np.inf
+    res = oracle.edit_decide(logits, committed, tau=-1.0)
+    assert res["undecidable"]
+    assert res["new_tokens"][5] == committed[5] and res["edit_mask"][5] == 0
+    assert res["argmax"][5] == -1 and np.isnan(res["confidence"][5])
+    others = np.array([r for r in range(12) if r != 5])
+    ref = oracle.edit_decide(logits[others], committed[others], tau=-1.0)
+    assert not ref["undecidable"]
+    for k in ("new_tokens", "edit_mask", "confidence", "argmax"):
+        np.testing.assert_array_equal(res[k][others], ref[k])
+    assert ref["edit_mask"].all()
+
+
+def test_neginf_logits_are_tokens_of_probability_zero():
+    """A -inf logit beside finite ones (a vocabulary mask) is a token of
+    probability 0: argmax and confidence equal torch's softmax over the finite
+    entries, i.e. the same row with those tokens removed."""
+    prob = edit_problem(20, 300, torch.float32, seed=10, peak_frac=0.5, peak_lo=1.0, peak_hi=6.0)
+    logits = prob.logits.numpy().copy()
+    g = np.random.default_rng(0)
+    hidden = g.random(logits.shape) < 0.3
+    hidden[:, 0] = True                       # the first token of every row is masked
+    logits[hidden] = -np.inf
+    res = oracle.edit_decide(logits, prob.committed.numpy(), tau=0.0)
+    assert not res["undecidable"]
+    p = torch.softmax(torch.from_numpy(logits).double(), dim=1)
+    np.testing.assert_array_equal(res["argmax"], p.argmax(dim=1).numpy())
+    np.testing.assert_allclose(res["confidence"], p.max(dim=1).values.numpy(), rtol=1e-13)
+    for r in range(3):
+        keep = np.flatnonzero(~hidden[r])
+        red = oracle.edit_decide(logits[r:r + 1, keep], np.array([0]), tau=0.0)
+        assert keep[red["argmax"][0]] == res["argmax"][r]
+        np.testing.assert_allclose(red["confidence"][0], res["confidence"][r], rtol=1e-14)
