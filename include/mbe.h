@@ -78,6 +78,7 @@ typedef enum { MBE_F32 = 0, MBE_BF16 = 1 } mbe_dtype;
 #define MBE_DEVERR_PAGE 0x4u          /* a block_table entry outside [0, num_pages) */
 #define MBE_DEVERR_CAPACITY 0x8u      /* work list larger than the workspace was sized for */
 #define MBE_DEVERR_PLAN 0x10u         /* mbe_window_attention_run found no plan for its parameters in the workspace */
+#define MBE_DEVERR_NONFINITE 0x20u    /* a logit row had no softmax (NaN / +inf logit, or every logit -inf) */
 
 /*
  * mbe_window_attention -- attention of one editing (or standard) pass.
@@ -168,6 +169,19 @@ mbe_status mbe_window_attention_run(const void* q, const void* k_win, const void
                                     void* workspace, size_t workspace_bytes, cudaStream_t stream);
 
 /*
+ * mbe_window_attention_plan_stats -- what the plan held in `workspace` (by
+ * mbe_window_attention or mbe_window_attention_plan) contains: the number of
+ * work units and the number of query slabs whose keys were cut into split-KV
+ * pieces (merged afterwards by log-sum-exp). Paper: Sec. 4.3 (mixed-shape
+ * forwards; here one device-side work list serves every shape). Synchronises
+ * `stream`, then copies 12 bytes of the workspace to the host.
+ * Errors: MBE_ERR_INVALID_ARG (null pointer, workspace smaller than 256 B),
+ * MBE_ERR_CUDA.
+ */
+mbe_status mbe_window_attention_plan_stats(const void* workspace, size_t workspace_bytes, int32_t* n_units,
+                                           int32_t* n_split_groups, cudaStream_t stream);
+
+/*
  * mbe_window_attention_noalloc -- mbe_window_attention for callers that cannot
  * allocate device memory. The paper has no counterpart: this is an interface
  * convenience of this library, not a step of the method.
@@ -184,8 +198,11 @@ mbe_status mbe_window_attention_run(const void* q, const void* k_win, const void
  *   - Shapes whose workspace (mbe_window_attention_workspace_size) exceeds
  *     64 MiB are rejected with MBE_ERR_WORKSPACE before anything is launched.
  *   - The first call on a device, with that device current, looks up the
- *     array's device address (cudaGetSymbolAddress); make that first call
- *     before any stream capture on that device.
+ *     array's device address (cudaGetSymbolAddress) and keeps it for the rest
+ *     of the process; make that first call before any stream capture on that
+ *     device. A cudaDeviceReset (or any other teardown of the device's primary
+ *     context) invalidates the kept address: do not call this entry point on
+ *     that device after such a reset.
  *   - All calls on a device share the one array and each call overwrites what
  *     the previous call left there. Calls whose kernels overlap on the GPU
  *     (for example on two streams without ordering between them) race and give
@@ -221,7 +238,10 @@ size_t mbe_window_attention_workspace_size(int32_t batch, int32_t num_q_heads, i
  * with tau_r = tau_per_row[r] if given, else tau.
  *
  *   logits     [rows, row_stride] of `dtype`, the first `vocab` entries of each
- *              row used; finite values (non-finite input gives unspecified output)
+ *              row used. A -inf logit is a token of probability 0 (a vocabulary
+ *              mask). A row with a NaN or +inf logit, or with every logit -inf,
+ *              has no softmax: it keeps its token (edit_mask 0), gets argmax -1
+ *              and confidence NaN, and the call sets MBE_DEVERR_NONFINITE.
  *   committed  int32 [rows]; new_tokens may alias committed
  *   editable_or_null uint8 [rows] (NULL: every row editable)
  *   new_tokens int32 [rows], edit_mask uint8 [rows], confidence fp32 [rows],
@@ -254,7 +274,10 @@ mbe_status mbe_edit_decide(const void* logits, mbe_dtype dtype, int64_t row_stri
  *                    3 if x != mask_id, editable, x_hat != x, c > omega_edit (Delta_t)
  *                    0 otherwise;  new_tokens[r] = kind ? x_hat : x
  * A block with masked rows of which none is in Gamma_t unmasks its most
- * confident masked row (lowest row on equal fp32 confidence).
+ * confident masked row (lowest row on equal fp32 confidence). Logit rows
+ * without a softmax are handled as in mbe_edit_decide (token kept, kind 0,
+ * argmax -1, confidence and entropy NaN, MBE_DEVERR_NONFINITE) and are never
+ * the forced row: a block whose masked rows all lack one unmasks none.
  *   entropy_or_null[r] = -sum_v p_v ln p_v (fp32)
  *   block_changed_or_null[s * max_blocks_per_seq + b] = 1 iff some row of block
  *     b changed token (0 for blocks past the sequence's rows); it is the
@@ -422,7 +445,9 @@ mbe_status mbe_block_mask_attention_bwd(const void* q, const void* k, const void
  *     chunks: 16 bytes per row and 256 tokens at most).
  * The logits are accumulated in fp32 on the tensor cores (bf16 products), so
  * they differ from exact dot products by fp32 rounding of the running sums;
- * decisions are taken on those fp32 values. hidden_dim must be a multiple of 8
+ * decisions are taken on those fp32 values. A row whose logits include NaN or
+ * +inf (from non-finite hidden or weight values) gets no decision, as in
+ * mbe_edit_decide (MBE_DEVERR_NONFINITE). hidden_dim must be a multiple of 8
  * and hidden / weight 16-byte aligned.
  * Errors: MBE_ERR_INVALID_ARG, MBE_ERR_WORKSPACE, MBE_ERR_UNSUPPORTED
  * (rows or vocab above 2^30), MBE_ERR_CUDA; a bounded wait that expires sets
@@ -530,6 +555,25 @@ void mbe_pass_loop_destroy(mbe_pass_loop* loop);
  * timeout bit was set, else MBE_ERR_DEVICE_CHECK; *flags_or_null receives the
  * MBE_DEVERR_* bits. */
 mbe_status mbe_get_device_error(cudaStream_t stream, uint32_t* flags_or_null);
+
+/* Default wall-clock limit of one bounded device wait: 1 s. */
+#define MBE_DEFAULT_WAIT_LIMIT_NS 1000000000ull
+
+/*
+ * mbe_set_wait_limit_ns -- failure-detection hook (no counterpart in the
+ * paper). Sets the wall-clock limit, in nanoseconds, of each bounded wait
+ * (an mbarrier phase wait inside the attention, LM-head and attention-
+ * backward kernels) of every kernel launched after the call, from any host
+ * thread, and returns the previous limit. The default is
+ * MBE_DEFAULT_WAIT_LIMIT_NS. A kernel whose wait runs out sets
+ * MBE_DEVERR_TIMEOUT, lets the copies and tensor-core operations it already
+ * issued finish, releases its tensor memory and returns, so the context stays
+ * usable; the outputs of that call are incomplete. With a limit of 0 every
+ * wait that is not complete at its first try runs out, which lets a test drive
+ * that path without any fault. The waits of the abort path itself always keep
+ * the default limit. Lowering the limit is meant for tests only.
+ */
+uint64_t mbe_set_wait_limit_ns(uint64_t limit_ns);
 
 /* Host-thread-local description of the last CUDA runtime failure the library
  * saw (the call site, the error name and message); useful after MBE_ERR_CUDA. */

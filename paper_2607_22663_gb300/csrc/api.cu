@@ -1,11 +1,14 @@
 // Status strings, version, the last CUDA error and the device error word query of libmbe.
+#include <atomic>
 #include <cstdio>
 #include "common.cuh"
 
 namespace mbe {
 namespace {
 thread_local char g_last_error[256] = "no CUDA error recorded";
+std::atomic<uint64_t> g_wait_limit_ns{MBE_DEFAULT_WAIT_LIMIT_NS};
 }
+uint64_t wait_limit_ns() { return g_wait_limit_ns.load(std::memory_order_relaxed); }
 void record_cuda_error(cudaError_t e, const char* where) {
   snprintf(g_last_error, sizeof(g_last_error), "%s: %s (%s)", where, cudaGetErrorName(e), cudaGetErrorString(e));
 }
@@ -42,3 +45,7 @@ extern "C" const char* mbe_status_string(mbe_status status) {
 }
 
 extern "C" int32_t mbe_version(void) { return 100; }
+
+extern "C" uint64_t mbe_set_wait_limit_ns(uint64_t limit_ns) {
+  return mbe::g_wait_limit_ns.exchange(limit_ns, std::memory_order_relaxed);
+}

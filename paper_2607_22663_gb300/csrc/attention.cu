@@ -10,7 +10,7 @@
 //     dynamic scheduling.
 //  2. attn_kernel (persistent, one CTA per SM, 12 warps):
 //       warp 0      TMA producer: Q slab once per unit, then K/V tiles of 128
-//                   keys into a 2-stage ring (paged prefix via a 4-D tensor
+//                   keys into a ring of K and V tiles (paged prefix via a 4-D tensor
 //                   map with the page id as a coordinate; window via 3-D)
 //       warp 1      MMA issuer: S_i = Q_i K^T (SS form) and O_i += P_i V
 //                   (TS form, P read from TMEM), tcgen05, accumulators in TMEM
@@ -365,6 +365,7 @@ struct AttnParams {
   // is set iff query block qb attends to key block kb; block_log2 = log2(block_size)
   const uint32_t* mask;
   int mask_rows, mask_words, block_log2;
+  uint64_t wait_ns;  // limit of the ordinary mbarrier waits
 };
 
 // Block-mask mode: does any query block of packed rows [row0, row0 + 256) see a
@@ -440,6 +441,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ uint32_t tmem_base_s;
   __shared__ int abort_s;
   volatile int* abort_flag = &abort_s;
+  const uint64_t wait_ns = p.wait_ns;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t sbase = smem_u32(smem);
@@ -498,7 +500,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const bool done = uidx >= n_units;
       const int uslot = u_it & 1;
       if (u_it >= 2) {
-        ok = __all_sync(kAll, mbar_wait(bar(bars.u_empty[uslot]), ((u_it >> 1) - 1) & 1, abort_flag));
+        ok = __all_sync(kAll, mbar_wait(bar(bars.u_empty[uslot]), ((u_it >> 1) - 1) & 1, abort_flag, wait_ns));
         if (!ok) break;
       }
       WorkUnit wu;
@@ -544,7 +546,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int n_qt = (W * p.G - wu.row0) > kTileRows ? 2 : 1;
       const int cu = p.cu_window[wu.seq];
       if (q_loads >= 1) {
-        ok = __all_sync(kAll, mbar_wait(bar(bars.q_empty), (q_loads - 1) & 1, abort_flag));
+        ok = __all_sync(kAll, mbar_wait(bar(bars.q_empty), (q_loads - 1) & 1, abort_flag, wait_ns));
         if (!ok) break;
       }
       if (lane == 0) {
@@ -599,7 +601,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int kv = 0; kv < 2; ++kv, ++item) {
           const uint32_t sl = slot_of(item), use = item / S::kSlots;
           if (use >= 1) {
-            ok = __all_sync(kAll, mbar_wait(bar(bars.empty[sl]), (use - 1) & 1, abort_flag));
+            ok = __all_sync(kAll, mbar_wait(bar(bars.empty[sl]), (use - 1) & 1, abort_flag, wait_ns));
             if (!ok) break;
           }
           const uint32_t dst = sbase + S::kRing + sl * S::kItem;
@@ -627,7 +629,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (!ok && lane == 0) {
       *abort_flag = 1;
       atomicOr(&g_error_word, MBE_DEVERR_TIMEOUT);
-      // let the copies already issued land before the CTA can exit
+    }
+    // The copies already issued land before the CTA can exit, also when another
+    // role aborted after this loop ended (without an abort they have all been
+    // consumed, and these waits return at once).
+    if (lane == 0) {
       const int zero = 0;
       for (uint32_t n = (item >= S::kSlots ? item - S::kSlots : 0); n < item; ++n)
         mbar_wait(bar(bars.full[slot_of(n)]), (n / S::kSlots) & 1, &zero);
@@ -642,7 +648,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t p_cnt[2] = {0, 0}, o_cnt[2] = {0, 0};
       bool ok = true;
       auto item_addr = [&](uint32_t n) { return sbase + S::kRing + (n % S::kSlots) * S::kItem; };
-      auto wait_item = [&](uint32_t n) { return mbar_wait(bar(bars.full[n % S::kSlots]), (n / S::kSlots) & 1, abort_flag); };
+      auto wait_item = [&](uint32_t n) { return mbar_wait(bar(bars.full[n % S::kSlots]), (n / S::kSlots) & 1, abort_flag, wait_ns); };
       auto release_item = [&](uint32_t n) { umma_commit(bar(bars.empty[n % S::kSlots])); };
       auto issue_qk = [&](int i, uint32_t ka) {
         const uint32_t qa = sbase + S::kQ + i * S::kQTile;
@@ -661,7 +667,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       for (;;) {
         const int slot = u_it & 1;
-        if (!mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag)) { ok = false; break; }
+        if (!mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag, wait_ns)) { ok = false; break; }
         const WorkUnit wu = unit_ring[slot];
         int n_t = wu.tile_end - wu.tile_begin;
         if constexpr (kMask) {
@@ -673,7 +679,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (wu.seq < 0) break;
         const int W = wu.window_mode & 0x3FFFFFFF;
         const int n_qt = (W * p.G - wu.row0) > kTileRows ? 2 : 1;
-        if (!mbar_wait(bar(bars.q_full), q_it & 1, abort_flag)) { ok = false; break; }
+        if (!mbar_wait(bar(bars.q_full), q_it & 1, abort_flag, wait_ns)) { ok = false; break; }
         ++q_it;
         // items of tile ki: K = 2 ki, V = 2 ki + 1
         if (!wait_item(2 * kv_it)) { ok = false; break; }
@@ -688,9 +694,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t ki = kv_it + j;
           if (!wait_item(2 * ki + 1)) { ok = false; break; }
           for (int i = 0; i < n_qt; ++i) {
-            if (!mbar_wait(bar(bars.p_full[i]), p_cnt[i] & 1, abort_flag)) { ok = false; break; }
+            if (!mbar_wait(bar(bars.p_full[i]), p_cnt[i] & 1, abort_flag, wait_ns)) { ok = false; break; }
             ++p_cnt[i];
-            if (j == 0 && o_cnt[i] > 0 && !mbar_wait(bar(bars.o_empty[i]), (o_cnt[i] - 1) & 1, abort_flag)) {
+            if (j == 0 && o_cnt[i] > 0 && !mbar_wait(bar(bars.o_empty[i]), (o_cnt[i] - 1) & 1, abort_flag, wait_ns)) {
               ok = false;
               break;
             }
@@ -738,7 +744,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok = true;
     for (;;) {
       const int slot = u_it & 1;
-      ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag));
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag, wait_ns));
       if (!ok) break;
       const WorkUnit wu = unit_ring[slot];
       // block-mask mode keeps the ring slot (and its tile bitmask) until its tiles are done
@@ -792,7 +798,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           t = wu.tile_begin + j;
         }
         const uint32_t ki = kv_it + j;
-        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.s_full[wg]), s_cnt & 1, abort_flag));
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.s_full[wg]), s_cnt & 1, abort_flag, wait_ns));
         if (!ok) break;
         ++s_cnt;
         tc_fence_after();
@@ -934,7 +940,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int v0 = (t == nP - 1) ? P % kTileKeys : (t - nP == (W - 1) / kTileKeys ? W % kTileKeys : 0);
         if (wg == 0 && v0 != 0) {
           const uint32_t nv = 2 * ki + 1;  // the V item of this tile
-          ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.full[nv % S::kSlots]), (nv / S::kSlots) & 1, abort_flag));
+          ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.full[nv % S::kSlots]), (nv / S::kSlots) & 1, abort_flag, wait_ns));
           if (!ok) break;
           uint8_t* vt = smem + S::kRing + (nv % S::kSlots) * S::kItem;
           const int per_row = S::kHalves * 8;  // 16-byte chunks per key row
@@ -953,7 +959,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       kv_it += n_t;
       if (kMask) release_unit();
       // epilogue: O_i is complete once o_full fires
-      ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.o_full[wg]), o_cnt & 1, abort_flag));
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.o_full[wg]), o_cnt & 1, abort_flag, wait_ns));
       if (!ok) break;
       ++o_cnt;
       tc_fence_after();
@@ -1238,6 +1244,7 @@ mbe_status run(const void* q, const void* k_win, const void* v_win, const void* 
   ap.mask_words = mask.words;
   ap.block_log2 = 0;
   while ((1 << ap.block_log2) < block_size) ++ap.block_log2;
+  ap.wait_ns = wait_limit_ns();
   attn_kernel<D, kMask><<<di->num_sms, kThreads, Smem<D>::kBytes, stream>>>(tq, tkw, tvw, tkc, tvc, ap);
   if (launch_status("attn_kernel launch") != MBE_OK) return MBE_ERR_CUDA;
   MergeParams mp{sig, batch, total_q_tokens, hdr, reinterpret_cast<const MergeGroup*>(ws + L.groups), ap.part_o,
@@ -1385,6 +1392,20 @@ extern "C" mbe_status mbe_window_attention_run(const void* q, const void* k_win,
                         window_len, cu_window, mask_mode, batch, total_q_tokens, num_q_heads, num_kv_heads, head_dim,
                         block_size, page_size, max_window, max_prefix, softmax_scale, out, lse_or_null, workspace,
                         workspace_bytes, false, stream);
+}
+
+extern "C" mbe_status mbe_window_attention_plan_stats(const void* workspace, size_t workspace_bytes, int32_t* n_units,
+                                                      int32_t* n_split_groups, cudaStream_t stream) {
+  if (!workspace || workspace_bytes < sizeof(Header) || !n_units || !n_split_groups) return MBE_ERR_INVALID_ARG;
+  int32_t h[3] = {0, 0, 0};
+  if (cudaMemcpyAsync(h, workspace, sizeof(h), cudaMemcpyDeviceToHost, stream) != cudaSuccess ||
+      cudaStreamSynchronize(stream) != cudaSuccess) {
+    record_cuda_error(cudaGetLastError(), "mbe_window_attention_plan_stats");
+    return MBE_ERR_CUDA;
+  }
+  *n_units = h[1];
+  *n_split_groups = h[2];
+  return MBE_OK;
 }
 
 // ------------------------------------------------------------------ no-allocation variant

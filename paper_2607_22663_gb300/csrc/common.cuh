@@ -25,6 +25,10 @@ uint32_t refresh_take_error();
 uint32_t lm_head_take_error();
 uint32_t train_take_error();
 
+// Wall-clock limit (ns) of the ordinary mbarrier waits of kernels launched
+// from now on (mbe_set_wait_limit_ns; 1 s by default).
+uint64_t wait_limit_ns();
+
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 // Remembers (per host thread) the last CUDA failure seen by the library.

@@ -32,24 +32,23 @@ __device__ __forceinline__ void absorb_vector(Stats& a, const uint4& v, int col0
   constexpr int N = Vec<T>::N;
   float x[N];
   Vec<T>::unpack(v, x);
-  const float lm = vec_max(x);
-  if (lm > a.m) {  // rare after the first vectors; a.m starts at -inf
-    if (a.idx < 0) {
-      a.s = 0.f;
-      a.t = 0.f;
-      a.m = lm;
-    } else {
-      rebase(a, lm);
-    }
-    a.idx = col0 + first_index(x, lm);
+  const float lm = vec_max(x);  // NaN if some element is NaN
+  if (unusable(lm)) {
+    a.s = nan_f32();
+    return;
   }
-  // u = l log2e - m log2e and e = 2^u, two elements per packed FMA / add
+  if (lm > a.m) raise_max(a, lm, col0 + first_index(x, lm));  // rare after the first vectors
+  // u = l log2e - m log2e (clamped below, so that -inf logits add 0 to t) and
+  // e = 2^u, two elements per packed FMA / add
+  const float mr = ref_max(a);
   const float2 L = make_float2(kLog2e, kLog2e);
-  const float2 ms = make_float2(-a.m * kLog2e, -a.m * kLog2e);
+  const float2 ms = make_float2(-mr * kLog2e, -mr * kLog2e);
   float2 s = make_float2(0.f, 0.f), t = make_float2(0.f, 0.f);
 #pragma unroll
   for (int k = 0; k < N; k += 2) {
-    const float2 u = ffma2(make_float2(x[k], x[k + 1]), L, ms);
+    float2 u = ffma2(make_float2(x[k], x[k + 1]), L, ms);
+    u.x = fmaxf(u.x, kMinU);
+    u.y = fmaxf(u.y, kMinU);
     const float2 e = make_float2(ex2(u.x), ex2(u.y));
     s = fadd2(s, e);
     t = ffma2(e, u, t);
@@ -107,8 +106,19 @@ __global__ void __launch_bounds__(kThreads) denoise_row_kernel(const T* __restri
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) merge(b, shfl_xor(b, off));
   if (lane != 0) return;
-  const float c = 1.0f / b.s;
   const int32_t cur = a.tokens[row];
+  if (undecidable(b)) {
+    // no softmax (a NaN or +inf logit, or every logit -inf): the token stays,
+    // and the row is never the forced one of its block (argmax -1)
+    atomicOr(&g_error_word, MBE_DEVERR_NONFINITE);
+    a.new_tokens[row] = cur;
+    a.kind[row] = 0;
+    a.confidence[row] = nan_f32();
+    a.argmax[row] = -1;
+    if (a.entropy) a.entropy[row] = nan_f32();
+    return;
+  }
+  const float c = 1.0f / b.s;
   uint8_t k = 0;
   if (cur == a.mask_id) {
     if (c > a.omega_mask) k = 1;
@@ -149,6 +159,7 @@ __global__ void __launch_bounds__(256) denoise_block_kernel(const int32_t* __res
       if (tokens[r] != mask_id) continue;
       any_masked = true;
       if (kind[r] == 1) any_unmasked = true;
+      if (argmax[r] < 0) continue;  // a row without a softmax is never forced
       const float c = confidence[r];
       if (c > best_c || (c == best_c && r < best_r)) {
         best_c = c;
@@ -166,7 +177,8 @@ __global__ void __launch_bounds__(256) denoise_block_kernel(const int32_t* __res
         best_r = orr;
       }
     }
-    if (any_masked && !any_unmasked && lane == 0) {
+    // best_r stays 0x7FFFFFFF when no masked row of the block has a softmax
+    if (any_masked && !any_unmasked && best_r != 0x7FFFFFFF && lane == 0) {
       kind[best_r] = 2;
       new_tokens[best_r] = argmax[best_r];
     }

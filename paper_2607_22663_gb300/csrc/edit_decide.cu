@@ -18,25 +18,38 @@ namespace {
 
 using namespace rows;
 
+// Online (max, sum, argmax) state of a row. Empty: m = -inf, s = 0, idx = -1.
+// A NaN or +inf logit makes s NaN, which every later step keeps (s is only
+// scaled and added to), so the row's final s tells that it has no softmax.
 struct Triple {
   float m;  // running maximum
   float s;  // sum of exp(l - m)
-  int idx;  // lowest index attaining m
+  int idx;  // lowest index attaining m; -1 while no element above -inf was seen
 };
 
-// Adds one element (or a vector's maximum first) to the triple.
-__device__ __forceinline__ void absorb_max(Triple& t, float lm, int li) {
+// Makes lm (index li) the running maximum if it is larger (an empty state has
+// m = -inf: its s, 0 or NaN, is scaled by ex2(-inf) = 0 and stays 0 or NaN).
+__device__ __forceinline__ void raise_max(Triple& t, float lm, int li) {
   if (lm > t.m) {
-    t.s *= ex2((t.m - lm) * kLog2e);  // m = -inf gives ex2(-inf) = 0
+    t.s *= ex2((t.m - lm) * kLog2e);
     t.m = lm;
     t.idx = li;
   }
 }
 
+// Exponent reference: 0 while empty, so that -inf logits give ex2(-inf) = 0.
+__device__ __forceinline__ float ref_max(const Triple& t) { return t.idx < 0 ? 0.f : t.m; }
+
+// An empty side contributes its s (0, or NaN) and nothing else.
 __device__ __forceinline__ void merge(Triple& a, const Triple& b) {
-  if (b.idx < 0) return;  // b saw no element
+  if (b.idx < 0) {
+    a.s += b.s;
+    return;
+  }
   if (a.idx < 0) {
+    const float z = a.s;
     a = b;
+    a.s += z;
     return;
   }
   if (b.m > a.m) {
@@ -64,15 +77,16 @@ __device__ __forceinline__ void absorb_vector(Triple& t, const uint4& v, int col
   constexpr int N = Vec<T>::N;
   float x[N];
   Vec<T>::unpack(v, x);
-  float lm = x[0];
-  int li = 0;
-#pragma unroll
-  for (int k = 1; k < N; ++k)
-    if (x[k] > lm) { lm = x[k]; li = k; }
-  absorb_max(t, lm, col0 + li);
+  const float lm = vec_max(x);  // NaN if some element is NaN
+  if (unusable(lm)) {
+    t.s = nan_f32();
+    return;
+  }
+  if (lm > t.m) raise_max(t, lm, col0 + first_index(x, lm));
+  const float mr = ref_max(t);
   float acc = 0.f;
 #pragma unroll
-  for (int k = 0; k < N; ++k) acc += ex2((x[k] - t.m) * kLog2e);
+  for (int k = 0; k < N; ++k) acc += ex2((x[k] - mr) * kLog2e);
   t.s += acc;
 }
 
@@ -107,8 +121,12 @@ __global__ void __launch_bounds__(kThreads) edit_decide_kernel(const T* __restri
   }
   for (int c = scalar_from + threadIdx.x; c < vocab; c += kThreads) {
     const float x = to_f32<T>(rp[c]);
-    absorb_max(t, x, c);
-    t.s += ex2((x - t.m) * kLog2e);
+    if (unusable(x)) {
+      t.s = nan_f32();
+    } else {
+      raise_max(t, x, c);
+      t.s += ex2((x - ref_max(t)) * kLog2e);
+    }
   }
   // warp merge
 #pragma unroll
@@ -128,8 +146,17 @@ __global__ void __launch_bounds__(kThreads) edit_decide_kernel(const T* __restri
       merge(a, o);
     }
     if (lane == 0) {
-      const float c = 1.0f / a.s;
       const int32_t x = committed[row];
+      if (a.idx < 0 || !(a.s > 0.f)) {
+        // no softmax (a NaN or +inf logit, or every logit -inf): no decision
+        atomicOr(&g_error_word, MBE_DEVERR_NONFINITE);
+        new_tokens[row] = x;
+        edit_mask[row] = 0;
+        confidence[row] = nan_f32();
+        if (argmax_out) argmax_out[row] = -1;
+        return;
+      }
+      const float c = 1.0f / a.s;
       const float tr = tau_per_row ? tau_per_row[row] : tau;
       const bool can = editable ? (editable[row] != 0) : true;
       const bool ed = can && (a.idx != x) && (c > tr);

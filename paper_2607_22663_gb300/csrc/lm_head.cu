@@ -56,6 +56,7 @@ struct Params {
   int tpu;  // tiles per unit
   int n_m, n_chunks, n_units, n_kb;
   Partial* part;  // [rows, n_chunks]
+  uint64_t wait_ns;  // limit of the ordinary mbarrier waits
 };
 
 struct Bars {
@@ -68,18 +69,12 @@ __device__ __forceinline__ void absorb32(Stats& a, const float (&x)[32], int col
 #pragma unroll
   for (int k = 3; k < 31; k += 2) cm = fmax3(cm, x[k], x[k + 1]);
   cm = fmaxf(cm, x[31]);
-  if (cm > a.m) {
-    if (a.idx < 0) {
-      a.s = 0.f;
-      a.t = 0.f;
-      a.m = cm;
-    } else {
-      rebase(a, cm);
-    }
-    a.idx = col0 + first_index(x, cm);
-  }
+  // a NaN logit is skipped by the maximum but gives e = NaN below, and a +inf
+  // one becomes the maximum with u = NaN for itself: s turns NaN either way
+  if (cm > a.m) raise_max(a, cm, col0 + first_index(x, cm));
+  const float mr = ref_max(a);
   const float2 L = make_float2(kLog2e, kLog2e);
-  const float2 ms = make_float2(-a.m * kLog2e, -a.m * kLog2e);
+  const float2 ms = make_float2(-mr * kLog2e, -mr * kLog2e);
   float2 s = make_float2(0.f, 0.f), t = make_float2(0.f, 0.f);
 #pragma unroll
   for (int k = 0; k < 32; k += 2) {
@@ -101,6 +96,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ uint32_t tmem_base_s;
   __shared__ int abort_s;
   volatile int* abort_flag = &abort_s;
+  const uint64_t wait_ns = p.wait_ns;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t sbase = smem_u32(smem);
   auto bar = [](uint64_t& b) { return smem_u32(&b); };
@@ -142,7 +138,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int nt = chunk * p.tpu + t;
           for (int kb = 0; kb < p.n_kb; ++kb, ++it) {
             const uint32_t s = it % kStages;
-            if (it >= kStages && !mbar_wait(bar(bars.empty[s]), ((it / kStages) - 1) & 1, abort_flag)) {
+            if (it >= kStages && !mbar_wait(bar(bars.empty[s]), ((it / kStages) - 1) & 1, abort_flag, wait_ns)) {
               ok = false;
               break;
             }
@@ -156,11 +152,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) {
         *abort_flag = 1;
         atomicOr(&g_error_word, MBE_DEVERR_TIMEOUT);
-        // let the copies already issued land before the CTA can exit
-        const int zero = 0;
-        for (uint32_t n = (it >= kStages ? it - kStages : 0); n < it; ++n)
-          mbar_wait(bar(bars.full[n % kStages]), (n / kStages) & 1, &zero);
       }
+      // The copies already issued land before the CTA can exit, also when another
+      // role aborted after this loop ended (they return at once otherwise).
+      const int zero = 0;
+      for (uint32_t n = (it >= kStages ? it - kStages : 0); n < it; ++n)
+        mbar_wait(bar(bars.full[n % kStages]), (n / kStages) & 1, &zero);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
@@ -173,7 +170,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int nt_count = tiles_of(chunk);
         for (int t = 0; t < nt_count && ok; ++t, ++tile) {
           const uint32_t acc = tile & 1;
-          if (tile >= 2 && !mbar_wait(bar(bars.acc_empty[acc]), ((tile >> 1) - 1) & 1, abort_flag)) {
+          if (tile >= 2 && !mbar_wait(bar(bars.acc_empty[acc]), ((tile >> 1) - 1) & 1, abort_flag, wait_ns)) {
             ok = false;
             break;
           }
@@ -181,7 +178,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t d_tmem = tmem + acc * kBN;
           for (int kb = 0; kb < p.n_kb; ++kb, ++it) {
             const uint32_t s = it % kStages;
-            if (!mbar_wait(bar(bars.full[s]), (it / kStages) & 1, abort_flag)) {
+            if (!mbar_wait(bar(bars.full[s]), (it / kStages) & 1, abort_flag, wait_ns)) {
               ok = false;
               break;
             }
@@ -219,7 +216,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       Stats st{__int_as_float(0xff800000u), 0.f, 0.f, -1};
       for (int t = 0; t < nt_count; ++t, ++tile) {
         const uint32_t acc = tile & 1;
-        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.acc_full[acc]), (tile >> 1) & 1, abort_flag));
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.acc_full[acc]), (tile >> 1) & 1, abort_flag, wait_ns));
         if (!ok) break;
         tc_fence_after();
         const int col0 = (chunk * p.tpu + t) * kBN;
@@ -275,9 +272,19 @@ __global__ void __launch_bounds__(256) lm_head_decide_kernel(const Partial* __re
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) merge(st, shfl_xor(st, off));
   if (lane != 0) return;
+  const int32_t cur = committed[row];
+  if (undecidable(st)) {
+    // no softmax (the projection produced a NaN or +inf logit): no decision
+    atomicOr(&g_error_word, MBE_DEVERR_NONFINITE);
+    new_tokens[row] = cur;
+    edit_mask[row] = 0;
+    confidence[row] = nan_f32();
+    if (argmax_out) argmax_out[row] = -1;
+    if (entropy) entropy[row] = nan_f32();
+    return;
+  }
   const float c = 1.0f / st.s;
   const float tr = tau_per_row ? tau_per_row[row] : tau;
-  const int32_t cur = committed[row];
   const bool ed = (editable == nullptr || editable[row] != 0) && st.idx != cur && c > tr;
   new_tokens[row] = ed ? st.idx : cur;
   edit_mask[row] = ed ? 1 : 0;
@@ -377,6 +384,7 @@ extern "C" mbe_status mbe_lm_head_edit_decide(const void* hidden, const void* we
   p.n_units = p.n_m * p.n_chunks;
   p.n_kb = (hidden_dim + kBK - 1) / kBK;
   p.part = static_cast<Partial*>(workspace);
+  p.wait_ns = wait_limit_ns();
   const int grid = std::min(p.n_units, ds->num_sms);
   lm_head_kernel<<<grid, kThreads, kSmemBytes, stream>>>(th, tw, p);
   mbe_status st = launch_status("lm_head_kernel");

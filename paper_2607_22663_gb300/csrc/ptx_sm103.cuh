@@ -2,16 +2,20 @@
 // mbarriers, TMA tensor loads, and the tcgen05 tensor-core path (TMEM
 // allocation, MMA issue/commit, TMEM loads/stores, ordering fences).
 //
-// Every wait on an mbarrier is bounded: after kWaitLimitNs of wall time (or
-// once another role of the CTA has raised the abort flag) the wait returns
-// false and the caller records an error instead of spinning forever.
+// Every wait on an mbarrier is bounded: after a wall-clock limit (1 s unless
+// the caller lowered it with mbe_set_wait_limit_ns, or once another role of
+// the CTA has raised the abort flag) the wait returns false and the caller
+// records an error instead of spinning forever.
 #pragma once
 #include <cstdint>
 #include <cuda.h>
 
 namespace mbe {
 
-// Wall-clock bound on any single mbarrier wait (nanoseconds).
+// Wall-clock bound on any single mbarrier wait (nanoseconds). Kernels take the
+// limit of their ordinary waits from their launch parameters (this value
+// unless lowered for a test); the waits of an abort path, which let copies and
+// MMAs already issued finish, always use this one.
 constexpr uint64_t kWaitLimitNs = 1000ull * 1000ull * 1000ull;  // 1 s
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -49,16 +53,31 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Waits for the phase with the given parity to complete. Returns false if the
-// wall-clock limit passed or *abort became non-zero first.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const volatile int* abort) {
+// Non-blocking test for the completion of the phase with the given parity.
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Waits for the phase with the given parity to complete. Returns false if
+// limit_ns of wall time passed or *abort became non-zero first; with a limit
+// of 0 the phase must already be complete (one non-blocking test).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const volatile int* abort,
+                                          uint64_t limit_ns = kWaitLimitNs) {
+  if (limit_ns == 0) return mbar_test_wait(bar, parity);
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((it & 63u) == 0) {
       if (*abort) return false;
-      if (global_timer_ns() - t0 > kWaitLimitNs) return false;
+      if (global_timer_ns() - t0 > limit_ns) return false;
     }
   }
 }

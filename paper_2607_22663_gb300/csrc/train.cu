@@ -125,6 +125,7 @@ struct Params {
   int mask_rows, mask_words, block_log2;
   int batch, total_tokens, Hq, Hkv, G, lgG;
   float scale, scale_log2;
+  uint64_t wait_ns;  // limit of the ordinary mbarrier waits
 };
 
 struct Unit {
@@ -236,6 +237,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ uint32_t tmem_base_s;
   __shared__ int abort_s;
   volatile int* abort_flag = &abort_s;
+  const uint64_t wait_ns = p.wait_ns;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t sbase = smem_u32(smem);
   auto bar = [](uint64_t& b) { return smem_u32(&b); };
@@ -289,7 +291,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (;;) {
       const int slot = u_it & 1;
       if (u_it >= 2) {
-        ok = __all_sync(kAll, mbar_wait(bar(bars.u_empty[slot]), ((u_it >> 1) - 1) & 1, abort_flag));
+        ok = __all_sync(kAll, mbar_wait(bar(bars.u_empty[slot]), ((u_it >> 1) - 1) & 1, abort_flag, wait_ns));
         if (!ok) break;
       }
       bool done;
@@ -300,7 +302,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const volatile uint32_t* bits = ring_bits[slot];
       if (popc_bits(bits) == 0) continue;
       if (kv_loads >= 1) {
-        ok = __all_sync(kAll, mbar_wait(bar(bars.kv_empty), (kv_loads - 1) & 1, abort_flag));
+        ok = __all_sync(kAll, mbar_wait(bar(bars.kv_empty), (kv_loads - 1) & 1, abort_flag, wait_ns));
         if (!ok) break;
       }
       if (lane == 0) {
@@ -317,7 +319,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int tok = un.cu + ((i * kTile) >> p.lgG);
         const uint32_t sq = q_loads % 3, sd = do_loads & 1;
         if (q_loads >= 3) {
-          ok = __all_sync(kAll, mbar_wait(bar(bars.q_empty[sq]), ((q_loads / 3) - 1) & 1, abort_flag));
+          ok = __all_sync(kAll, mbar_wait(bar(bars.q_empty[sq]), ((q_loads / 3) - 1) & 1, abort_flag, wait_ns));
           if (!ok) break;
         }
         if (lane == 0) {
@@ -328,7 +330,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         ++q_loads;
         if (do_loads >= 2) {
-          ok = __all_sync(kAll, mbar_wait(bar(bars.do_empty[sd]), ((do_loads >> 1) - 1) & 1, abort_flag));
+          ok = __all_sync(kAll, mbar_wait(bar(bars.do_empty[sd]), ((do_loads >> 1) - 1) & 1, abort_flag, wait_ns));
           if (!ok) break;
         }
         if (lane == 0) {
@@ -356,7 +358,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int b = 0; b < nqb; ++b)
             if (mask_bit(p, un.seq, qb0 + b, kb_first + lane)) kvis |= 1u << b;
         if (cols >= 1) {
-          ok = __all_sync(kAll, mbar_wait(bar(bars.col_empty), (cols - 1) & 1, abort_flag));
+          ok = __all_sync(kAll, mbar_wait(bar(bars.col_empty), (cols - 1) & 1, abort_flag, wait_ns));
           if (!ok) break;
         }
 #pragma unroll
@@ -374,7 +376,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (!ok && lane == 0) {
       *abort_flag = 1;
       atomicOr(&g_error_word, MBE_DEVERR_TIMEOUT);
-      // let the copies already issued land before the CTA can exit
+    }
+    // The copies already issued land before the CTA can exit, also when another
+    // role aborted after this loop ended (they return at once otherwise).
+    if (lane == 0) {
       const int zero = 0;
       if (kv_loads >= 1) mbar_wait(bar(bars.kv_full), (kv_loads - 1) & 1, &zero);
       for (uint32_t n = (q_loads >= 3 ? q_loads - 3 : 0); n < q_loads; ++n)
@@ -391,7 +396,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       // S^T = K Q_t^T into the S region (issued after dV of tile t - 1, the last reader there)
       auto issue_s = [&](uint32_t t) {
-        if (!mbar_wait(bar(bars.q_full[t % 3]), (t / 3) & 1, abort_flag)) return false;
+        if (!mbar_wait(bar(bars.q_full[t % 3]), (t / 3) & 1, abort_flag, wait_ns)) return false;
         tc_fence_after();
         const uint32_t qa = sbase + kRingA + (t % 3) * kTileBytes;
 #pragma unroll
@@ -407,7 +412,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       // dP^T = V dO_t^T into the dP region (issued after dK of tile t - 1, the last reader there)
       auto issue_dp = [&](uint32_t t) {
-        if (!mbar_wait(bar(bars.do_full[t & 1]), (t >> 1) & 1, abort_flag)) return false;
+        if (!mbar_wait(bar(bars.do_full[t & 1]), (t >> 1) & 1, abort_flag, wait_ns)) return false;
         tc_fence_after();
         const uint32_t da = sbase + kRingB + (t & 1) * kTileBytes;
 #pragma unroll
@@ -423,22 +428,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       for (;;) {
         const int slot = u_it & 1;
-        if (!mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag)) { ok = false; break; }
+        if (!mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag, wait_ns)) { ok = false; break; }
         const Unit un = ring[slot];
         const int n_q = popc_bits(ring_bits[slot]);
         mbar_arrive(bar(bars.u_empty[slot]));
         ++u_it;
         if (un.seq < 0) break;
         if (n_q == 0) continue;
-        if (!mbar_wait(bar(bars.kv_full), units & 1, abort_flag)) { ok = false; break; }
+        if (!mbar_wait(bar(bars.kv_full), units & 1, abort_flag, wait_ns)) { ok = false; break; }
         if (!issue_s(tiles) || !issue_dp(tiles)) { ok = false; break; }
         for (int j = 0; j < n_q; ++j) {
           const uint32_t t = tiles + j;
           const uint32_t qa = sbase + kRingA + (t % 3) * kTileBytes, da = sbase + kRingB + (t & 1) * kTileBytes;
           // dV as soon as P^T is in TMEM (over S^T), then the next tile's S^T; both run
           // while the compute warps form dS^T
-          if (!mbar_wait(bar(bars.pt_full), t & 1, abort_flag)) { ok = false; break; }
-          if (j == 0 && units >= 1 && !mbar_wait(bar(bars.acc_empty), (units - 1) & 1, abort_flag)) {
+          if (!mbar_wait(bar(bars.pt_full), t & 1, abort_flag, wait_ns)) { ok = false; break; }
+          if (j == 0 && units >= 1 && !mbar_wait(bar(bars.acc_empty), (units - 1) & 1, abort_flag, wait_ns)) {
             ok = false;
             break;
           }
@@ -451,7 +456,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           umma_commit(bar(bars.do_empty[t & 1]));
           if (j + 1 < n_q && !issue_s(t + 1)) { ok = false; break; }
           // dK once dS^T is in TMEM (over dP^T), then the next tile's dP^T
-          if (!mbar_wait(bar(bars.ds_full), t & 1, abort_flag)) { ok = false; break; }
+          if (!mbar_wait(bar(bars.ds_full), t & 1, abort_flag, wait_ns)) { ok = false; break; }
           tc_fence_after();
 #pragma unroll
           for (int kk = 0; kk < kTile / 16; ++kk)
@@ -485,7 +490,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok = true;
     for (;;) {
       const int slot = u_it & 1;
-      ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag));
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag, wait_ns));
       if (!ok) break;
       const Unit un = ring[slot];
       const volatile uint32_t* bits = ring_bits[slot];
@@ -511,7 +516,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       const int kb_rel = (key >> p.block_log2) - ((un.t * kTile) >> p.block_log2);
       for (int i = next_bit(bits, -1); i >= 0; i = next_bit(bits, i), ++tiles) {
-        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.col_full), tiles & 1, abort_flag));
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.col_full), tiles & 1, abort_flag, wait_ns));
         if (!ok) break;
         const int qb0 = qblock0(p, i), nqb = qblock_count(p, un, i);
         const uint32_t all = nqb >= 32 ? 0xFFFFFFFFu : ((1u << nqb) - 1u);
@@ -520,7 +525,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // TMEM loads are warp-wide: the warp skips them only if no lane needs them
         const bool any_vis = __any_sync(0xffffffffu, qvis != 0u);
         const bool every = __all_sync(0xffffffffu, qvis == all);
-        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.s_full), tiles & 1, abort_flag));
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.s_full), tiles & 1, abort_flag, wait_ns));
         if (!ok) break;
         tc_fence_after();
         uint32_t sv[64];
@@ -558,7 +563,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(bar(bars.pt_full));
         // dP^T of this tile
-        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.dp_full), tiles & 1, abort_flag));
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.dp_full), tiles & 1, abort_flag, wait_ns));
         if (!ok) break;
         tc_fence_after();
         // dS^T = P^T o (dP^T - delta), packed to bf16 pairs
@@ -602,7 +607,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       release();
       // dK (first half of the pair) and dV (second half) of the unit's keys: thread = key row
-      ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.acc_full), units & 1, abort_flag));
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.acc_full), units & 1, abort_flag, wait_ns));
       if (!ok) break;
       tc_fence_after();
       {
@@ -660,6 +665,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ uint32_t tmem_base_s;
   __shared__ int abort_s;
   volatile int* abort_flag = &abort_s;
+  const uint64_t wait_ns = p.wait_ns;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t sbase = smem_u32(smem);
   auto bar = [](uint64_t& b) { return smem_u32(&b); };
@@ -711,7 +717,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (;;) {
       const int slot = u_it & 1;
       if (u_it >= 2) {
-        ok = __all_sync(kAll, mbar_wait(bar(bars.u_empty[slot]), ((u_it >> 1) - 1) & 1, abort_flag));
+        ok = __all_sync(kAll, mbar_wait(bar(bars.u_empty[slot]), ((u_it >> 1) - 1) & 1, abort_flag, wait_ns));
         if (!ok) break;
       }
       bool done;
@@ -722,7 +728,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const volatile uint32_t* bits = ring_bits[slot];
       if (popc_bits(bits) == 0) continue;
       if (qd_loads >= 1) {
-        ok = __all_sync(kAll, mbar_wait(bar(bars.qd_empty), (qd_loads - 1) & 1, abort_flag));
+        ok = __all_sync(kAll, mbar_wait(bar(bars.qd_empty), (qd_loads - 1) & 1, abort_flag, wait_ns));
         if (!ok) break;
       }
       if (lane == 0) {
@@ -737,7 +743,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int j = next_bit(bits, -1); j >= 0 && ok; j = next_bit(bits, j)) {
         const uint32_t sk = k_loads % 3, sv = v_loads & 1;
         if (k_loads >= 3) {
-          ok = __all_sync(kAll, mbar_wait(bar(bars.k_empty[sk]), ((k_loads / 3) - 1) & 1, abort_flag));
+          ok = __all_sync(kAll, mbar_wait(bar(bars.k_empty[sk]), ((k_loads / 3) - 1) & 1, abort_flag, wait_ns));
           if (!ok) break;
         }
         if (lane == 0) {
@@ -748,7 +754,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         ++k_loads;
         if (v_loads >= 2) {
-          ok = __all_sync(kAll, mbar_wait(bar(bars.v_empty[sv]), ((v_loads >> 1) - 1) & 1, abort_flag));
+          ok = __all_sync(kAll, mbar_wait(bar(bars.v_empty[sv]), ((v_loads >> 1) - 1) & 1, abort_flag, wait_ns));
           if (!ok) break;
         }
         if (lane == 0) {
@@ -764,6 +770,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (!ok && lane == 0) {
       *abort_flag = 1;
       atomicOr(&g_error_word, MBE_DEVERR_TIMEOUT);
+    }
+    // The copies already issued land before the CTA can exit (see dkdv_kernel).
+    if (lane == 0) {
       const int zero = 0;
       if (qd_loads >= 1) mbar_wait(bar(bars.qd_full), (qd_loads - 1) & 1, &zero);
       for (uint32_t n = (k_loads >= 3 ? k_loads - 3 : 0); n < k_loads; ++n)
@@ -781,7 +790,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // S = Q K_t^T into S buffer t & 1 (issued after dQ of tile t - 2, which read dS there)
       auto issue_s = [&](uint32_t t) {
         const uint32_t b = t & 1;
-        if (!mbar_wait(bar(bars.k_full[t % 3]), (t / 3) & 1, abort_flag)) return false;
+        if (!mbar_wait(bar(bars.k_full[t % 3]), (t / 3) & 1, abort_flag, wait_ns)) return false;
         tc_fence_after();
         const uint32_t ka = sbase + kRingA + (t % 3) * kTileBytes;
 #pragma unroll
@@ -797,8 +806,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       // dP = dO V_t^T once the compute warps have read dP of tile t - 1
       auto issue_dp = [&](uint32_t t) {
-        if (t >= 1 && !mbar_wait(bar(bars.dp_free), (t - 1) & 1, abort_flag)) return false;
-        if (!mbar_wait(bar(bars.v_full[t & 1]), (t >> 1) & 1, abort_flag)) return false;
+        if (t >= 1 && !mbar_wait(bar(bars.dp_free), (t - 1) & 1, abort_flag, wait_ns)) return false;
+        if (!mbar_wait(bar(bars.v_full[t & 1]), (t >> 1) & 1, abort_flag, wait_ns)) return false;
         tc_fence_after();
         const uint32_t va = sbase + kRingB + (t & 1) * kTileBytes;
 #pragma unroll
@@ -815,23 +824,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       for (;;) {
         const int slot = u_it & 1;
-        if (!mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag)) { ok = false; break; }
+        if (!mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag, wait_ns)) { ok = false; break; }
         const Unit un = ring[slot];
         const int n_k = popc_bits(ring_bits[slot]);
         mbar_arrive(bar(bars.u_empty[slot]));
         ++u_it;
         if (un.seq < 0) break;
         if (n_k == 0) continue;
-        if (!mbar_wait(bar(bars.qd_full), units & 1, abort_flag)) { ok = false; break; }
+        if (!mbar_wait(bar(bars.qd_full), units & 1, abort_flag, wait_ns)) { ok = false; break; }
         // S two tiles ahead: it runs while the compute warps form dS of the tile before
         if (!issue_s(tiles) || !issue_dp(tiles) || (n_k >= 2 && !issue_s(tiles + 1))) { ok = false; break; }
         for (int j = 0; j < n_k; ++j) {
           const uint32_t t = tiles + j;
-          if (!mbar_wait(bar(bars.ds_full), t & 1, abort_flag)) { ok = false; break; }
+          if (!mbar_wait(bar(bars.ds_full), t & 1, abort_flag, wait_ns)) { ok = false; break; }
           // the next tile's dP first: the compute warps wait for it, and its region was
           // read before ds_full
           if (j + 1 < n_k && !issue_dp(t + 1)) { ok = false; break; }
-          if (j == 0 && units >= 1 && !mbar_wait(bar(bars.acc_empty), (units - 1) & 1, abort_flag)) {
+          if (j == 0 && units >= 1 && !mbar_wait(bar(bars.acc_empty), (units - 1) & 1, abort_flag, wait_ns)) {
             ok = false;
             break;
           }
@@ -872,7 +881,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok = true;
     for (;;) {
       const int slot = u_it & 1;
-      ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag));
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.u_full[slot]), (u_it >> 1) & 1, abort_flag, wait_ns));
       if (!ok) break;
       const Unit un = ring[slot];
       const volatile uint32_t* bits = ring_bits[slot];
@@ -912,7 +921,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int n_vis = min(kTile, un.len - j * kTile);
         const bool any_vis = __any_sync(0xffffffffu, kbits != 0u);
         const bool every = __all_sync(0xffffffffu, !qv || (kbits == tile_mask && n_vis == kTile));
-        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.s_full[b]), (tiles >> 1) & 1, abort_flag));
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.s_full[b]), (tiles >> 1) & 1, abort_flag, wait_ns));
         if (!ok) break;
         tc_fence_after();
         uint32_t sv[64];
@@ -949,7 +958,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int e = 0; e < 4; ++e) pw[4 * g8 + e] = w[e];
           }
         }
-        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.dp_full), tiles & 1, abort_flag));
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.dp_full), tiles & 1, abort_flag, wait_ns));
         if (!ok) break;
         tc_fence_after();
         uint32_t dsa[32];
@@ -981,7 +990,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       release();
       // dQ * scale of this row, this warp's half of the head dimension
-      ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.acc_full), units & 1, abort_flag));
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.acc_full), units & 1, abort_flag, wait_ns));
       if (!ok) break;
       tc_fence_after();
 #pragma unroll 1
@@ -1266,6 +1275,7 @@ extern "C" mbe_status mbe_block_mask_attention_bwd(const void* q, const void* k,
   p.lgG = lgG;
   p.scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(kD));
   p.scale_log2 = p.scale * kLog2e;
+  p.wait_ns = wait_limit_ns();
   // warps the plans launch: every unit of sequences no longer than max_seq_len
   const int64_t per_seq_kv = (static_cast<int64_t>(max_seq_len) + kTile - 1) / kTile;
   const int64_t per_seq_q = ((static_cast<int64_t>(max_seq_len) << lgG) + kTile - 1) / kTile;

@@ -20,6 +20,8 @@ MBE_OK = 0
 STATUS_NAMES = {0: "MBE_OK", 1: "MBE_ERR_INVALID_ARG", 2: "MBE_ERR_UNSUPPORTED", 3: "MBE_ERR_CUDA",
                 4: "MBE_ERR_TIMEOUT", 5: "MBE_ERR_WORKSPACE", 6: "MBE_ERR_DEVICE_CHECK"}
 DEVERR_TIMEOUT, DEVERR_LENGTH, DEVERR_PAGE, DEVERR_CAPACITY, DEVERR_PLAN = 0x1, 0x2, 0x4, 0x8, 0x10
+DEVERR_NONFINITE = 0x20
+DEFAULT_WAIT_LIMIT_NS = 1_000_000_000
 BLOCK_CAUSAL, MULTI_BLOCK_BIDIRECTIONAL, BLOCK_MASK = 0, 1, 2
 HEADER = _build.INCLUDE / "mbe.h"
 
@@ -114,6 +116,10 @@ def lib(build_if_missing: bool = True):
     L.mbe_last_error_string.argtypes = []
     L.mbe_version.restype = i32
     L.mbe_version.argtypes = []
+    L.mbe_set_wait_limit_ns.restype = ctypes.c_uint64
+    L.mbe_set_wait_limit_ns.argtypes = [ctypes.c_uint64]
+    L.mbe_window_attention_plan_stats.restype = ctypes.c_int
+    L.mbe_window_attention_plan_stats.argtypes = [P, sz, ctypes.POINTER(i32), ctypes.POINTER(i32), P]
     _lib = L
     return L
 
@@ -579,3 +585,19 @@ def get_device_error(stream=None):
     flags = ctypes.c_uint32(0)
     st = lib().mbe_get_device_error(_stream(stream), ctypes.byref(flags))
     return st, flags.value
+
+
+def set_wait_limit_ns(limit_ns: int) -> int:
+    """Sets the limit of the kernels' bounded waits (mbe_set_wait_limit_ns);
+    returns the previous limit."""
+    return int(lib().mbe_set_wait_limit_ns(int(limit_ns)))
+
+
+def window_attention_plan_stats(workspace, stream=None):
+    """(work units, split-KV merge groups) of the plan held in `workspace`."""
+    _need(workspace, "workspace", torch.uint8)
+    n_units, n_groups = ctypes.c_int32(0), ctypes.c_int32(0)
+    _check("mbe_window_attention_plan_stats",
+           lib().mbe_window_attention_plan_stats(_ptr(workspace), workspace.numel(), ctypes.byref(n_units),
+                                                 ctypes.byref(n_groups), _stream(stream)))
+    return n_units.value, n_groups.value

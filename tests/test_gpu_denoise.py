@@ -176,3 +176,45 @@ def test_denoise_serving_size_sampled():
     h_ref = torch.distributions.Categorical(logits=lg.double()).entropy().numpy()
     assert np.abs(res["entropy"][rows].cpu().numpy() - h_ref).max() <= H_ATOL
     assert mbe.get_device_error() == (0, 0)
+
+
+@pytest.mark.parametrize("bad", ["nan", "all_neginf"])
+def test_block_whose_masked_rows_lack_a_softmax_unmasks_nothing(bad):
+    """Forced unmasking (Sec. 2.3) never picks a row without a softmax: a block
+    whose masked rows all have a NaN logit, or all -inf logits, unmasks none and
+    writes only its own rows (no row index is chosen for it). Other rows carry
+    random -inf vocabulary masks, whose entropies must also match the oracle."""
+    B, V = 32, 4096
+    lengths = [64, 96]
+    logits, tokens, cu, mask_id = _problem(lengths, V, torch.float32, seed=77, mask_frac=0.4)
+    R = sum(lengths)
+    blk = np.arange(96, 128)                               # block 1 of sequence 1
+    tokens[torch.from_numpy(blk)] = mask_id
+    for r in blk:
+        if bad == "nan":
+            logits[r, (r * 37) % V] = float("nan")
+        else:
+            logits[r, :] = float("-inf")
+    g = torch.Generator().manual_seed(5)
+    vm = torch.rand(R, V, generator=g) < 0.2
+    vm[torch.from_numpy(blk)] = False
+    logits = logits.masked_fill(vm, float("-inf"))
+    res = mbe.denoise_update(logits.to(DEV), tokens.to(DEV), cu.to(DEV), block_size=B, mask_id=mask_id,
+                             omega_mask=0.9, omega_edit=0.5, max_blocks=3)
+    st, flags = mbe.get_device_error()
+    assert st == 6 and flags == mbe.DEVERR_NONFINITE
+    ref = oracle.denoise_update(logits.numpy(), tokens.numpy(), cu.numpy(), B, mask_id, 0.9, 0.5, max_blocks=3)
+    assert ref["undecidable"]
+    gk = {k: v.cpu().numpy() for k, v in res.items() if v is not None}
+    assert (gk["kind"][blk] == 0).all() and (gk["new_tokens"][blk] == mask_id).all()
+    assert (gk["argmax"][blk] == -1).all() and np.isnan(gk["confidence"][blk]).all()
+    assert gk["block_changed"][1, 1] == 0
+    good = np.setdiff1d(np.arange(R), blk)
+    np.testing.assert_array_equal(gk["argmax"][good], ref["argmax"][good])
+    rel = np.abs(gk["confidence"][good] - ref["confidence"][good]) / ref["confidence"][good]
+    assert rel.max() <= 1e-5
+    assert np.abs(gk["entropy"][good] - ref["entropy"][good]).max() <= H_ATOL
+    np.testing.assert_array_equal(gk["kind"], ref["kind"])
+    np.testing.assert_array_equal(gk["new_tokens"], ref["new_tokens"])
+    np.testing.assert_array_equal(gk["block_changed"], ref["block_changed"])
+    np.testing.assert_array_equal(gk["seq_changes"], ref["seq_changes"])

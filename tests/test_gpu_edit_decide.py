@@ -119,3 +119,41 @@ def test_new_tokens_may_alias_committed():
     c = prob.committed.clone()
     mbe.edit_decide(prob.logits, c, tau=0.0, new_tokens=c)
     assert torch.equal(c, ref[0])
+
+
+@pytest.mark.parametrize("dtype,vocab", [(torch.float32, 1000), (torch.bfloat16, 32768), (torch.bfloat16, 37)])
+def test_rows_without_softmax_and_vocabulary_masks(dtype, vocab):
+    """Rows with a NaN or +inf logit, or with every logit -inf, get no decision:
+    the token stays, argmax is -1, confidence NaN, and the call raises
+    MBE_DEVERR_NONFINITE. -inf logits beside finite ones are tokens of
+    probability 0, also where they fill whole 16-byte vectors at the start of a
+    thread's stride or the scalar tail. Every other row matches the oracle."""
+    R = 40
+    g = torch.Generator().manual_seed(vocab)
+    logits = torch.randn(R, vocab, generator=g) * 2.0
+    logits[torch.arange(R), torch.randint(0, vocab, (R,), generator=g)] += 5.0
+    committed = torch.randint(0, vocab, (R,), generator=g, dtype=torch.int64).to(torch.int32)
+    logits[3, vocab // 2] = float("nan")
+    logits[7, vocab - 1] = float("inf")
+    logits[11, :] = float("-inf")
+    logits[13, 0] = float("nan")
+    logits[13, 1:] = float("-inf")
+    logits[17, : min(vocab - 1, 4096)] = float("-inf")       # leading vectors of every thread
+    logits[19, :-1] = float("-inf")                           # only the last entry (scalar tail if ragged) is finite
+    logits[21] = logits[21].masked_fill(torch.rand(vocab, generator=g) < 0.3, float("-inf"))
+    lc = logits.to(dtype)
+    res = mbe.edit_decide(lc.to(DEV), committed.to(DEV), tau=0.0)
+    st, flags = mbe.get_device_error()
+    assert st == 6 and flags == mbe.DEVERR_NONFINITE
+    ref = _oracle(lc, committed, tau=0.0)
+    assert ref["undecidable"]
+    new_g, mask_g, conf_g, am_g = [t.cpu().numpy() for t in res]
+    bad = np.array([3, 7, 11, 13])
+    assert (ref["argmax"][bad] == -1).all()
+    np.testing.assert_array_equal(am_g[bad], -1)
+    np.testing.assert_array_equal(new_g[bad], committed.numpy()[bad])
+    assert not mask_g[bad].any() and np.isnan(conf_g[bad]).all()
+    good = np.array([r for r in range(R) if r not in bad])
+    compare_edit(res, ref, lc[good].double(), np.zeros(len(good)), rows=good)
+    assert am_g[19] == vocab - 1 and conf_g[19] == 1.0
+    assert mbe.get_device_error() == (0, 0)

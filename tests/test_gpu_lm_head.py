@@ -143,3 +143,28 @@ def test_argument_errors():
     # zero rows: nothing to do
     out = mbe.lm_head_edit_decide(hd[:0], wd, cd[:0])
     assert out[0].numel() == 0
+
+
+def test_non_finite_hidden_row_gets_no_decision():
+    """A hidden row holding NaN (or +inf) makes every logit of its row NaN: that
+    row keeps its token with argmax -1 and confidence / entropy NaN, and
+    MBE_DEVERR_NONFINITE is raised. Each row's logits depend on its own hidden
+    row only, so every other row is bit-identical to the run without it."""
+    R, V, d = 160, 3000, 256
+    h, w, committed, _ = _problem(R, V, d, seed=9)
+    hd, wd, cd = h.to(DEV), w.to(DEV), committed.to(DEV)
+    ref = mbe.lm_head_edit_decide(hd, wd, cd, tau=0.0, want_entropy=True)
+    assert mbe.get_device_error() == (0, 0)
+    hb = hd.clone()
+    hb[5, 17] = float("nan")
+    hb[130, :] = float("inf")
+    res = mbe.lm_head_edit_decide(hb, wd, cd, tau=0.0, want_entropy=True)
+    st, flags = mbe.get_device_error()
+    assert st == 6 and flags == mbe.DEVERR_NONFINITE
+    bad = [5, 130]
+    new, mask, conf, am, ent = res
+    assert (am[bad] == -1).all() and torch.equal(new[bad], cd[bad]) and not mask[bad].any()
+    assert torch.isnan(conf[bad]).all() and torch.isnan(ent[bad]).all()
+    good = torch.tensor([r for r in range(R) if r not in bad], device=DEV)
+    for a, b in zip(res, ref):
+        assert torch.equal(a[good], b[good])
