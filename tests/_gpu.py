@@ -1,11 +1,15 @@
 """GPU-test helpers: run the CUDA path through the binding, carve sampled
 sequences out of a large problem for the oracle, and compare."""
+import os
+
 import numpy as np
 import torch
 
 from paper_2607_22663_gb300 import mbe
 from paper_2607_22663_gb300.workloads import AttnProblem, bf16_bits
 from paper_2607_22663_gb300.workloads import extract_sequences as subproblem
+from tests._bars import derived_bar, excess, walk_bar
+from tests._util import oracle_walk_scale
 
 ATTN_ATOL = 1e-2      # max abs error of bf16 attention outputs vs the fp64 oracle
 CONF_RTOL = 1e-5      # relative error of fp32 confidences vs the fp64 oracle
@@ -31,15 +35,26 @@ def oracle_attention(prob: AttnProblem, units=None, scale=None):
                                    prob.page_size, scale=scale, units=units)
 
 
+# (test, worst |err| / output RMS over its (sequence, head) pairs, worst err / bar)
+# of every attention comparison of the session; printed in the terminal summary
+ATTN_REPORT = []
+
+
 def compare_attention(prob: AttnProblem, out_gpu, lse_gpu, seqs=None, heads=None, scale=None, derived_bound=False):
     """Compare GPU outputs of the listed (sequence, q-head) pairs with the oracle.
 
-    Default bar: max abs error <= ATTN_ATOL. With derived_bound, each element
-    must instead satisfy |err| <= u * (max|v| + |o_ref|) + 1e-4, u = 2^-8 the
-    bf16 unit roundoff: the probabilities are rounded to bf16 before the PV
-    product (error <= u * sum_j p_j |v_j| <= u * max|v|) and the output is
-    rounded to bf16 (error <= u * |o|); fp32 accumulation adds < 1e-4. This is
-    the bar for inputs sharpened so that outputs are O(1).
+    Bars (tests/_bars.py), per element:
+      - default: max abs error <= ATTN_ATOL (the stated tolerance) and the
+        random-walk bar u |o| + 6.54 u sigma + 1e-5 derived from bf16 rounding
+        of P, with sigma = sqrt(sum_j P_j^2 v_j^2) from the oracle; for diffuse
+        attention that is a few percent of the output, so the comparison keeps
+        its power when thousands of keys shrink the outputs to ~1e-2;
+      - derived_bound: for sharpened inputs whose outputs are O(1), the
+        worst-case bar (u + fp32 accumulation) sum_j P_j |v_j| + u |o| with
+        sum_j P_j |v_j| from the oracle run on |V| (outputs of size ~4 round
+        by more than 1e-2, so the absolute bound does not apply there).
+    The LSE must be within 2e-3 relative. Records the worst error relative to
+    each pair's output RMS and to its bar in ATTN_REPORT.
     Returns (max abs error, max abs error / output RMS)."""
     seqs = list(range(prob.batch)) if seqs is None else list(seqs)
     Hq = prob.num_q_heads
@@ -47,8 +62,13 @@ def compare_attention(prob: AttnProblem, out_gpu, lse_gpu, seqs=None, heads=None
     sub = subproblem(prob, seqs)
     units = [(i, h) for i in range(len(seqs)) for h in heads]
     o_ref, l_ref = oracle_attention(sub, units=units, scale=scale)
+    if derived_bound:
+        absv = AttnProblem(**{**sub.__dict__, "v_cache": sub.v_cache.abs(), "v_win": sub.v_win.abs()})
+        spv, _ = oracle_attention(absv, units=units, scale=scale)
+    else:
+        sig = oracle_walk_scale(sub, units=units, scale=scale)
     cu_all = prob.cu_window.cpu()
-    worst, worst_rel = 0.0, 0.0
+    worst, worst_rel, worst_bar = 0.0, 0.0, 0.0
     for i, s in enumerate(seqs):
         W = prob.window_host[s]
         if W == 0:
@@ -56,17 +76,24 @@ def compare_attention(prob: AttnProblem, out_gpu, lse_gpu, seqs=None, heads=None
         t0, u0 = int(cu_all[s]), int(sub.cu_window[i])
         g = out_gpu[t0:t0 + W][:, heads].float().cpu().numpy()
         r = o_ref[u0:u0 + W][:, heads]
-        err = np.abs(g - r).max()
-        rms = np.sqrt((r ** 2).mean()) + 1e-30
-        if derived_bound:
-            vmax = max(prob.v_cache.float().abs().max().item(), prob.v_win.float().abs().max().item())
-            bound = 2.0 ** -8 * (vmax + np.abs(r)) + 1e-4
-            assert (np.abs(g - r) <= bound).all(), f"error above the derived bf16 bound (max err {err})"
-        worst, worst_rel = max(worst, err), max(worst_rel, err / rms)
+        for j, h in enumerate(heads):
+            e, rr = np.abs(g[:, j] - r[:, j]), r[:, j]
+            if derived_bound:
+                bar = derived_bar(rr, spv[u0:u0 + W][:, h], prob.prefix_host[s] + W)
+            else:
+                bar = walk_bar(rr, sig[u0:u0 + W][:, h])
+            rms = np.sqrt((rr ** 2).mean()) + 1e-30
+            worst_rel = max(worst_rel, float(e.max()) / rms)
+            x = excess(e, bar)
+            worst_bar = max(worst_bar, x)
+            assert x <= 1.0, (f"sequence {s} head {h}: error {e.max():.3e} exceeds the derived bar "
+                              f"by {x:.2f}x (output rms {rms:.3e})")
+        worst = max(worst, float(np.abs(g - r).max()))
         if lse_gpu is not None:
             lg = lse_gpu[t0:t0 + W][:, heads].cpu().numpy()
             lr = l_ref[u0:u0 + W][:, heads]
             np.testing.assert_allclose(lg, lr, rtol=0, atol=2e-3 * max(1.0, np.abs(lr).max()))
+    ATTN_REPORT.append((os.environ.get("PYTEST_CURRENT_TEST", "?").split(" ")[0], worst_rel, worst_bar))
     if not derived_bound:
         assert worst <= ATTN_ATOL, f"max abs error {worst} > {ATTN_ATOL} (rel to rms {worst_rel})"
     return worst, worst_rel

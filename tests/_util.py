@@ -34,3 +34,19 @@ def oracle_attention(prob, units=None, scale=None):
 def to_bf16_round(x: np.ndarray) -> np.ndarray:
     """Round float64 values to the nearest bf16 (ties to even), returned as float64."""
     return torch.from_numpy(np.ascontiguousarray(x)).to(torch.bfloat16).double().numpy()
+
+
+def oracle_walk_scale(prob, units=None, scale=None):
+    """sqrt(sum_j P_j^2 v_jd^2) per output element [T, Hq, D] (tests/_bars.py):
+    the oracle on the scores for lse, and on doubled scores with the values
+    squared (rounded to bf16) for the weighted sum of v^2."""
+    import math
+
+    from paper_2607_22663_gb300.workloads import AttnProblem
+    from tests._bars import sigma_walk
+    sc = scale if scale is not None else 1.0 / math.sqrt(prob.head_dim)
+    _, lse = oracle_attention(prob, units=units, scale=sc)
+    sq = lambda t: (t.float() ** 2).to(torch.bfloat16)
+    prob2 = AttnProblem(**{**prob.__dict__, "v_cache": sq(prob.v_cache), "v_win": sq(prob.v_win)})
+    out2, lse2 = oracle_attention(prob2, units=units, scale=2.0 * sc)
+    return sigma_walk(lse, lse2, out2)

@@ -24,3 +24,16 @@ def pytest_collection_modifyitems(config, items):
     for it in items:
         if "gpu" in it.keywords:
             it.add_marker(skip)
+
+
+def pytest_terminal_summary(terminalreporter, exitstatus, config):
+    """Attention parity, relative to each compared pair's output RMS."""
+    try:
+        from tests._gpu import ATTN_REPORT
+    except Exception:
+        return
+    if not ATTN_REPORT:
+        return
+    terminalreporter.write_sep("-", "attention parity: worst |err| / output RMS, worst err / bar (tests/_bars.py)")
+    for name, rel, bar in ATTN_REPORT:
+        terminalreporter.write_line(f"{rel:8.4f}  {bar:6.3f}  {name}")

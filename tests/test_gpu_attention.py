@@ -172,12 +172,46 @@ def test_gqa_equals_replicated_kv_heads():
     assert (out.float() - out_r.float()).abs().max().item() <= 1e-2
 
 
+def _planned_run(prob, q_scale_note=None):
+    """Plan into an explicit workspace, report the plan's split groups, then run."""
+    args = (prob.q, prob.k_win, prob.v_win, prob.k_cache, prob.v_cache, prob.block_table, prob.prefix_len,
+            prob.window_len, prob.cu_window, prob.mask_mode)
+    kw = dict(block_size=prob.block_size, max_window=prob.max_window, max_prefix=prob.max_prefix)
+    need = mbe.window_attention_workspace_size(prob.batch, prob.num_q_heads, prob.num_kv_heads, prob.head_dim,
+                                               prob.max_window, prob.max_prefix)
+    ws = torch.empty(need, dtype=torch.uint8, device=DEV)
+    mbe.window_attention_plan(prob.prefix_len, prob.window_len, prob.cu_window, prob.mask_mode,
+                              total_q_tokens=prob.total_tokens, num_q_heads=prob.num_q_heads,
+                              num_kv_heads=prob.num_kv_heads, head_dim=prob.head_dim, workspace=ws, **kw)
+    n_units, n_groups = mbe.window_attention_plan_stats(ws)
+    out, lse = mbe.window_attention_run(*args, return_lse=True, workspace=ws, **kw)
+    assert mbe.get_device_error() == (0, 0)
+    return out, lse, n_units, n_groups
+
+
 def test_split_kv_matches_oracle_and_unsplit():
-    """Few long sequences force split-KV pieces and the LSE merge."""
+    """Few long sequences force split-KV pieces and the LSE merge; each compared
+    (sequence, head) pair is held to the bar relative to its output RMS."""
     prob = attention_problem([20000, 9000], [64, 64], [BIDIRECTIONAL, BLOCK_CAUSAL], 32, 8, 128, 32, 64, seed=13,
                              device=DEV)
-    out, lse = run_attention(prob)
+    out, lse, n_units, n_groups = _planned_run(prob)
+    assert n_groups > 0 and n_units > 2 * 8
+    ref, ref_lse = run_attention(prob)
+    assert torch.equal(out, ref) and torch.equal(lse, ref_lse)
     compare_attention(prob, out, lse, heads=[0, 5, 17, 31])
+
+
+def test_split_kv_sharpened_outputs_order_one():
+    """Queries sharpened x6 over prefixes of 20k-24k keys: the plan cuts the keys
+    into split-KV pieces merged by log-sum-exp, and the outputs are O(1), so the
+    worst-case bar u sum_j p_j |v_j| + u |o| (sum_j p_j |v_j| from the oracle on
+    |V|) pins the weight of every piece in the merge."""
+    prob = attention_problem([24000, 20000], [64, 64], [BIDIRECTIONAL, BLOCK_CAUSAL], 32, 8, 128, 32, 64, seed=19,
+                             device=DEV, q_scale=6.0)
+    out, lse, n_units, n_groups = _planned_run(prob)
+    assert n_groups > 0
+    compare_attention(prob, out, lse, heads=[0, 9, 22, 31], derived_bound=True)
+    assert out.float().abs().max().item() > 1.0
 
 
 def test_bad_page_id_sets_flag_without_fault():

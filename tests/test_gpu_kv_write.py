@@ -7,7 +7,7 @@ import torch
 import oracle
 from paper_2607_22663_gb300 import mbe
 from paper_2607_22663_gb300 import workloads as wl
-from paper_2607_22663_gb300.workloads import BIDIRECTIONAL, attention_problem, bf16_bits
+from paper_2607_22663_gb300.workloads import BIDIRECTIONAL, BLOCK_CAUSAL, AttnProblem, attention_problem, bf16_bits
 from tests._gpu import compare_attention, run_attention
 
 pytestmark = pytest.mark.gpu
@@ -51,14 +51,32 @@ def test_block_write_mask():
 
 
 def test_long32k_write_then_attend():
-    """The long-context workload: write each window, then a standard pass over
-    the next block sees the written keys at positions [P, P+W)."""
-    w = wl.long32k(DEV, windows=(64,))
+    """The long-context workload: the window of an editing pass is written at
+    positions [P, P+W) (bit-exact against the oracle), then a standard pass over
+    the next block (block-causal, prefix P+W) reads the written keys from the
+    cache and matches the oracle on that cache."""
+    w = wl.long32k(DEV, windows=(64, 128))   # the cache reserves room for 128 window tokens
     prob = w["attn"][0]
     kc, vc, st, _ = _gpu_write(prob)
     assert st == 0
     kr, vr = _oracle_write(prob)
     assert np.array_equal(bf16_bits(kc), kr) and np.array_equal(bf16_bits(vc), vr)
+    g = torch.Generator(device=DEV).manual_seed(44)
+    B, n = 32, prob.batch
+    rnd = lambda *shape: torch.randn(*shape, generator=g, device=DEV).to(torch.bfloat16)
+    nxt = AttnProblem(q=rnd(n * B, 32, 128), k_win=rnd(n * B, 8, 128), v_win=rnd(n * B, 8, 128), k_cache=kc,
+                      v_cache=vc, block_table=prob.block_table, prefix_len=prob.prefix_len + prob.window_len,
+                      window_len=torch.full((n,), B, dtype=torch.int32, device=DEV),
+                      cu_window=torch.arange(0, n * B + 1, B, dtype=torch.int32, device=DEV),
+                      mask_mode=torch.full((n,), BLOCK_CAUSAL, dtype=torch.uint8, device=DEV), block_size=B,
+                      page_size=prob.page_size, prefix_host=[p + 64 for p in prob.prefix_host], window_host=[B] * n,
+                      mode_host=[BLOCK_CAUSAL] * n)
+    out, lse = run_attention(nxt)
+    compare_attention(nxt, out, lse, seqs=[0, 3], heads=[0, 13, 31])
+    # the written rows matter: the same pass over the cache before the write differs
+    stale = AttnProblem(**{**nxt.__dict__, "k_cache": prob.k_cache, "v_cache": prob.v_cache})
+    out_stale, _ = run_attention(stale)
+    assert not torch.equal(out_stale, out)
 
 
 def test_bad_page_flagged_and_skipped():
