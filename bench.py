@@ -345,6 +345,7 @@ def time_extras(w, a0, dev, stream, peaks, reps=10):
     ent = torch.rand(a0.batch, 3, a0.block_size, device=dev)
     nv = torch.full((a0.batch,), 3, dtype=torch.int32, device=dev)
     ms_sel = ev_time(lambda: mbe.tail_entropy_select(ent, nv, rho=0.25, k_max=4))
+    workloads = time_workloads(dev, stream, peaks)
     lm_head = time_lm_head(w, dev, peaks, ev_time)
     sft = time_sft_attention(dev, peaks, ev_time)
     refresh = time_refresh(w, dev, stream, peaks, ev_time)
@@ -356,7 +357,104 @@ def time_extras(w, a0, dev, stream, peaks, reps=10):
                                "frac_hbm": round(byts / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"], 4),
                                "rows": R, "vocab": V},
             "tail_entropy_select": {"us": round(ms_sel * 1e3, 2), "sequences": a0.batch, "k_max": 4, "rho": 0.25},
-            "lm_head_edit_decide": lm_head, "sft_attention": sft, "refresh": refresh, "pass_loop": loop}
+            "lm_head_edit_decide": lm_head, "sft_attention": sft, "refresh": refresh, "pass_loop": loop,
+            **workloads}
+
+
+def time_workloads(dev, stream, peaks, reps=10):
+    """Device-timed attention of the other workloads, one block each:
+    long32k (long-context editing: windows of 64, 128 and 256 queries over a
+    32768-token prefix, each call followed by the window's KV write), varlen64
+    (64 sequences of mixed window sizes and both mask modes, plus its edit
+    decision) and batch8 (8 uniform sequences). Every attention call plans and
+    runs (mbe_window_attention), as a one-layer pass does. Inputs larger than
+    L2, except batch8, for which a 256 MiB buffer is written before every call;
+    only the calls themselves lie between their CUDA events."""
+    from paper_2607_22663_gb300 import mbe
+    from paper_2607_22663_gb300 import workloads as wl
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    res = {}
+    for name in ("long32k", "varlen64", "batch8"):
+        w = wl.WORKLOADS[name](dev)
+        calls, ep = w["attn"], w["edit"]
+        with_kv_write = name == "long32k"
+        need = max(mbe.window_attention_workspace_size(a.batch, a.num_q_heads, a.num_kv_heads, a.head_dim,
+                                                       a.max_window, a.max_prefix) for a in calls)
+        ws = torch.empty(need, dtype=torch.uint8, device=dev)
+        outs = [torch.empty_like(a.q) for a in calls]
+        abytes = [attention_bytes(a.prefix_host, a.window_host, a.num_q_heads, a.num_kv_heads, a.head_dim)
+                  for a in calls]
+        flops = [attention_flops(a.prefix_host, a.window_host, a.mode_host, a.num_q_heads, a.head_dim, a.block_size)
+                 for a in calls]
+        small = max(abytes) < 2 * 129e6
+
+        def attend(i, a):
+            mbe.window_attention(a.q, a.k_win, a.v_win, a.k_cache, a.v_cache, a.block_table, a.prefix_len,
+                                 a.window_len, a.cu_window, a.mask_mode, block_size=a.block_size,
+                                 max_window=a.max_window, max_prefix=a.max_prefix, out=outs[i], workspace=ws)
+
+        def write(a):
+            mbe.kv_window_write(a.k_win, a.v_win, a.k_cache, a.v_cache, a.block_table, a.prefix_len, a.window_len,
+                                a.cu_window, block_size=a.block_size, max_window=a.max_window)
+
+        ev = [[[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in calls] for _ in range(reps + 3)]
+        for r in range(reps + 3):
+            for i, a in enumerate(calls):
+                if small:
+                    flush.fill_(r & 0xFF)
+                ev[r][i][0].record(stream)
+                attend(i, a)
+                ev[r][i][1].record(stream)
+                if with_kv_write:
+                    write(a)
+                ev[r][i][2].record(stream)
+        torch.cuda.synchronize()
+        ms = [statistics.mean(ev[r][i][0].elapsed_time(ev[r][i][1]) for r in range(3, reps + 3))
+              for i in range(len(calls))]
+        t = sum(ms) * 1e-3
+        tf = sum(flops) / t / 1e12
+        gbs = sum(abytes) / t / 1e9
+        blk = {"attention_ms_per_call": [round(x, 4) for x in ms], "window": [a.max_window for a in calls],
+               "attention_tflops": round(tf, 1), "frac_bf16_peak_sustained": round(tf / peaks["bf16_tflops_sustained"], 4),
+               "frac_bf16_peak_burst": round(tf / peaks["bf16_tflops"], 4), "attention_gbs": round(gbs, 1),
+               "frac_hbm": round(gbs / peaks["hbm_gbs"], 4), "flops": flops, "bytes": abytes,
+               "l2": "256 MiB written before each call" if small else "inputs larger than L2",
+               "config": workload_config(w)}
+        if with_kv_write:
+            kv_ms = [statistics.mean(ev[r][i][1].elapsed_time(ev[r][i][2]) for r in range(3, reps + 3))
+                     for i in range(len(calls))]
+            kv_bytes = [2 * 2 * sum(a.window_host) * a.num_kv_heads * a.head_dim * 2 for a in calls]
+            blk["kv_write_ms_per_call"] = [round(x, 4) for x in kv_ms]
+            blk["kv_write_gbs"] = [round(b / (x * 1e-3) / 1e9, 1) for b, x in zip(kv_bytes, kv_ms)]
+            blk["windows_per_s"] = round(calls[0].batch * len(calls) / ((sum(ms) + sum(kv_ms)) * 1e-3), 1)
+        if ep is not None:
+            new = torch.empty(ep.logits.shape[0], dtype=torch.int32, device=dev)
+            msk = torch.empty_like(new, dtype=torch.uint8)
+            cf = torch.empty_like(new, dtype=torch.float32)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            tot = 0.0
+            for r in range(reps + 3):
+                if small:
+                    flush.fill_(r & 0xFF)
+                e0.record(stream)
+                mbe.edit_decide(ep.logits, ep.committed, tau=ep.tau, tau_per_row=ep.tau_per_row, new_tokens=new,
+                                edit_mask=msk, confidence=cf, want_argmax=False)
+                e1.record(stream)
+                torch.cuda.synchronize()
+                if r >= 3:
+                    tot += e0.elapsed_time(e1)
+            ems = tot / reps
+            eb = edit_bytes(ep.logits.shape[0], ep.logits.shape[1], ep.logits.element_size())
+            blk["edit_decide"] = {"ms": round(ems, 4), "gbs": round(eb / (ems * 1e-3) / 1e9, 1),
+                                  "frac_hbm": round(eb / (ems * 1e-3) / 1e9 / peaks["hbm_gbs"], 4)}
+            blk["windows_per_s"] = round(calls[0].batch / ((sum(ms) + ems) * 1e-3), 1)
+        elif not with_kv_write:
+            blk["windows_per_s"] = round(calls[0].batch / t, 1)
+        res[name] = blk
+        del w, calls, ep, ws, outs
+        torch.cuda.empty_cache()
+    del flush
+    return res
 
 
 def time_lm_head(w, dev, peaks, ev_time, hidden=4096):
