@@ -549,12 +549,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         ok = __all_sync(kAll, mbar_wait(bar(bars.q_empty), (q_loads - 1) & 1, abort_flag, wait_ns));
         if (!ok) break;
       }
-      if (lane == 0) {
-        mbar_arrive_expect_tx(bar(bars.q_full), n_qt * S::kQTile);
-        for (int qt = 0; qt < n_qt; ++qt)
-          for (int h = 0; h < S::kHalves; ++h)
-            tma_load_3d(sbase + S::kQ + qt * S::kQTile + h * S::kHalfBytes, &tm_q, bar(bars.q_full), h * 64,
-                        wu.kv_head * p.G, cu + (wu.row0 + qt * kTileRows) / p.G);
+      // the boxes of a load are issued by as many lanes at once (lane = box), each
+      // completing on the same barrier, whose byte count lane 0 sets first
+      if (lane == 0) mbar_arrive_expect_tx(bar(bars.q_full), n_qt * S::kQTile);
+      __syncwarp();
+      if (lane < n_qt * S::kHalves) {
+        const int qt = lane / S::kHalves, h = lane % S::kHalves;
+        tma_load_3d(sbase + S::kQ + qt * S::kQTile + h * S::kHalfBytes, &tm_q, bar(bars.q_full), h * 64,
+                    wu.kv_head * p.G, cu + (wu.row0 + qt * kTileRows) / p.G);
       }
       ++q_loads;
       const int P = wu.prefix;
@@ -575,8 +577,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         return pg;
       };
       int pg_base = -(1 << 30), pg_lo = 0, pg_hi = 0;
-      auto page_of = [&](int lp) {  // warp-uniform lp >= pg_base
-        return __shfl_sync(kAll, lp < pg_base + 32 ? pg_lo : pg_hi, (lp - pg_base) & 31);
+      auto page_of = [&](int lp) {  // per-lane lp in [pg_base, pg_base + 64)
+        const int lo = __shfl_sync(kAll, pg_lo, (lp - pg_base) & 31);
+        const int hi = __shfl_sync(kAll, pg_hi, (lp - pg_base) & 31);
+        return lp < pg_base + 32 ? lo : hi;
       };
       auto ensure_window = [&](int lp) {  // makes lp the current page window's anchor if needed
         if (lp < pg_base || lp >= pg_base + 64) {
@@ -607,20 +611,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t dst = sbase + S::kRing + sl * S::kItem;
           const uint32_t fb = bar(bars.full[sl]);
           if (lane == 0) mbar_arrive_expect_tx(fb, S::kItem);
+          __syncwarp();
           if (t < nP) {
+            // lane = box: page box l = lane / halves, column half h = lane % halves
+            // (at most 16 boxes: 128 keys over pages of 8 or more, two halves)
             const CUtensorMap* tm = kv ? &tm_vc : &tm_kc;
-            for (int l = 0; l < p.loads_per_tile; ++l) {
-              const int key0 = t * kTileKeys + l * p.box_rows;
-              const int page = page_of(key0 / p.page_size);
-              if (lane == 0)
-                for (int h = 0; h < S::kHalves; ++h)
-                  tma_load_4d(dst + h * S::kHalfBytes + l * p.box_rows * 128, tm, fb, h * 64, key0 % p.page_size,
-                              wu.kv_head, page);
-            }
-          } else if (lane == 0) {
+            const int l = lane / S::kHalves, h = lane % S::kHalves;
+            const int key0 = t * kTileKeys + min(l, p.loads_per_tile - 1) * p.box_rows;
+            const int page = page_of(key0 / p.page_size);
+            if (l < p.loads_per_tile)
+              tma_load_4d(dst + h * S::kHalfBytes + l * p.box_rows * 128, tm, fb, h * 64, key0 % p.page_size,
+                          wu.kv_head, page);
+          } else if (lane < S::kHalves) {
             const int tok = cu + (t - nP) * kTileKeys;
-            for (int h = 0; h < S::kHalves; ++h)
-              tma_load_3d(dst + h * S::kHalfBytes, kv ? &tm_vw : &tm_kw, fb, h * 64, wu.kv_head, tok);
+            tma_load_3d(dst + lane * S::kHalfBytes, kv ? &tm_vw : &tm_kw, fb, lane * 64, wu.kv_head, tok);
           }
         }
       }
