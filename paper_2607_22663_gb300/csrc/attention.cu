@@ -17,7 +17,11 @@
 //       warps 4-11  two softmax warpgroups, one per 128-row query tile: TMEM
 //                   load of S, exp2 against the running max (the row max is
 //                   taken first only where the max may have moved by 2^8),
-//                   P written back to TMEM as bf16, lazy rescaling of O, epilogue
+//                   P written back to TMEM as bf16, lazy rescaling of O, epilogue.
+//                   A unit with a single query tile ("split unit") gives the
+//                   even key tiles to chain 0 and the odd ones to chain 1, both
+//                   on the same rows; warpgroup 0 merges the two (m, l, O) in
+//                   TMEM before its epilogue.
 //     GQA: the G query heads sharing a KV head are packed into the rows of a
 //     tile (row = token * G + head), so every K/V tile feeds 256 query rows.
 //     The mask is applied per row as a visible-column count: every prefix key
@@ -424,6 +428,7 @@ struct Bars {
   uint64_t full[kMaxSlots], empty[kMaxSlots];
   uint64_t s_full[2], p_full[2], o_full[2], o_empty[2];
   uint64_t u_full[2], u_empty[2];
+  uint64_t x_full, x_empty;  // split units: (m, l) of chain 1 handed to warpgroup 0
 };
 
 template <int D, bool kMask>
@@ -440,6 +445,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ uint32_t unit_tiles[kMask ? 2 : 1][kMask ? kMaskTileWords : 1];
   __shared__ uint32_t tmem_base_s;
   __shared__ int abort_s;
+  __shared__ float2 xchg[kTileRows];  // split units: running max and sum of chain 1, per row
   volatile int* abort_flag = &abort_s;
   const uint64_t wait_ns = p.wait_ns;
 
@@ -464,6 +470,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(bar(bars.u_full[i]), 1);
       mbar_init(bar(bars.u_empty[i]), 9);
     }
+    mbar_init(bar(bars.x_full), 4);
+    mbar_init(bar(bars.x_empty), 4);
     mbar_fence_init();
   }
   if (warp == 1) {
@@ -654,8 +662,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto item_addr = [&](uint32_t n) { return sbase + S::kRing + (n % S::kSlots) * S::kItem; };
       auto wait_item = [&](uint32_t n) { return mbar_wait(bar(bars.full[n % S::kSlots]), (n / S::kSlots) & 1, abort_flag, wait_ns); };
       auto release_item = [&](uint32_t n) { umma_commit(bar(bars.empty[n % S::kSlots])); };
-      auto issue_qk = [&](int i, uint32_t ka) {
-        const uint32_t qa = sbase + S::kQ + i * S::kQTile;
+      // S of chain i = Q tile qt times K (qt = i, or 0 for both chains of a split unit)
+      auto issue_qk = [&](int i, uint32_t ka, int qt) {
+        const uint32_t qa = sbase + S::kQ + qt * S::kQTile;
 #pragma unroll
         for (int h = 0; h < S::kHalves; ++h)
 #pragma unroll
@@ -686,10 +695,57 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait(bar(bars.q_full), q_it & 1, abort_flag, wait_ns)) { ok = false; break; }
         ++q_it;
         // items of tile ki: K = 2 ki, V = 2 ki + 1
+        if (n_qt == 1 && n_t >= 2) {
+          // Split unit (one query tile, two or more key tiles): chain c takes the key
+          // tiles j = c, c + 2, ..., both against query tile 0, so that the two chains
+          // overlap as they do for two query tiles; the epilogue merges them.
+          for (int c = 0; c < 2 && ok; ++c) {
+            if (!wait_item(2 * (kv_it + c))) { ok = false; break; }
+            tc_fence_after();
+            issue_qk(c, item_addr(2 * (kv_it + c)), 0);
+            umma_commit(bar(bars.s_full[c]));
+            release_item(2 * (kv_it + c));
+          }
+          if (!ok) break;
+          if (n_t == 2) umma_commit(bar(bars.q_empty));
+          for (int j0 = 0; j0 < n_t && ok; j0 += 2) {
+#pragma unroll
+            for (int c = 0; c < 2; ++c) {  // chain c as a constant: no indexed counters
+              const int j = j0 + c;
+              if (j >= n_t || !ok) break;
+              const uint32_t ki = kv_it + j;
+              if (!wait_item(2 * ki + 1)) { ok = false; break; }
+              if (!mbar_wait(bar(bars.p_full[c]), p_cnt[c] & 1, abort_flag, wait_ns)) { ok = false; break; }
+              ++p_cnt[c];
+              if (j < 2 && o_cnt[c] > 0 && !mbar_wait(bar(bars.o_empty[c]), (o_cnt[c] - 1) & 1, abort_flag, wait_ns)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              issue_pv(c, item_addr(2 * ki + 1), j >= 2);
+              if (j + 2 >= n_t) umma_commit(bar(bars.o_full[c]));  // the chain's last tile
+              release_item(2 * ki + 1);
+              if (j + 2 < n_t) {
+                const uint32_t kn = 2 * (ki + 2);
+                if (!wait_item(kn)) { ok = false; break; }
+                tc_fence_after();
+                issue_qk(c, item_addr(kn), 0);
+                umma_commit(bar(bars.s_full[c]));
+                release_item(kn);
+                if (j + 3 == n_t) umma_commit(bar(bars.q_empty));  // the unit's last QK
+              }
+            }
+          }
+          if (!ok) break;
+          kv_it += n_t;
+          ++o_cnt[0];
+          ++o_cnt[1];
+          continue;
+        }
         if (!wait_item(2 * kv_it)) { ok = false; break; }
         tc_fence_after();
         for (int i = 0; i < n_qt; ++i) {
-          issue_qk(i, item_addr(2 * kv_it));
+          issue_qk(i, item_addr(2 * kv_it), i);
           umma_commit(bar(bars.s_full[i]));
         }
         release_item(2 * kv_it);
@@ -714,7 +770,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!wait_item(kn)) { ok = false; break; }
                 tc_fence_after();
               }
-              issue_qk(i, item_addr(kn));
+              issue_qk(i, item_addr(kn), i);
               umma_commit(bar(bars.s_full[i]));
               if (i == n_qt - 1) {
                 release_item(kn);
@@ -744,7 +800,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t t_lane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
     const uint32_t tS = t_lane + kTmemS + 128 * wg;
     const uint32_t tO = t_lane + wg * D;
-    uint32_t u_it = 0, s_cnt = 0, o_cnt = 0, kv_it = 0;
+    uint32_t u_it = 0, s_cnt = 0, o_cnt = 0, kv_it = 0, x_cnt = 0;
     bool ok = true;
     for (;;) {
       const int slot = u_it & 1;
@@ -773,12 +829,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       const int P = wu.prefix;
       const int nP = (P + kTileKeys - 1) / kTileKeys;
-      if (wg >= n_qt) {
+      // split unit: both warpgroups work on query tile 0, warpgroup c on key tiles c, c + 2, ...
+      const bool split = n_qt == 1 && n_t >= 2;
+      if (wg >= n_qt && !split) {
         kv_it += n_t;
         if (kMask) release_unit();
         continue;
       }
-      const int R = wu.row0 + kTileRows * wg + r;
+      const int R = wu.row0 + kTileRows * (split ? 0 : wg) + r;
       const int qi = R / p.G, hh = R - qi * p.G;
       const bool valid = qi < W;
       const int lim = (mode == MBE_BLOCK_CAUSAL) ? min(W, (qi / p.block_size + 1) * p.block_size) : W;
@@ -801,6 +859,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         } else {
           t = wu.tile_begin + j;
         }
+        if (split && (j & 1) != wg) continue;
         const uint32_t ki = kv_it + j;
         ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.s_full[wg]), s_cnt & 1, abort_flag, wait_ns));
         if (!ok) break;
@@ -926,8 +985,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tmem_st64(tS, v);
         l = l * alpha + (l0 + l1);
-        if (rescale && j > 0) {
-          // O holds PV of tiles < j (complete: s_full(j) was committed after them)
+        if (rescale && j >= (split ? 2 : 1)) {
+          // O holds PV of this chain's earlier tiles (complete: s_full of this tile
+          // was committed after them)
 #pragma unroll 1
           for (int c = 0; c < D / 32; ++c) {
             uint32_t o[32];
@@ -942,7 +1002,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // last window tile (whatever follows the window in k_win / v_win, even
         // NaN) are masked in S but still enter P V as 0 * V: zero them in V.
         const int v0 = (t == nP - 1) ? P % kTileKeys : (t - nP == (W - 1) / kTileKeys ? W % kTileKeys : 0);
-        if (wg == 0 && v0 != 0) {
+        if ((split || wg == 0) && v0 != 0) {
           const uint32_t nv = 2 * ki + 1;  // the V item of this tile
           ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.full[nv % S::kSlots]), (nv / S::kSlots) & 1, abort_flag, wait_ns));
           if (!ok) break;
@@ -967,6 +1027,46 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       ++o_cnt;
       tc_fence_after();
+      if (split && wg == 1) {
+        // chain 1 of a split unit hands its running max and sum to warpgroup 0, which
+        // reads O_1 from TMEM (same lanes), merges and releases both O buffers
+        if (x_cnt > 0) {
+          ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.x_empty), (x_cnt - 1) & 1, abort_flag, wait_ns));
+          if (!ok) break;
+        }
+        ++x_cnt;
+        xchg[r] = make_float2(m, l);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(bars.x_full));
+        continue;
+      }
+      if (split) {
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(bars.x_full), x_cnt & 1, abort_flag, wait_ns));
+        if (!ok) break;
+        ++x_cnt;
+        tc_fence_after();  // O_1 is complete: warpgroup 1 saw its o_full before x_full
+        const float2 c1 = xchg[r];
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(bars.x_empty));
+        const float mm = fmaxf(m, c1.x);
+        const float a0 = (m == neg_inf()) ? 0.f : ex2f(m - mm);
+        const float a1 = (c1.x == neg_inf()) ? 0.f : ex2f(c1.x - mm);
+        l = l * a0 + c1.y * a1;
+        m = mm;
+        // O_0 <- a0 O_0 + a1 O_1 in TMEM; the epilogue below then reads O_0 only
+#pragma unroll 1
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t o0[32], o1[32];
+          tmem_ld32(tO + 32 * c, o0);
+          tmem_ld32(t_lane + D + 32 * c, o1);
+#pragma unroll
+          for (int k = 0; k < 32; ++k)
+            o0[k] = __float_as_uint(fmaf(__uint_as_float(o0[k]), a0, __uint_as_float(o1[k]) * a1));
+          tmem_st32(tO + 32 * c, o0);
+        }
+        tmem_st_wait();
+      }
       const float inv_l = l > 0.f ? 1.f / l : 0.f;
       const float lse2 = l > 0.f ? m + __log2f(l) : neg_inf();
       if (wu.slot < 0) {
@@ -1010,7 +1110,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(bar(bars.o_empty[wg]));
+      if (lane == 0) {
+        mbar_arrive(bar(bars.o_empty[wg]));
+        if (split) mbar_arrive(bar(bars.o_empty[1]));
+      }
     }
     if (!ok && lane == 0) {
       *abort_flag = 1;
@@ -1111,6 +1214,7 @@ __device__ __forceinline__ void merge_row_warp(const MergeParams& p, const Merge
 // Grid-stride over (split group, row) items, one warp per item.
 template <int D>
 __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const MergeParams p) {
+
   // the attention kernel has finished: re-arm the work counter so that the same
   // plan can serve the next run
   if (blockIdx.x == 0 && threadIdx.x == 0) p.hdr->counter = 0;
