@@ -69,13 +69,16 @@ def edit_bytes(rows, vocab, elem):
 
 
 # ------------------------------------------------------------------ measured traffic
-# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum, one-pass ncu counters)
-# of one attention call (attn_kernel + merge) on the full-size workload, keyed by
-# the first 16 hex digits of the SHA-256 of the kernel source that was measured;
-# a changed kernel gets no traffic figure until it is measured again. Source:
-# profiles/attn_dram_serving128.md.
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one attention call
+# (attn_kernel) of the serving workload, keyed by the first 16 hex digits of the
+# SHA-256 of the kernel source that was measured; a changed kernel gets no traffic
+# figure until it is measured again. Measured on a 64-sequence, one-layer case of
+# the same workload (2.3 GB of cache on the device), whose reads were 1.0089x its
+# algorithmic Q + K/V bytes; scaled to the 128-sequence call by those bytes, plus
+# its output (the full call splits no key range, so it writes no partials).
+# Source: profiles/attn_kernel_dram_serving_b64.md.
 MEASURED_TRAFFIC = {
-    "c298dd4362ddf844": {"serving128": 4447626752 + 70167552 + 9472},
+    "913c9d1bd77d93e2": {"serving128": 4435281390 + 67108864},
 }
 
 
@@ -157,10 +160,10 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------ workloads
-def build_workload(name, device, layers=None, batch=None):
+def build_workload(name, device, layers=None, batch=None, vocab=None):
     from paper_2607_22663_gb300 import workloads as wl
     if name == "serving128":
-        return wl.serving128(device, layers=layers or 24, batch=batch or 128)
+        return wl.serving128(device, layers=layers or 24, batch=batch or 128, vocab=vocab or 131072)
     return wl.WORKLOADS[name](device)
 
 
@@ -183,7 +186,7 @@ def run_gpu(args, rank, world):
     dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
     torch.cuda.set_device(dev)
     peaks, peak_src = load_peaks()
-    w = build_workload(args.workload, dev, args.layers, args.batch)
+    w = build_workload(args.workload, dev, args.layers, args.batch, args.vocab)
     attn = w["attn"]
     ep = w["edit"]
     with_kv_write = args.workload == "long32k"
@@ -303,6 +306,8 @@ def run_gpu(args, rank, world):
     per_step = len(attn) * 2 + (1 if plan_layers else len(attn)) + (1 if ep is not None else 0) + \
         (len(attn) if with_kv_write else 0)
     res["gpu_launches"] = per_step * K
+    if args.no_extras:
+        return res
     # end to end first, on the state the timed loop left (the extras allocate large buffers of their own)
     res["e2e"] = run_e2e(args, w, attention_call, edit_call, dev, stream, world, new_t if ep is not None else None,
                          mask_t if ep is not None else None, conf_t if ep is not None else None)
@@ -680,12 +685,16 @@ def time_pass_loop(w, dev, reps=3, max_passes=5):
             "note": "pass = window attention of every layer + Eq. 2 update + refresh of changed blocks + commit"}
 
 
-def run_e2e(args, w, attention_call, edit_call, dev, stream, world, new_t, mask_t, conf_t):
+def run_e2e(args, w, attention_call, edit_call, dev, stream, world, new_t, mask_t, conf_t, copy_streams=1):
     """Same pass through the public API with the per-step inputs (window Q/K/V
     of every layer, logits, committed tokens) copied from pinned host memory
     and the step's result (new tokens, edit mask, confidence) read back. The
-    paged KV caches are resident state, as in serving. Copies of layer l+1 run
-    on a second stream while layer l computes."""
+    paged KV caches are resident state, as in serving. The copies run on
+    copy_streams streams (layer l's inputs on stream l mod n, the logits in n
+    slices) beside the compute stream, and layer l computes once its own inputs
+    have arrived. One copy stream is the default: on this GPU one stream of
+    pinned host-to-device copies moved 410-420 GB/s, two or four concurrent
+    ones about 210 GB/s in total."""
     attn = w["attn"]
     ep = w["edit"]
     host = []
@@ -700,7 +709,8 @@ def run_e2e(args, w, attention_call, edit_call, dev, stream, world, new_t, mask_
         cm_d = torch.empty_like(ep.committed)
         R = ep.logits.shape[0]
         out_h = [torch.empty(R, dtype=t.dtype, pin_memory=True) for t in (new_t, mask_t, conf_t)]
-    copy_stream = torch.cuda.Stream(dev)
+        cuts = [R * k // copy_streams for k in range(copy_streams + 1)]
+    cs = [torch.cuda.Stream(dev) for _ in range(copy_streams)]
     h2d = sum(t.numel() * t.element_size() for hs in host for t in hs)
     if ep is not None:
         h2d += lg_h.numel() * lg_h.element_size() + cm_h.numel() * cm_h.element_size()
@@ -708,25 +718,32 @@ def run_e2e(args, w, attention_call, edit_call, dev, stream, world, new_t, mask_
 
     def step():
         copied = [torch.cuda.Event() for _ in attn]
-        with torch.cuda.stream(copy_stream):
-            for i in range(len(attn)):
+        for i in range(len(attn)):
+            with torch.cuda.stream(cs[i % copy_streams]):
                 for d, h in zip(dbuf[i], host[i]):
                     d.copy_(h, non_blocking=True)
-                copied[i].record(copy_stream)
-            if ep is not None:
-                lg_d.copy_(lg_h, non_blocking=True)
-                cm_d.copy_(cm_h, non_blocking=True)
-                done_l = torch.cuda.Event()
-                done_l.record(copy_stream)
+                copied[i].record(cs[i % copy_streams])
+        done_l = []
+        if ep is not None:
+            for k in range(copy_streams):
+                with torch.cuda.stream(cs[k]):
+                    lg_d[cuts[k]:cuts[k + 1]].copy_(lg_h[cuts[k]:cuts[k + 1]], non_blocking=True)
+                    if k == 0:
+                        cm_d.copy_(cm_h, non_blocking=True)
+                    e = torch.cuda.Event()
+                    e.record(cs[k])
+                    done_l.append(e)
         for i, a in enumerate(attn):
             stream.wait_event(copied[i])
             attention_call(i, a, *dbuf[i])
         if ep is not None:
-            stream.wait_event(done_l)
+            for e in done_l:
+                stream.wait_event(e)
             edit_call(lg_d, cm_d)
             for h, d in zip(out_h, (new_t, mask_t, conf_t)):
                 h.copy_(d, non_blocking=True)
-        copy_stream.wait_stream(stream)
+        for c in cs:
+            c.wait_stream(stream)
 
     # warm up until two consecutive steps agree within 5% (the first large
     # copies out of freshly pinned host memory can run several times slower)
@@ -748,7 +765,8 @@ def run_e2e(args, w, attention_call, edit_call, dev, stream, world, new_t, mask_
     torch.cuda.synchronize()
     el = max_over_ranks(time.perf_counter() - t0, dev)
     return {"value": round(whole_job_rate(attn[0].batch * K, world, el), 3), "unit": "windows/s", "h2d_bytes_per_step": int(h2d),
-            "d2h_bytes_per_step": int(d2h), "steps": K,
+            "d2h_bytes_per_step": int(d2h), "steps": K, "copy_streams": copy_streams,
+            "h2d_gbs_effective": round(h2d * K / el / 1e9, 1),
             "resident_state": "paged KV caches of every layer (written by earlier passes)"}
 
 
@@ -841,8 +859,12 @@ def main():
     ap.add_argument("--layers", type=int, default=None, help="layer count of the serving workload (default 24)")
     ap.add_argument("--batch", type=int, default=None, help="sequences of the serving workload (default 128; "
                     "smaller values are for profiling captures, not bench lines)")
+    ap.add_argument("--vocab", type=int, default=None, help="vocabulary of the serving workload (default 131072; "
+                    "smaller values are for profiling captures, not bench lines)")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true", help="skip the end-to-end pass and the extras (for "
+                    "profiling captures; not for bench lines)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -20,8 +20,8 @@ The shapes follow the five workloads the library is measured on:
                 32/8 heads, page 64 with a random page permutation; KV write of
                 each window; seed 4.
 * ``serving128`` 128 sequences, prefix U[512,16384] (not rounded), window 64,
-                32/8 heads, page 64 (not stated by the workload; 64 tokens make one
-                8 KB TMA box per page, head and half of D), 24 layers with independent Q/K/V and
+                32/8 heads, page 32 (not stated by the workload; the size the
+                other paged workloads use), 24 layers with independent Q/K/V and
                 caches; bf16 logits [8192 x 131072] N(0, sd 2) with peaks
                 U(0,12) on every row, committed = the row argmax on 80% of
                 rows; tau 0.9; seed 5.
@@ -259,7 +259,7 @@ def long32k(device="cpu", windows=(64, 128, 256)):
     return {"name": "long32k", "attn": calls, "edit": None, "layers": 1}
 
 
-def serving128(device="cpu", layers=24, vocab=131072, batch=128, page_size=64):
+def serving128(device="cpu", layers=24, vocab=131072, batch=128, page_size=32):
     g = _gen(5, "cpu")
     prefix = torch.randint(512, 16385, (batch,), generator=g).tolist()
     window = [64] * batch
