@@ -521,6 +521,25 @@ mbe_status mbe_gather_rows(const void* src, int64_t src_rows, int64_t row_bytes,
                            int64_t rows, const int32_t* rows_used_or_null, void* dst, cudaStream_t stream);
 
 /*
+ * mbe_gather_rows_multi -- mbe_gather_rows for n_tensors (1..MBE_GATHER_MAX)
+ * tensors that share one row map, in one launch: dsts[t][k] =
+ * srcs[t][src_row[k]] for rows of row_bytes[t] bytes, with the zero rows, the
+ * MBE_DEVERR_LENGTH flag and the rows_used_or_null limit of mbe_gather_rows.
+ * This is how the refresh batch of Sec. 4.3 compacts a layer's Q, K and V
+ * together. srcs, row_bytes and dsts are host arrays of n_tensors entries;
+ * the buffers they point to are device buffers with src_rows source rows and
+ * at least `rows` destination rows, none overlapping. When every row is a
+ * whole number of 16-byte chunks and every buffer is 16-byte aligned the copy
+ * is one kernel launch; otherwise it is one mbe_gather_rows per tensor.
+ * Errors: MBE_ERR_INVALID_ARG (n_tensors out of range, null pointers,
+ * negative sizes), MBE_ERR_CUDA.
+ */
+#define MBE_GATHER_MAX 4
+mbe_status mbe_gather_rows_multi(int32_t n_tensors, const void* const* srcs, const int64_t* row_bytes,
+                                 void* const* dsts, int64_t src_rows, const int32_t* src_row, int64_t rows,
+                                 const int32_t* rows_used_or_null, cudaStream_t stream);
+
+/*
  * Editing-pass loop on the device. Paper: Sec. 4.1 (the window is edited by
  * repeated passes until a pass changes no token or N_MBE passes have run) and
  * Sec. 4.3 (one graph serves every shape of the pass).

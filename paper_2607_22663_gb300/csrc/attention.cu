@@ -1141,92 +1141,120 @@ struct MergeParams {
   int Hq, G;
 };
 
-// One warp per packed query row of a split group: lane l holds D/32
-// consecutive output columns, so every partial row is read as one coalesced
-// 4 D-byte line; the weights 2^(lse_k - M) are common to the row.
+// One warp per block of kMergeRows packed query rows of a split group: lane l
+// holds D/32 consecutive output columns of every row, so every partial row is
+// read as one coalesced 4 D-byte line; the loads of all rows of the block and of
+// kMergeBatch splits are issued before any is used, so that groups with few
+// splits still keep several lines per warp in flight.
+constexpr int kMergeRows = 4;
+constexpr int kMergeBatch = 2;
+
 template <int D>
-__device__ __forceinline__ void merge_row_warp(const MergeParams& p, const MergeGroup& grp, int r, int lane) {
+__device__ __forceinline__ void merge_rows_warp(const MergeParams& p, const MergeGroup& grp, int r0, int lane) {
   constexpr int kPer = D / 32;  // 4 for D = 128, 2 for D = 64
-  const int R = grp.row0 + r;
-  const int qi = R / p.G, hh = R - qi * p.G;
-  if (qi >= grp.window) return;
   const int cu = p.cu_window[grp.seq];
   if (cu < 0 || static_cast<int64_t>(cu) + grp.window > p.total_tokens) return;
-  const float* lse = p.part_lse + static_cast<int64_t>(grp.slot_base) * kUnitRows + r;  // split k at k * kUnitRows
-  const float* part = p.part_o + (static_cast<int64_t>(grp.slot_base) * kUnitRows + r) * D + lane * kPer;
+  bool live[kMergeRows];
+  int64_t orow[kMergeRows];
+  bool any = false;
+#pragma unroll
+  for (int rr = 0; rr < kMergeRows; ++rr) {
+    const int R = grp.row0 + r0 + rr;
+    const int qi = R / p.G, hh = R - qi * p.G;
+    live[rr] = qi < grp.window;
+    any |= live[rr];
+    orow[rr] = static_cast<int64_t>(cu + qi) * p.Hq + grp.kv_head * p.G + hh;
+  }
+  if (!any) return;
+  // partial row r of split k: lse at (slot_base + k) * kUnitRows + r, O at that row * D
+  const int64_t base = static_cast<int64_t>(grp.slot_base) * kUnitRows + r0;
   const int n = grp.n_splits;
-  // Online merge: eight splits per step, all their loads issued before any is
-  // used; the running maximum M of the splits' log-sum-exps rescales what has
-  // been summed so far when it grows (one pass over the partials).
-  constexpr int kBatch = 8;
-  float M = neg_inf(), wsum = 0.f;
-  float acc[kPer];
+  // Online merge: the running maximum M of the splits' log-sum-exps rescales
+  // what has been summed so far when it grows (one pass over the partials).
+  float M[kMergeRows], wsum[kMergeRows], acc[kMergeRows][kPer];
 #pragma unroll
-  for (int d = 0; d < kPer; ++d) acc[d] = 0.f;
-  for (int k0 = 0; k0 < n; k0 += kBatch) {
-    float lk[kBatch], v[kBatch][kPer];
+  for (int rr = 0; rr < kMergeRows; ++rr) {
+    M[rr] = neg_inf();
+    wsum[rr] = 0.f;
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) {
+    for (int d = 0; d < kPer; ++d) acc[rr][d] = 0.f;
+  }
+  for (int k0 = 0; k0 < n; k0 += kMergeBatch) {
+    float lk[kMergeRows][kMergeBatch], v[kMergeRows][kMergeBatch][kPer];
+#pragma unroll
+    for (int u = 0; u < kMergeBatch; ++u) {
       const int k = k0 + u;
-      lk[u] = neg_inf();
 #pragma unroll
-      for (int d = 0; d < kPer; ++d) v[u][d] = 0.f;
-      if (k < n) {
-        lk[u] = lse[static_cast<int64_t>(k) * kUnitRows];
-        const float* src = part + static_cast<int64_t>(k) * kUnitRows * D;
-        if constexpr (kPer == 4) {
-          const float4 x = *reinterpret_cast<const float4*>(src);
-          v[u][0] = x.x; v[u][1] = x.y; v[u][2] = x.z; v[u][3] = x.w;
-        } else {
-          const float2 x = *reinterpret_cast<const float2*>(src);
-          v[u][0] = x.x; v[u][1] = x.y;
+      for (int rr = 0; rr < kMergeRows; ++rr) {
+        lk[rr][u] = neg_inf();
+#pragma unroll
+        for (int d = 0; d < kPer; ++d) v[rr][u][d] = 0.f;
+        if (k < n && live[rr]) {
+          const int64_t row = base + static_cast<int64_t>(k) * kUnitRows + rr;
+          lk[rr][u] = p.part_lse[row];
+          const float* src = p.part_o + row * D + lane * kPer;
+          if constexpr (kPer == 4) {
+            const float4 x = *reinterpret_cast<const float4*>(src);
+            v[rr][u][0] = x.x; v[rr][u][1] = x.y; v[rr][u][2] = x.z; v[rr][u][3] = x.w;
+          } else {
+            const float2 x = *reinterpret_cast<const float2*>(src);
+            v[rr][u][0] = x.x; v[rr][u][1] = x.y;
+          }
         }
       }
     }
-    float mb = lk[0];
 #pragma unroll
-    for (int u = 1; u < kBatch; ++u) mb = fmaxf(mb, lk[u]);
-    if (mb > M) {
-      const float c = (M == neg_inf()) ? 0.f : ex2f(M - mb);
-      wsum *= c;
+    for (int rr = 0; rr < kMergeRows; ++rr) {
+      float mb = lk[rr][0];
 #pragma unroll
-      for (int d = 0; d < kPer; ++d) acc[d] *= c;
-      M = mb;
-    }
+      for (int u = 1; u < kMergeBatch; ++u) mb = fmaxf(mb, lk[rr][u]);
+      if (mb > M[rr]) {
+        const float c = (M[rr] == neg_inf()) ? 0.f : ex2f(M[rr] - mb);
+        wsum[rr] *= c;
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) {
-      const float w = (lk[u] == neg_inf()) ? 0.f : ex2f(lk[u] - M);
-      wsum += w;
+        for (int d = 0; d < kPer; ++d) acc[rr][d] *= c;
+        M[rr] = mb;
+      }
 #pragma unroll
-      for (int d = 0; d < kPer; ++d) acc[d] += w * v[u][d];
+      for (int u = 0; u < kMergeBatch; ++u) {
+        const float w = (lk[rr][u] == neg_inf()) ? 0.f : ex2f(lk[rr][u] - M[rr]);
+        wsum[rr] += w;
+#pragma unroll
+        for (int d = 0; d < kPer; ++d) acc[rr][d] += w * v[rr][u][d];
+      }
     }
   }
-  const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
-  const int64_t orow = static_cast<int64_t>(cu + qi) * p.Hq + grp.kv_head * p.G + hh;
-  __nv_bfloat16* dst = p.out + orow * D + lane * kPer;
-  if constexpr (kPer == 4)
-    *reinterpret_cast<uint2*>(dst) = make_uint2(pack_bf16x2(acc[0] * inv, acc[1] * inv), pack_bf16x2(acc[2] * inv, acc[3] * inv));
-  else
-    *reinterpret_cast<uint32_t*>(dst) = pack_bf16x2(acc[0] * inv, acc[1] * inv);
-  if (p.lse && lane == 0) p.lse[orow] = (wsum > 0.f ? M + __log2f(wsum) : neg_inf()) * 0.6931471805599453f;
+#pragma unroll
+  for (int rr = 0; rr < kMergeRows; ++rr) {
+    if (!live[rr]) continue;
+    const float inv = wsum[rr] > 0.f ? 1.f / wsum[rr] : 0.f;
+    __nv_bfloat16* dst = p.out + orow[rr] * D + lane * kPer;
+    if constexpr (kPer == 4)
+      *reinterpret_cast<uint2*>(dst) = make_uint2(pack_bf16x2(acc[rr][0] * inv, acc[rr][1] * inv),
+                                                  pack_bf16x2(acc[rr][2] * inv, acc[rr][3] * inv));
+    else
+      *reinterpret_cast<uint32_t*>(dst) = pack_bf16x2(acc[rr][0] * inv, acc[rr][1] * inv);
+    if (p.lse && lane == 0)
+      p.lse[orow[rr]] = (wsum[rr] > 0.f ? M[rr] + __log2f(wsum[rr]) : neg_inf()) * 0.6931471805599453f;
+  }
 }
 
-// Grid-stride over (split group, row) items, one warp per item.
+// Grid-stride over (split group, block of kMergeRows rows) items, one warp per item.
 template <int D>
-__global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const MergeParams p) {
-
+__global__ void __launch_bounds__(kMergeThreads, 2) attn_merge_kernel(const MergeParams p) {
   // the attention kernel has finished: re-arm the work counter so that the same
   // plan can serve the next run
   if (blockIdx.x == 0 && threadIdx.x == 0) p.hdr->counter = 0;
   if (!sig_equal(p.hdr->sig, p.sig)) return;
-  const int64_t n_items = static_cast<int64_t>(p.hdr->n_groups) * kUnitRows;
+  constexpr int kBlocks = kUnitRows / kMergeRows;
+  const int64_t n_items = static_cast<int64_t>(p.hdr->n_groups) * kBlocks;
   const int lane = threadIdx.x & 31;
   const int64_t warps = static_cast<int64_t>(gridDim.x) * (kMergeThreads / 32);
   for (int64_t it = static_cast<int64_t>(blockIdx.x) * (kMergeThreads / 32) + threadIdx.x / 32; it < n_items;
        it += warps) {
-    const MergeGroup grp = p.groups[it / kUnitRows];
+    const MergeGroup grp = p.groups[it / kBlocks];
     if (grp.seq < 0 || grp.seq >= p.batch) continue;
-    merge_row_warp<D>(p, grp, static_cast<int>(it % kUnitRows), lane);
+    merge_rows_warp<D>(p, grp, static_cast<int>(it % kBlocks) * kMergeRows, lane);
   }
 }
 
@@ -1357,8 +1385,8 @@ mbe_status run(const void* q, const void* k_win, const void* v_win, const void* 
   if (launch_status("attn_kernel launch") != MBE_OK) return MBE_ERR_CUDA;
   MergeParams mp{sig, batch, total_q_tokens, hdr, reinterpret_cast<const MergeGroup*>(ws + L.groups), ap.part_o,
                  ap.part_lse, cu_window, ap.out, lse, Hq, G};
-  const int64_t merge_grid =
-      std::max<int64_t>(1, std::min<int64_t>(L.max_groups * (kUnitRows / (kMergeThreads / 32)), 2 * di->num_sms));
+  const int64_t merge_grid = std::max<int64_t>(
+      1, std::min<int64_t>(L.max_groups * (kUnitRows / kMergeRows / (kMergeThreads / 32)), 2 * di->num_sms));
   attn_merge_kernel<D><<<static_cast<unsigned>(merge_grid), kMergeThreads, 0, stream>>>(mp);
   if (launch_status("attn_merge_kernel launch") != MBE_OK) return MBE_ERR_CUDA;
   return MBE_OK;

@@ -138,6 +138,40 @@ __global__ void __launch_bounds__(256) gather_rows_kernel(const V* __restrict__ 
   }
 }
 
+// The same for up to MBE_GATHER_MAX tensors sharing one row map, 16-byte
+// chunks: chunk c of a destination row belongs to tensor t where
+// off[t] <= c < off[t + 1] (off[t] = chunks per row of the tensors before t).
+struct GatherSet {
+  const uint4* src[MBE_GATHER_MAX];
+  uint4* dst[MBE_GATHER_MAX];
+  int64_t elems[MBE_GATHER_MAX];     // 16-byte chunks per row of tensor t
+  int64_t off[MBE_GATHER_MAX + 1];
+  int n;
+};
+
+__global__ void __launch_bounds__(256) gather_rows_multi_kernel(const GatherSet g, int64_t src_rows,
+                                                                const int32_t* __restrict__ map, int64_t rows,
+                                                                const int32_t* __restrict__ rows_used) {
+  if (rows_used) rows = min(rows, static_cast<int64_t>(max(*rows_used, 0)));
+  const int64_t per_row = g.off[g.n];
+  const int64_t total = rows * per_row;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < total; i += stride) {
+    const int64_t k = i / per_row, c = i - k * per_row;
+    int t = 0;
+#pragma unroll
+    for (int u = 1; u < MBE_GATHER_MAX; ++u) t += (u < g.n && c >= g.off[u]) ? 1 : 0;
+    const int64_t cc = c - g.off[t];
+    const int32_t r = map[k];
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (r >= 0 && r < src_rows)
+      v = g.src[t][r * g.elems[t] + cc];
+    else if (r >= src_rows && c == 0)
+      atomicOr(&g_error_word, MBE_DEVERR_LENGTH);
+    g.dst[t][k * g.elems[t] + cc] = v;
+  }
+}
+
 // Ends a pass: counts it and keeps the loop going while some sequence changed
 // a token and fewer than max_passes passes have run.
 __global__ void __launch_bounds__(256) pass_loop_condition_kernel(cudaGraphConditionalHandle handle,
@@ -228,6 +262,50 @@ extern "C" mbe_status mbe_gather_rows(const void* src, int64_t src_rows, int64_t
     gather_rows_kernel<uint8_t><<<g, 256, 0, stream>>>(static_cast<const uint8_t*>(src), src_rows, row_bytes,
                                                        src_row, rows, rows_used_or_null, static_cast<uint8_t*>(dst));
   return launch_status("gather_rows_kernel");
+}
+
+extern "C" mbe_status mbe_gather_rows_multi(int32_t n_tensors, const void* const* srcs, const int64_t* row_bytes,
+                                            void* const* dsts, int64_t src_rows, const int32_t* src_row,
+                                            int64_t rows, const int32_t* rows_used_or_null, cudaStream_t stream) {
+  using namespace mbe;
+  if (n_tensors < 1 || n_tensors > MBE_GATHER_MAX || !srcs || !row_bytes || !dsts || src_rows < 0 || rows < 0)
+    return MBE_ERR_INVALID_ARG;
+  bool vec = true;
+  for (int t = 0; t < n_tensors; ++t) {
+    if (row_bytes[t] < 1 || !dsts[t] || (src_rows > 0 && !srcs[t])) return MBE_ERR_INVALID_ARG;
+    const uintptr_t a = reinterpret_cast<uintptr_t>(srcs[t]) | reinterpret_cast<uintptr_t>(dsts[t]);
+    vec &= row_bytes[t] % 16 == 0 && a % 16 == 0;
+  }
+  if (rows == 0) return MBE_OK;
+  if (!src_row) return MBE_ERR_INVALID_ARG;
+  if (!vec) {  // rows that are not whole 16-byte chunks: one copy per tensor
+    for (int t = 0; t < n_tensors; ++t) {
+      const mbe_status st =
+          mbe_gather_rows(srcs[t], src_rows, row_bytes[t], src_row, rows, rows_used_or_null, dsts[t], stream);
+      if (st != MBE_OK) return st;
+    }
+    return MBE_OK;
+  }
+  GatherSet g{};
+  g.n = n_tensors;
+  g.off[0] = 0;
+  for (int t = 0; t < n_tensors; ++t) {
+    g.src[t] = static_cast<const uint4*>(srcs[t]);
+    g.dst[t] = static_cast<uint4*>(dsts[t]);
+    g.elems[t] = row_bytes[t] / 16;
+    g.off[t + 1] = g.off[t] + g.elems[t];
+  }
+  for (int t = n_tensors; t < MBE_GATHER_MAX; ++t) g.off[t + 1] = g.off[t];
+  const int sms = sm_count();
+  if (sms == 0) {
+    record_cuda_error(cudaGetLastError(), "cudaDeviceGetAttribute");
+    return MBE_ERR_CUDA;
+  }
+  int64_t ctas = (rows * g.off[n_tensors] + 255) / 256;
+  if (ctas > 4 * sms) ctas = 4 * sms;
+  gather_rows_multi_kernel<<<static_cast<unsigned>(ctas), 256, 0, stream>>>(g, src_rows, src_row, rows,
+                                                                             rows_used_or_null);
+  return launch_status("gather_rows_multi_kernel");
 }
 
 struct mbe_pass_loop {

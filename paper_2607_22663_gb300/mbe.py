@@ -98,6 +98,8 @@ def lib(build_if_missing: bool = True):
     L.mbe_refresh_plan.argtypes = [P, i32, P, P, P, P, i32, i32, i32, i32, i32, P, P, P, P, P, P, P, P]
     L.mbe_gather_rows.restype = ctypes.c_int
     L.mbe_gather_rows.argtypes = [P, i64, i64, P, i64, P, P, P]
+    L.mbe_gather_rows_multi.restype = ctypes.c_int
+    L.mbe_gather_rows_multi.argtypes = [i32, P, P, P, i64, P, i64, P, P]
     L.mbe_pass_loop_begin.restype = ctypes.c_int
     L.mbe_pass_loop_begin.argtypes = [i32, P, P, ctypes.POINTER(ctypes.c_void_p)]
     L.mbe_pass_loop_until_stable.restype = ctypes.c_int
@@ -534,6 +536,37 @@ def gather_rows(src, src_row, out=None, rows_used=None, stream=None):
                                _ptr(rows_used) if rows_used is not None else None, _ptr(out), _stream(stream))
     _check("mbe_gather_rows", st)
     return out
+
+
+def gather_rows_multi(pairs, src_row, rows_used=None, stream=None):
+    """mbe_gather_rows_multi: out[k] = src[src_row[k]] for every (src, out) in
+    `pairs` (at most 4 tensors with the same number of rows), one launch."""
+    _need(src_row, "src_row", torch.int32)
+    rows = src_row.numel()
+    if not 1 <= len(pairs) <= 4:
+        raise ValueError("gather_rows_multi takes 1 to 4 (src, out) pairs")
+    src_rows = pairs[0][0].shape[0]
+    srcs, dsts, nbytes = [], [], []
+    for src, out in pairs:
+        _need(src, "src", None)
+        _need(out, "out", src.dtype)
+        if src.shape[0] != src_rows:
+            raise ValueError("every src must have the same number of rows")
+        if tuple(out.shape[1:]) != tuple(src.shape[1:]) or out.shape[0] != rows:
+            raise ValueError("out must be [len(src_row)] + src.shape[1:]")
+        srcs.append(src.data_ptr())
+        dsts.append(out.data_ptr())
+        nbytes.append(max(1, (src[0].numel() if src_rows else out[0].numel() if rows else 1) * src.element_size()))
+    if rows_used is not None:
+        _need(rows_used, "rows_used", torch.int32)
+    n = len(pairs)
+    c_src = (ctypes.c_void_p * n)(*srcs)
+    c_dst = (ctypes.c_void_p * n)(*dsts)
+    c_bytes = (ctypes.c_int64 * n)(*nbytes)
+    st = lib().mbe_gather_rows_multi(n, c_src, c_bytes, c_dst, src_rows, _ptr(src_row), rows,
+                                     _ptr(rows_used) if rows_used is not None else None, _stream(stream))
+    _check("mbe_gather_rows_multi", st)
+    return [out for _, out in pairs]
 
 
 class PassLoop:

@@ -103,6 +103,42 @@ def test_gather_rows(shape, dtype):
     assert mbe.get_device_error() == (0, 0)
 
 
+def test_gather_rows_multi():
+    """One launch for several tensors sharing a row map equals one gather per
+    tensor; rows that are not whole 16-byte chunks take the per-tensor path."""
+    g = torch.Generator().manual_seed(11)
+    R, n = 45, 70
+    idx = torch.randint(-1, R, (n,), generator=g, dtype=torch.int32)
+    sets = [[torch.randn(R, 4, 128, generator=g).to(torch.bfloat16), torch.randn(R, 2, 128, generator=g).to(torch.bfloat16),
+             torch.randn(R, 2, 64, generator=g).to(torch.bfloat16)],
+            [torch.randint(0, 9, (R,), generator=g, dtype=torch.int32), torch.randn(R, 2, 128, generator=g).to(torch.bfloat16)],
+            [torch.randint(0, 255, (R, 3), generator=g).to(torch.uint8)]]
+    for srcs in sets:
+        d_srcs = [x.to(DEV) for x in srcs]
+        outs = [torch.full((n,) + x.shape[1:], 7, dtype=x.dtype, device=DEV) for x in srcs]
+        mbe.gather_rows_multi(list(zip(d_srcs, outs)), idx.to(DEV))
+        for x, o in zip(srcs, outs):
+            ref = torch.zeros((n,) + x.shape[1:], dtype=x.dtype)
+            ok = idx >= 0
+            ref[ok] = x[idx[ok].long()]
+            assert torch.equal(o.cpu(), ref)
+        assert mbe.get_device_error() == (0, 0)
+        # a device row count leaves the rows from it on untouched; an index past the
+        # source gives a zero row and the length flag
+        bad = idx.clone()
+        bad[2] = R + 3
+        cnt = torch.tensor([33], dtype=torch.int32, device=DEV)
+        outs2 = [torch.full_like(o, 5) for o in outs]
+        mbe.gather_rows_multi(list(zip(d_srcs, outs2)), bad.to(DEV), rows_used=cnt)
+        for o, o2 in zip(outs, outs2):
+            got = o2.cpu()
+            assert not got[2].any() and torch.equal(got[3:33], o.cpu()[3:33]) and (got[33:] == 5).all()
+        st, flags = mbe.get_device_error()
+        assert flags == mbe.DEVERR_LENGTH
+    with pytest.raises(ValueError):
+        mbe.gather_rows_multi([], idx.to(DEV))
+
+
 def _refresh_problem(seed):
     B = 32
     prefix, window = [100, 0, 2000, 517, 64], [64, 96, 33, 128, 32]
@@ -156,9 +192,10 @@ def _gpu_refresh(prob, old, changed, B, stream=None, bufs=None):
     plan = mbe.refresh_plan(bufs["changed"], d.prefix_len, d.window_len, d.cu_window, d.block_table, block_size=B,
                             max_window=mw, total_rows=T, out=bufs["plan"], stream=stream)
     bufs["plan"] = plan
-    for src, dst in ((d.q, bufs["q"]), (d.k_win, bufs["k"]), (d.v_win, bufs["v"])):
-        # only the refresh rows are gathered; the rest of the buffers are never read
-        mbe.gather_rows(src, plan["src_row"], out=dst, rows_used=plan["count"][1:], stream=stream)
+    # only the refresh rows are gathered (Q, K and V in one launch); the rest of the
+    # buffers are never read
+    mbe.gather_rows_multi([(d.q, bufs["q"]), (d.k_win, bufs["k"]), (d.v_win, bufs["v"])], plan["src_row"],
+                          rows_used=plan["count"][1:], stream=stream)
     mbe.kv_window_write(bufs["k"], bufs["v"], d.k_cache, d.v_cache, plan["block_table"], plan["prefix_len"],
                         plan["window_len"], plan["cu_window"], block_size=B, max_window=B, stream=stream)
     mbe.window_attention(bufs["q"], bufs["k"], bufs["v"], d.k_cache, d.v_cache, plan["block_table"],
