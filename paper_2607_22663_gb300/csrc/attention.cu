@@ -1073,25 +1073,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int cu = p.cu_window[wu.seq];
         __nv_bfloat16* orow =
             p.out + (static_cast<int64_t>(cu + qi) * p.Hq + wu.kv_head * p.G + hh) * D;
+        // O / l as bf16, 32 columns per TMEM load, with 32-byte stores: the row is
+        // 32-byte aligned and each store fills one sector
 #pragma unroll
         for (int c = 0; c < D / 32; ++c) {
           uint32_t o[32];
           tmem_ld32(tO + 32 * c, o);
           if (valid) {
-            uint4* dst = reinterpret_cast<uint4*>(orow + 32 * c);
+            uint32_t w[16];
 #pragma unroll
-            for (int v = 0; v < 4; ++v) {
-              uint4 w;
-              w.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv_l, __uint_as_float(o[8 * v + 1]) * inv_l);
-              w.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv_l, __uint_as_float(o[8 * v + 3]) * inv_l);
-              w.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv_l, __uint_as_float(o[8 * v + 5]) * inv_l);
-              w.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv_l, __uint_as_float(o[8 * v + 7]) * inv_l);
-              dst[v] = w;
-            }
+            for (int k = 0; k < 16; ++k)
+              w[k] = pack_bf16x2(__uint_as_float(o[2 * k]) * inv_l, __uint_as_float(o[2 * k + 1]) * inv_l);
+#pragma unroll
+            for (int v = 0; v < 2; ++v)
+              st_global_v8(orow + 32 * c + 16 * v, w[8 * v], w[8 * v + 1], w[8 * v + 2], w[8 * v + 3], w[8 * v + 4],
+                           w[8 * v + 5], w[8 * v + 6], w[8 * v + 7]);
           }
         }
         if (valid && p.lse) p.lse[static_cast<int64_t>(cu + qi) * p.Hq + wu.kv_head * p.G + hh] = lse2 * 0.6931471805599453f;
       } else {
+        // split piece: fp32 O / l and the log2-sum-exp, merged afterwards
         const int prow = kTileRows * wg + r;
         float* po = p.part_o + (static_cast<int64_t>(wu.slot) * kUnitRows + prow) * D;
 #pragma unroll
@@ -1099,11 +1100,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           uint32_t o[32];
           tmem_ld32(tO + 32 * c, o);
           if (valid) {
-            float4* dst = reinterpret_cast<float4*>(po + 32 * c);
 #pragma unroll
-            for (int v = 0; v < 8; ++v)
-              dst[v] = make_float4(__uint_as_float(o[4 * v]) * inv_l, __uint_as_float(o[4 * v + 1]) * inv_l,
-                                   __uint_as_float(o[4 * v + 2]) * inv_l, __uint_as_float(o[4 * v + 3]) * inv_l);
+            for (int v = 0; v < 4; ++v) {
+              uint32_t w[8];
+#pragma unroll
+              for (int k = 0; k < 8; ++k) w[k] = __float_as_uint(__uint_as_float(o[8 * v + k]) * inv_l);
+              st_global_v8(po + 32 * c + 8 * v, w[0], w[1], w[2], w[3], w[4], w[5], w[6], w[7]);
+            }
           }
         }
         if (valid) p.part_lse[static_cast<int64_t>(wu.slot) * kUnitRows + prow] = lse2;
