@@ -166,23 +166,43 @@ __device__ __forceinline__ int cost_bucket(int cost, int chunk) {
 }
 
 __global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p) {
-  __shared__ int s_total, s_nunits, s_ngroups, s_nslots, s_bad;
+  __shared__ int s_total, s_nunits, s_ngroups, s_nslots, s_bad, s_tmin, s_tmax, s_nslab, s_sigma;
   __shared__ int hist[kBuckets];
   __shared__ int warp_sums[32];
   const int tid = threadIdx.x;
-  if (tid == 0) { s_total = 0; s_nunits = 0; s_ngroups = 0; s_nslots = 0; s_bad = 0; }
+  if (tid == 0) {
+    s_total = 0; s_nunits = 0; s_ngroups = 0; s_nslots = 0; s_bad = 0;
+    s_tmin = 0x7FFFFFFF; s_tmax = 0; s_nslab = 0; s_sigma = 0;
+  }
   for (int b = tid; b < kBuckets; b += blockDim.x) hist[b] = 0;
   __syncthreads();
-  // pass 1: validate and count key tiles and (sequence, KV head) pairs
-  int local = 0, bad = 0;
+  // pass 1: validate and count key tiles and slabs; the shortest and longest slab
+  int local = 0, bad = 0, nslab = 0, tmin = 0x7FFFFFFF, tmax = 0;
   for (int s = tid; s < p.batch; s += blockDim.x) {
     const int P = seq_prefix(p, s), W = p.window_len[s], mode = seq_mode(p, s);
     if (!seq_ok(p, s, P, W, mode)) { bad = 1; continue; }
     const int slabs = (W * p.G + kUnitRows - 1) / kUnitRows;
-    for (int sl = 0; sl < slabs; ++sl) local += slab_tiles(P, W, mode, sl * kUnitRows, p.G, p.block_size) * p.Hkv;
+    for (int sl = 0; sl < slabs; ++sl) {
+      const int T = slab_tiles(P, W, mode, sl * kUnitRows, p.G, p.block_size);
+      local += T * p.Hkv;
+      tmin = min(tmin, T);
+      tmax = max(tmax, T);
+    }
+    nslab += slabs * p.Hkv;
   }
-  atomicAdd(&s_total, local);
-  if (bad) atomicOr(&s_bad, 1);
+  // one shared-memory atomic per warp (all 1024 threads on one address serialise)
+  local = __reduce_add_sync(0xffffffffu, local);
+  nslab = __reduce_add_sync(0xffffffffu, nslab);
+  tmin = __reduce_min_sync(0xffffffffu, tmin);
+  tmax = __reduce_max_sync(0xffffffffu, tmax);
+  bad = __reduce_or_sync(0xffffffffu, bad);
+  if ((tid & 31) == 0) {
+    atomicAdd(&s_total, local);
+    atomicAdd(&s_nslab, nslab);
+    atomicMin(&s_tmin, tmin);
+    atomicMax(&s_tmax, tmax);
+    if (bad) atomicOr(&s_bad, 1);
+  }
   __syncthreads();
   // Piece length: for each candidate (about 1..kSplitFactor pieces per SM)
   // count the units it makes and estimate the makespan as
@@ -210,12 +230,15 @@ __global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p
       }
     }
 #pragma unroll
-    for (int k = 0; k < kSplitFactor; ++k) atomicAdd(&s_units[k], cnt[k]);
+    for (int k = 0; k < kSplitFactor; ++k) {
+      cnt[k] = __reduce_add_sync(0xffffffffu, cnt[k]);
+      if ((tid & 31) == 0) atomicAdd(&s_units[k], cnt[k]);
+    }
   }
   __syncthreads();
   int chunk = cand[0];
+  float best = 3.4e38f;
   {
-    float best = 3.4e38f;
 #pragma unroll
     for (int k = 0; k < kSplitFactor; ++k) {
       const int U = max(1, s_units[k]);
@@ -227,6 +250,18 @@ __global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p
       }
     }
   }
+  // Slabs of one length T (few long sequences of one shape): cutting the
+  // concatenated key tiles of all slabs at multiples of total / SMs gives every
+  // SM the same number of tiles in at most ceil(share / T) + 1 pieces, where equal
+  // pieces per slab leave a fraction of a wave.
+  const int T_uni = s_tmax;
+  const bool stream_k = [&] {
+    if (s_tmin != s_tmax || s_nslab < 1 || s_total < 2 * kMinChunk * p.num_sms) return false;
+    const float share = static_cast<float>(s_total) / p.num_sms;
+    const float est = ceilf(share) + (ceilf(share / T_uni) + 1.f) * kUnitStartTiles;
+    return est < best * 0.98f;
+  }();
+  if (stream_k) chunk = min(T_uni, (s_total + p.num_sms - 1) / p.num_sms);  // the longest piece
   // pass 2: emit units (unsorted) and merge groups. The units of piece k of all
   // slabs of one (sequence, KV head) are emitted together (a "piece"): they
   // read the same K/V tiles, and the sort keeps them adjacent so that they run
@@ -259,6 +294,37 @@ __global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p
     const int P = seq_prefix(p, s), W = p.window_len[s], mode = seq_mode(p, s);
     if (!seq_ok(p, s, P, W, mode)) continue;
     const int slabs = (W * p.G + kUnitRows - 1) / kUnitRows;
+    if (stream_k) {
+      if (grp > 0) continue;
+      // slab sigma covers tiles [sigma T, sigma T + T) of the concatenation; SM share i
+      // ends at b_i = floor(i total / SMs); a slab is cut at every b_i strictly inside it
+      const int64_t total = s_total, S = p.num_sms;
+      const int sigma0 = atomicAdd(&s_sigma, slabs);
+      for (int sl = 0; sl < slabs; ++sl) {
+        const int64_t lo = static_cast<int64_t>(sigma0 + sl) * T_uni, hi = lo + T_uni;
+        const int64_t i_lo = ((lo + 1) * S + total - 1) / total;  // first i with b_i > lo
+        const int64_t i_hi = (hi * S + total - 1) / total - 1;    // last i with b_i < hi
+        const int n = static_cast<int>(i_hi >= i_lo ? i_hi - i_lo + 2 : 1);
+        int slot0 = -1;
+        if (n > 1) {
+          const int gi = atomicAdd(&s_ngroups, 1);
+          slot0 = atomicAdd(&s_nslots, n);
+          if (gi < p.max_groups && slot0 + n <= p.max_slots)
+            p.groups[gi] = MergeGroup{s, g, sl * kUnitRows, n, slot0, W, 0, 0};
+          else
+            overflow = true;
+        }
+        int64_t cut = lo;
+        for (int k = 0; k < n; ++k) {
+          const int64_t next = k + 1 < n ? ((i_lo + k) * total) / S : hi;
+          const WorkUnit u{s, g, sl * kUnitRows, static_cast<int>(cut - lo), static_cast<int>(next - lo),
+                           n > 1 ? slot0 + k : -1, P, W | (mode << 30)};
+          emit_piece(&u, 1, static_cast<int>(next - cut));
+          cut = next;
+        }
+      }
+      continue;
+    }
     const int ng = slabs <= kMaxGroupedSlabs ? slabs : 1;  // slabs per piece
     if (grp * ng >= slabs) continue;
     {
