@@ -692,21 +692,29 @@ def run_e2e(args, w, attention_call, edit_call, dev, stream, world, new_t, mask_
     paged KV caches are resident state, as in serving. The copies run on
     copy_streams streams (layer l's inputs on stream l mod n, the logits in n
     slices) beside the compute stream, and layer l computes once its own inputs
-    have arrived. One copy stream is the default: on this GPU one stream of
-    pinned host-to-device copies moved 410-420 GB/s, two or four concurrent
-    ones about 210 GB/s in total."""
+    have arrived. The device input buffers are double-buffered across steps:
+    step k copies into set k mod 2 as soon as step k - 2 (the last reader of that
+    set) has finished, so the copies of one step overlap the compute of the one
+    before and the steady state runs at max(copy time, compute time). One copy
+    stream is the default: on this GPU one stream of pinned host-to-device copies
+    moved about 208 GB/s, idle or beside the attention kernels, and two or four
+    concurrent ones no more. Some steps' host-to-device copies stall for
+    100-470 ms (seen with no kernel running as well), and the timed steps
+    include whatever stalls occur."""
     attn = w["attn"]
     ep = w["edit"]
+    nbuf = 2
     host = []
-    dbuf = []
+    dbuf = [[] for _ in range(nbuf)]
     for a in attn:
         host.append(tuple(t.cpu().pin_memory() for t in (a.q, a.k_win, a.v_win)))
-        dbuf.append(tuple(torch.empty_like(t) for t in (a.q, a.k_win, a.v_win)))
+        for b in range(nbuf):
+            dbuf[b].append(tuple(torch.empty_like(t) for t in (a.q, a.k_win, a.v_win)))
     if ep is not None:
         lg_h = ep.logits.cpu().pin_memory()
         cm_h = ep.committed.cpu().pin_memory()
-        lg_d = torch.empty_like(ep.logits)
-        cm_d = torch.empty_like(ep.committed)
+        lg_d = [torch.empty_like(ep.logits) for _ in range(nbuf)]
+        cm_d = [torch.empty_like(ep.committed) for _ in range(nbuf)]
         R = ep.logits.shape[0]
         out_h = [torch.empty(R, dtype=t.dtype, pin_memory=True) for t in (new_t, mask_t, conf_t)]
         cuts = [R * k // copy_streams for k in range(copy_streams + 1)]
@@ -715,35 +723,42 @@ def run_e2e(args, w, attention_call, edit_call, dev, stream, world, new_t, mask_
     if ep is not None:
         h2d += lg_h.numel() * lg_h.element_size() + cm_h.numel() * cm_h.element_size()
     d2h = sum(t.numel() * t.element_size() for t in out_h) if ep is not None else 0
+    freed = [None] * nbuf   # compute-stream event after the last read of buffer set b
+    counter = [0]
 
     def step():
+        b = counter[0] % nbuf
+        counter[0] += 1
+        if freed[b] is not None:
+            for c in cs:
+                c.wait_event(freed[b])
         copied = [torch.cuda.Event() for _ in attn]
         for i in range(len(attn)):
             with torch.cuda.stream(cs[i % copy_streams]):
-                for d, h in zip(dbuf[i], host[i]):
+                for d, h in zip(dbuf[b][i], host[i]):
                     d.copy_(h, non_blocking=True)
                 copied[i].record(cs[i % copy_streams])
         done_l = []
         if ep is not None:
             for k in range(copy_streams):
                 with torch.cuda.stream(cs[k]):
-                    lg_d[cuts[k]:cuts[k + 1]].copy_(lg_h[cuts[k]:cuts[k + 1]], non_blocking=True)
+                    lg_d[b][cuts[k]:cuts[k + 1]].copy_(lg_h[cuts[k]:cuts[k + 1]], non_blocking=True)
                     if k == 0:
-                        cm_d.copy_(cm_h, non_blocking=True)
+                        cm_d[b].copy_(cm_h, non_blocking=True)
                     e = torch.cuda.Event()
                     e.record(cs[k])
                     done_l.append(e)
         for i, a in enumerate(attn):
             stream.wait_event(copied[i])
-            attention_call(i, a, *dbuf[i])
+            attention_call(i, a, *dbuf[b][i])
         if ep is not None:
             for e in done_l:
                 stream.wait_event(e)
-            edit_call(lg_d, cm_d)
+            edit_call(lg_d[b], cm_d[b])
             for h, d in zip(out_h, (new_t, mask_t, conf_t)):
                 h.copy_(d, non_blocking=True)
-        for c in cs:
-            c.wait_stream(stream)
+        freed[b] = torch.cuda.Event()
+        freed[b].record(stream)
 
     # warm up until two consecutive steps agree within 5% (the first large
     # copies out of freshly pinned host memory can run several times slower)
@@ -765,7 +780,7 @@ def run_e2e(args, w, attention_call, edit_call, dev, stream, world, new_t, mask_
     torch.cuda.synchronize()
     el = max_over_ranks(time.perf_counter() - t0, dev)
     return {"value": round(whole_job_rate(attn[0].batch * K, world, el), 3), "unit": "windows/s", "h2d_bytes_per_step": int(h2d),
-            "d2h_bytes_per_step": int(d2h), "steps": K, "copy_streams": copy_streams,
+            "d2h_bytes_per_step": int(d2h), "steps": K, "copy_streams": copy_streams, "input_buffer_sets": nbuf,
             "h2d_gbs_effective": round(h2d * K / el / 1e9, 1),
             "resident_state": "paged KV caches of every layer (written by earlier passes)"}
 
