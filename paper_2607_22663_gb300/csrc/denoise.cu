@@ -253,8 +253,9 @@ __global__ void __launch_bounds__(256) tail_entropy_kernel(const float* __restri
 template <typename T>
 mbe_status launch_rows(const void* logits, int32_t rows, const RowArgs& a, cudaStream_t stream) {
   const T* lp = static_cast<const T*>(logits);
+  // as in edit-decide: 512 threads from 256 KB rows, 256 threads for 8-256 KB rows
   const int64_t row_bytes = static_cast<int64_t>(a.vocab) * sizeof(T);
-  if (row_bytes >= 64 * 1024)
+  if (row_bytes >= 256 * 1024)
     denoise_row_kernel<T, 512><<<rows, 512, 0, stream>>>(lp, a);
   else if (row_bytes >= 8 * 1024)
     denoise_row_kernel<T, 256><<<rows, 256, 0, stream>>>(lp, a);

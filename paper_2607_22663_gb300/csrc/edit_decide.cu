@@ -174,8 +174,11 @@ mbe_status launch(const void* logits, int64_t row_stride, int32_t rows, int32_t 
                   float* confidence, int32_t* argmax_out, cudaStream_t stream) {
   const T* lp = static_cast<const T*>(logits);
   const bool vec_ok = aligned16(logits) && ((row_stride * static_cast<int64_t>(sizeof(T))) % 16 == 0);
+  // rows of 256 KB and more: 512 threads (32 vectors each); 8-256 KB: 256 threads,
+  // so that shorter rows still stream at least a few vectors per thread and eight
+  // CTAs per SM overlap one another's final reductions
   const int64_t row_bytes = static_cast<int64_t>(vocab) * sizeof(T);
-  if (row_bytes >= 64 * 1024) {
+  if (row_bytes >= 256 * 1024) {
     edit_decide_kernel<T, 512><<<rows, 512, 0, stream>>>(lp, row_stride, vocab, vec_ok, committed, tpr, tau, editable,
                                                          new_tokens, edit_mask, confidence, argmax_out);
   } else if (row_bytes >= 8 * 1024) {
