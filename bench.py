@@ -564,10 +564,9 @@ def refresh_pass(attn, changed, rb, stream=None):
                                max_window=a0.max_window, total_rows=a0.total_tokens, out=rb.plan, stream=stream)
     p = rb.plan
     for i, a in enumerate(attn):
-        mbe.gather_rows_multi([(a.q, rb.q), (a.k_win, rb.k), (a.v_win, rb.v)], p["src_row"], rows_used=p["count"][1:],
-                              stream=stream)
-        mbe.kv_window_write(rb.k, rb.v, a.k_cache, a.v_cache, p["block_table"], p["prefix_len"], p["window_len"],
-                            p["cu_window"], block_size=B, max_window=B, stream=stream)
+        # the changed rows' Q/K/V compacted and their K/V written into the cache, one launch
+        mbe.refresh_gather_write(a.q, a.k_win, a.v_win, p, a.k_cache, a.v_cache, out=(rb.q, rb.k, rb.v),
+                                 stream=stream)
         fn = mbe.window_attention if i == 0 else mbe.window_attention_run
         fn(rb.q, rb.k, rb.v, a.k_cache, a.v_cache, p["block_table"], p["prefix_len"], p["window_len"], p["cu_window"],
            p["mask_mode"], block_size=B, max_window=B, max_prefix=rb.max_prefix, out=rb.out, workspace=rb.ws,
@@ -602,7 +601,7 @@ def time_refresh(w, dev, stream, peaks, ev_time, frac=0.125):
     return {"ms_per_pass": round(ms, 4), "changed_blocks": int(changed.sum()), "blocks": int(sum(nblk)),
             "layers": len(attn), "attention_gbs": round(byts / (ms * 1e-3) / 1e9, 1),
             "frac_hbm": round(byts / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"], 4),
-            "note": "plan + per layer (one gather of the Q/K/V rows, KV write, attention of the changed blocks)"}
+            "note": "plan + per layer (the changed rows' Q/K/V compacted and their K/V written, one launch; attention of the changed blocks)"}
 
 
 def time_pass_loop(w, dev, reps=3, max_passes=5):

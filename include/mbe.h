@@ -540,6 +540,37 @@ mbe_status mbe_gather_rows_multi(int32_t n_tensors, const void* const* srcs, con
                                  const int32_t* rows_used_or_null, cudaStream_t stream);
 
 /*
+ * mbe_refresh_gather_write -- the per-layer row work of the targeted refresh
+ * (Sec. 4.3: the changed blocks are recomputed under standard attention and
+ * their KV written back) in one launch. For refresh row k < min(rows,
+ * *rows_used_or_null) of the layout written by mbe_refresh_plan it copies
+ * source row src_row[k] of q [src_rows, num_q_heads, head_dim], k_win and
+ * v_win [src_rows, num_kv_heads, head_dim] (bf16) into row k of q_out, k_out
+ * and v_out, and writes that K and V row into k_cache / v_cache
+ * [num_pages, num_kv_heads, page_size, head_dim] at the row's refresh-layout
+ * position: row k belongs to entry e, the largest e < num_entries with
+ * r_cu_window[e] <= k, and goes to position r_prefix_len[e] + k -
+ * r_cu_window[e] through block-table row e (r_block_table [num_entries,
+ * max_pages_per_seq]). The result equals mbe_gather_rows_multi of the three
+ * tensors followed by mbe_kv_window_write of k_out / v_out on the refresh
+ * layout. Rows with src_row[k] < 0 become zero rows and write no cache slot;
+ * src_row[k] >= src_rows gives a zero row and MBE_DEVERR_LENGTH; a position
+ * past the block-table row sets MBE_DEVERR_LENGTH and a page id outside
+ * [0, num_pages) MBE_DEVERR_PAGE (those rows write no cache slot). Rows from
+ * *rows_used_or_null on are left as they are. All buffers are device memory,
+ * 16-byte aligned, none overlapping.
+ * Errors: MBE_ERR_INVALID_ARG (null or misaligned pointers, bad sizes),
+ * MBE_ERR_CUDA.
+ */
+mbe_status mbe_refresh_gather_write(const void* q, const void* k_win, const void* v_win, int64_t src_rows,
+                                    int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim,
+                                    const int32_t* src_row, const int32_t* rows_used_or_null, int64_t rows,
+                                    const int32_t* r_prefix_len, const int32_t* r_cu_window,
+                                    const int32_t* r_block_table, int32_t num_entries, int32_t max_pages_per_seq,
+                                    void* k_cache, void* v_cache, int32_t num_pages, int32_t page_size,
+                                    void* q_out, void* k_out, void* v_out, cudaStream_t stream);
+
+/*
  * Editing-pass loop on the device. Paper: Sec. 4.1 (the window is edited by
  * repeated passes until a pass changes no token or N_MBE passes have run) and
  * Sec. 4.3 (one graph serves every shape of the pass).

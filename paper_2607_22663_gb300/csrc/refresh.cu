@@ -172,6 +172,70 @@ __global__ void __launch_bounds__(256) gather_rows_multi_kernel(const GatherSet 
   }
 }
 
+// The per-layer row work of the refresh in one launch: refresh row k (k <
+// *rows_used) is copied from source row src_row[k] of q / k_win / v_win into
+// the compact q_out / k_out / v_out, and its K and V go into the paged cache at
+// its refresh-layout position: entry e (the largest e with r_cu[e] <= k) row
+// i = k - r_cu[e] sits at r_prefix[e] + i of block-table row e. One CTA per row
+// at a time (grid-stride); chunks are 16 bytes.
+__global__ void __launch_bounds__(256) refresh_rows_kernel(
+    const uint4* __restrict__ q, const uint4* __restrict__ kw, const uint4* __restrict__ vw, int64_t src_rows,
+    const int32_t* __restrict__ src_row, const int32_t* __restrict__ rows_used, int64_t rows,
+    const int32_t* __restrict__ r_prefix, const int32_t* __restrict__ r_cu, const int32_t* __restrict__ r_bt,
+    int E, int max_pages, uint4* __restrict__ k_cache, uint4* __restrict__ v_cache, int num_pages, int page_size,
+    int q_chunks, int kv_chunks, int chunks_per_head, int Hkv, uint4* __restrict__ q_out, uint4* __restrict__ k_out,
+    uint4* __restrict__ v_out) {
+  __shared__ int64_t s_dst;  // cache offset (in chunks) of head 0 of this row's slot; -1: no cache write
+  if (rows_used) rows = min(rows, static_cast<int64_t>(max(*rows_used, 0)));
+  const int per_row = q_chunks + 2 * kv_chunks;
+  for (int64_t k = blockIdx.x; k < rows; k += gridDim.x) {
+    const int32_t r = src_row[k];
+    const bool have = r >= 0 && r < src_rows;
+    if (threadIdx.x == 0) {
+      int64_t dst = -1;
+      if (r >= src_rows) atomicOr(&g_error_word, MBE_DEVERR_LENGTH);
+      if (have && E > 0) {
+        int lo = 0, hi = E - 1;  // the largest e with r_cu[e] <= k
+        while (lo < hi) {
+          const int mid = (lo + hi + 1) >> 1;
+          if (r_cu[mid] <= k) lo = mid; else hi = mid - 1;
+        }
+        const int64_t pos = static_cast<int64_t>(r_prefix[lo]) + (k - r_cu[lo]);
+        const int64_t lp = pos / page_size;
+        const int page = (lp >= 0 && lp < max_pages) ? r_bt[static_cast<int64_t>(lo) * max_pages + lp] : -2;
+        if (lp < 0 || lp >= max_pages) {
+          atomicOr(&g_error_word, MBE_DEVERR_LENGTH);
+        } else if (page < 0 || page >= num_pages) {
+          atomicOr(&g_error_word, MBE_DEVERR_PAGE);
+        } else {
+          dst = (static_cast<int64_t>(page) * Hkv * page_size + pos % page_size) * chunks_per_head;
+        }
+      }
+      s_dst = dst;
+    }
+    __syncthreads();
+    const int64_t dst = s_dst;
+    for (int c = threadIdx.x; c < per_row; c += blockDim.x) {
+      uint4 x = make_uint4(0u, 0u, 0u, 0u);
+      if (c < q_chunks) {
+        if (have) x = q[static_cast<int64_t>(r) * q_chunks + c];
+        q_out[k * q_chunks + c] = x;
+        continue;
+      }
+      const int kv = (c - q_chunks) >= kv_chunks ? 1 : 0;
+      const int cc = c - q_chunks - kv * kv_chunks;
+      if (have) x = (kv ? vw : kw)[static_cast<int64_t>(r) * kv_chunks + cc];
+      (kv ? v_out : k_out)[k * kv_chunks + cc] = x;
+      if (dst >= 0) {
+        // head g of the slot: pages are [Hkv, page_size, D]
+        const int g = cc / chunks_per_head, w = cc - g * chunks_per_head;
+        (kv ? v_cache : k_cache)[dst + static_cast<int64_t>(g) * page_size * chunks_per_head + w] = x;
+      }
+    }
+    __syncthreads();  // s_dst is rewritten for the next row
+  }
+}
+
 // Ends a pass: counts it and keeps the loop going while some sequence changed
 // a token and fewer than max_passes passes have run.
 __global__ void __launch_bounds__(256) pass_loop_condition_kernel(cudaGraphConditionalHandle handle,
@@ -306,6 +370,40 @@ extern "C" mbe_status mbe_gather_rows_multi(int32_t n_tensors, const void* const
   gather_rows_multi_kernel<<<static_cast<unsigned>(ctas), 256, 0, stream>>>(g, src_rows, src_row, rows,
                                                                              rows_used_or_null);
   return launch_status("gather_rows_multi_kernel");
+}
+
+extern "C" mbe_status mbe_refresh_gather_write(
+    const void* q, const void* k_win, const void* v_win, int64_t src_rows, int32_t num_q_heads,
+    int32_t num_kv_heads, int32_t head_dim, const int32_t* src_row, const int32_t* rows_used_or_null, int64_t rows,
+    const int32_t* r_prefix_len, const int32_t* r_cu_window, const int32_t* r_block_table, int32_t num_entries,
+    int32_t max_pages_per_seq, void* k_cache, void* v_cache, int32_t num_pages, int32_t page_size, void* q_out,
+    void* k_out, void* v_out, cudaStream_t stream) {
+  using namespace mbe;
+  if (src_rows < 0 || rows < 0 || num_q_heads < 1 || num_kv_heads < 1 || head_dim < 8 || head_dim % 8 != 0 ||
+      num_entries < 0 || max_pages_per_seq < 1 || num_pages < 1 || page_size < 1)
+    return MBE_ERR_INVALID_ARG;
+  if (rows == 0) return MBE_OK;
+  if (!src_row || !q_out || !k_out || !v_out || !k_cache || !v_cache || (src_rows > 0 && (!q || !k_win || !v_win)) ||
+      (num_entries > 0 && (!r_prefix_len || !r_cu_window || !r_block_table)))
+    return MBE_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k_win) || !aligned16(v_win) || !aligned16(k_cache) || !aligned16(v_cache) ||
+      !aligned16(q_out) || !aligned16(k_out) || !aligned16(v_out))
+    return MBE_ERR_INVALID_ARG;
+  const int sms = sm_count();
+  if (sms == 0) {
+    record_cuda_error(cudaGetLastError(), "cudaDeviceGetAttribute");
+    return MBE_ERR_CUDA;
+  }
+  const int chunks_per_head = head_dim / 8;
+  int64_t ctas = rows;
+  if (ctas > 8 * sms) ctas = 8 * sms;
+  refresh_rows_kernel<<<static_cast<unsigned>(ctas), 256, 0, stream>>>(
+      static_cast<const uint4*>(q), static_cast<const uint4*>(k_win), static_cast<const uint4*>(v_win), src_rows,
+      src_row, rows_used_or_null, rows, r_prefix_len, r_cu_window, r_block_table, num_entries, max_pages_per_seq,
+      static_cast<uint4*>(k_cache), static_cast<uint4*>(v_cache), num_pages, page_size,
+      num_q_heads * chunks_per_head, num_kv_heads * chunks_per_head, chunks_per_head, num_kv_heads,
+      static_cast<uint4*>(q_out), static_cast<uint4*>(k_out), static_cast<uint4*>(v_out));
+  return launch_status("refresh_rows_kernel");
 }
 
 struct mbe_pass_loop {

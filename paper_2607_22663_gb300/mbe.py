@@ -100,6 +100,9 @@ def lib(build_if_missing: bool = True):
     L.mbe_gather_rows.argtypes = [P, i64, i64, P, i64, P, P, P]
     L.mbe_gather_rows_multi.restype = ctypes.c_int
     L.mbe_gather_rows_multi.argtypes = [i32, P, P, P, i64, P, i64, P, P]
+    L.mbe_refresh_gather_write.restype = ctypes.c_int
+    L.mbe_refresh_gather_write.argtypes = [P, P, P, i64, i32, i32, i32, P, P, i64, P, P, P, i32, i32, P, P, i32, i32,
+                                           P, P, P, P]
     L.mbe_pass_loop_begin.restype = ctypes.c_int
     L.mbe_pass_loop_begin.argtypes = [i32, P, P, ctypes.POINTER(ctypes.c_void_p)]
     L.mbe_pass_loop_until_stable.restype = ctypes.c_int
@@ -567,6 +570,30 @@ def gather_rows_multi(pairs, src_row, rows_used=None, stream=None):
                                      _ptr(rows_used) if rows_used is not None else None, _stream(stream))
     _check("mbe_gather_rows_multi", st)
     return [out for _, out in pairs]
+
+
+def refresh_gather_write(q, k_win, v_win, plan, k_cache, v_cache, *, out, stream=None):
+    """mbe_refresh_gather_write: compacts the refresh rows of `plan` (as returned
+    by refresh_plan) from q / k_win / v_win into out = (q_out, k_out, v_out) and
+    writes their K/V into k_cache / v_cache at the refresh-layout positions."""
+    q_out, k_out, v_out = out
+    for t, n in ((q, "q"), (k_win, "k_win"), (v_win, "v_win"), (k_cache, "k_cache"), (v_cache, "v_cache"),
+                 (q_out, "q_out"), (k_out, "k_out"), (v_out, "v_out")):
+        _need(t, n, torch.bfloat16)
+    src_rows, Hq, D = q.shape
+    Hkv = k_win.shape[1]
+    num_pages, _, page_size, _ = k_cache.shape
+    rows = plan["src_row"].numel()
+    if q_out.shape[0] < rows or k_out.shape[0] < rows or v_out.shape[0] < rows:
+        raise ValueError("the outputs must hold every refresh row of the plan")
+    E, max_pages = plan["block_table"].shape
+    st = lib().mbe_refresh_gather_write(_ptr(q), _ptr(k_win), _ptr(v_win), src_rows, Hq, Hkv, D, _ptr(plan["src_row"]),
+                                        _ptr(plan["count"][1:]), rows, _ptr(plan["prefix_len"]),
+                                        _ptr(plan["cu_window"]), _ptr(plan["block_table"]), E, max_pages,
+                                        _ptr(k_cache), _ptr(v_cache), num_pages, page_size, _ptr(q_out),
+                                        _ptr(k_out), _ptr(v_out), _stream(stream))
+    _check("mbe_refresh_gather_write", st)
+    return out
 
 
 class PassLoop:

@@ -171,10 +171,11 @@ def _refresh_max_prefix(prob):
     return max(p + B * ((w - 1) // B) for p, w in zip(prob.prefix_host, prob.window_host) if w > 0)
 
 
-def _gpu_refresh(prob, old, changed, B, stream=None, bufs=None):
+def _gpu_refresh(prob, old, changed, B, stream=None, bufs=None, fused=False):
     """The refresh on the GPU, every step through the library: write the cache
     as decoding left it, plan, gather Q/K/V of the changed rows, write them,
-    attend. With `bufs` nothing is allocated (graph capture)."""
+    attend (fused: the gather and the write in one mbe_refresh_gather_write).
+    With `bufs` nothing is allocated (graph capture)."""
     d = prob.to(DEV) if bufs is None else bufs["prob"]
     T = int(prob.cu_window[-1])
     E = prob.batch * changed.shape[1]
@@ -194,10 +195,14 @@ def _gpu_refresh(prob, old, changed, B, stream=None, bufs=None):
     bufs["plan"] = plan
     # only the refresh rows are gathered (Q, K and V in one launch); the rest of the
     # buffers are never read
-    mbe.gather_rows_multi([(d.q, bufs["q"]), (d.k_win, bufs["k"]), (d.v_win, bufs["v"])], plan["src_row"],
-                          rows_used=plan["count"][1:], stream=stream)
-    mbe.kv_window_write(bufs["k"], bufs["v"], d.k_cache, d.v_cache, plan["block_table"], plan["prefix_len"],
-                        plan["window_len"], plan["cu_window"], block_size=B, max_window=B, stream=stream)
+    if fused:
+        mbe.refresh_gather_write(d.q, d.k_win, d.v_win, plan, d.k_cache, d.v_cache,
+                                 out=(bufs["q"], bufs["k"], bufs["v"]), stream=stream)
+    else:
+        mbe.gather_rows_multi([(d.q, bufs["q"]), (d.k_win, bufs["k"]), (d.v_win, bufs["v"])], plan["src_row"],
+                              rows_used=plan["count"][1:], stream=stream)
+        mbe.kv_window_write(bufs["k"], bufs["v"], d.k_cache, d.v_cache, plan["block_table"], plan["prefix_len"],
+                            plan["window_len"], plan["cu_window"], block_size=B, max_window=B, stream=stream)
     mbe.window_attention(bufs["q"], bufs["k"], bufs["v"], d.k_cache, d.v_cache, plan["block_table"],
                          plan["prefix_len"], plan["window_len"], plan["cu_window"], plan["mask_mode"], block_size=B,
                          max_window=B, max_prefix=_refresh_max_prefix(prob), out=bufs["out"], workspace=bufs["ws"],
@@ -219,6 +224,27 @@ def test_refresh_attention_and_cache_match_oracle():
     np.testing.assert_array_equal(bf16_bits(bufs["prob"].v_cache.cpu()), vc_ref)
     # rows past the refresh rows are left as they were
     assert bufs["q"][n:].isnan().all() and bufs["v"][n:].isnan().all()
+
+
+def test_refresh_gather_write_matches_oracle_and_separate_calls():
+    """mbe_refresh_gather_write (gather + cache write in one launch) gives the
+    same compact rows, cache and attention output as mbe_gather_rows_multi
+    followed by mbe_kv_window_write, and matches the oracle."""
+    prob, old, changed, B = _refresh_problem(seed=23)
+    sep = _gpu_refresh(prob, old, changed, B)
+    fus = _gpu_refresh(prob, old, changed, B, fused=True)
+    torch.cuda.synchronize()
+    assert mbe.get_device_error() == (0, 0)
+    rows, out_ref, kc_ref, vc_ref = _oracle_refresh(prob, old, changed, B)
+    n = len(rows)
+    for key in ("q", "k", "v", "out"):
+        assert torch.equal(fus[key][:n], sep[key][:n]), key
+    assert fus["q"][n:].isnan().all() and fus["k"][n:].isnan().all() and fus["v"][n:].isnan().all()
+    for cache in ("k_cache", "v_cache"):
+        assert torch.equal(getattr(fus["prob"], cache), getattr(sep["prob"], cache))
+    np.testing.assert_array_equal(bf16_bits(fus["prob"].k_cache.cpu()), kc_ref)
+    np.testing.assert_array_equal(bf16_bits(fus["prob"].v_cache.cpu()), vc_ref)
+    assert np.abs(fus["out"][:n].float().cpu().numpy() - out_ref).max() <= ATTN_ATOL
 
 
 def test_refresh_in_a_captured_graph_matches_eager():
