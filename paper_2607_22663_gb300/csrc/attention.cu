@@ -161,8 +161,15 @@ __device__ __forceinline__ bool seq_ok(const SchedParams& p, int s, int P, int W
 }
 
 __device__ __forceinline__ int cost_bucket(int cost, int chunk) {
-  const int b = static_cast<int>((static_cast<int64_t>(cost - 1) * kBuckets) / chunk);
+  // 32-bit arithmetic while (cost - 1) * kBuckets fits (costs below 2^21 tiles)
+  const int b = cost < (1 << 21) ? ((cost - 1) * kBuckets) / chunk
+                                 : static_cast<int>((static_cast<int64_t>(cost - 1) * kBuckets) / chunk);
   return min(max(b, 0), kBuckets - 1);
+}
+
+// floor(k * T / n) for 0 <= k <= n <= T: 32-bit while k * T fits
+__device__ __forceinline__ int split_point(int k, int T, int n) {
+  return T < 46341 ? (k * T) / n : static_cast<int>((static_cast<int64_t>(k) * T) / n);
 }
 
 __global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p) {
@@ -214,8 +221,8 @@ __global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p
   int cand[kSplitFactor];
 #pragma unroll
   for (int k = 0; k < kSplitFactor; ++k) {
-    const int64_t target = static_cast<int64_t>(k + 1) * p.num_sms;
-    cand[k] = max(kMinChunk, static_cast<int>((s_total + target - 1) / target));
+    const int target = (k + 1) * p.num_sms;  // ceil(s_total / target) without overflow
+    cand[k] = max(kMinChunk, s_total / target + (s_total % target != 0 ? 1 : 0));
   }
   {
     int cnt[kSplitFactor] = {};
@@ -353,8 +360,8 @@ __global__ void __launch_bounds__(1024) attn_schedule_kernel(const SchedParams p
           int c = 0, cost = 1;
           for (int i = 0; i < cnt; ++i) {
             if (k >= n[i]) continue;
-            const int tb = static_cast<int>((static_cast<int64_t>(k) * T[i]) / n[i]);
-            const int te = static_cast<int>((static_cast<int64_t>(k + 1) * T[i]) / n[i]);
+            const int tb = split_point(k, T[i], n[i]);
+            const int te = split_point(k + 1, T[i], n[i]);
             u[c++] = WorkUnit{s, g, (s0 + i) * kUnitRows, tb, te, n[i] > 1 ? slot0[i] + k : -1, P, W | (mode << 30)};
             cost = max(cost, te - tb);
           }
@@ -1314,9 +1321,13 @@ __global__ void __launch_bounds__(kMergeThreads, 2) attn_merge_kernel(const Merg
   // the attention kernel has finished: re-arm the work counter so that the same
   // plan can serve the next run
   if (blockIdx.x == 0 && threadIdx.x == 0) p.hdr->counter = 0;
-  if (!sig_equal(p.hdr->sig, p.sig)) return;
+  // one thread reads the header (a plan with no split groups leaves at once)
+  __shared__ int s_groups;
+  if (threadIdx.x == 0) s_groups = sig_equal(p.hdr->sig, p.sig) ? p.hdr->n_groups : 0;
+  __syncthreads();
+  if (s_groups <= 0) return;
   constexpr int kBlocks = kUnitRows / kMergeRows;
-  const int64_t n_items = static_cast<int64_t>(p.hdr->n_groups) * kBlocks;
+  const int64_t n_items = static_cast<int64_t>(s_groups) * kBlocks;
   const int lane = threadIdx.x & 31;
   const int64_t warps = static_cast<int64_t>(gridDim.x) * (kMergeThreads / 32);
   for (int64_t it = static_cast<int64_t>(blockIdx.x) * (kMergeThreads / 32) + threadIdx.x / 32; it < n_items;
