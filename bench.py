@@ -78,7 +78,7 @@ def edit_bytes(rows, vocab, elem):
 # its output (the full call splits no key range, so it writes no partials).
 # Source: profiles/attn_kernel_dram_serving_b64.md.
 MEASURED_TRAFFIC = {
-    "507c7f9cf35c44d3": {"serving128": 4436122206 + 67108864},
+    "dc01577b12386ae2": {"serving128": 4437382166 + 67108864},
 }
 
 
