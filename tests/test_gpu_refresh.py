@@ -247,6 +247,36 @@ def test_refresh_gather_write_matches_oracle_and_separate_calls():
     assert np.abs(fus["out"][:n].float().cpu().numpy() - out_ref).max() <= ATTN_ATOL
 
 
+def test_refresh_gather_write_bad_page_flags_and_skips_like_separate_calls():
+    """A changed block whose page id lies outside the cache: the fused call sets
+    MBE_DEVERR_PAGE and skips those cache slots, as the KV write does, and both
+    paths leave identical compact rows and caches."""
+    prob, old, changed, B = _refresh_problem(seed=24)
+    d = prob.to(DEV)
+    bt = d.block_table.clone()
+    bt[0, (prob.prefix_host[0] + B) // prob.page_size] = d.k_cache.shape[0] + 7   # block 1 of sequence 0
+    changed[0, 1] = 1
+    plan = mbe.refresh_plan(changed.to(DEV), d.prefix_len, d.window_len, d.cu_window, bt, block_size=B,
+                            max_window=max(prob.window_host), total_rows=int(prob.cu_window[-1]))
+    res = []
+    for fused in (True, False):
+        outs = tuple(torch.zeros_like(x) for x in (d.q, d.k_win, d.v_win))
+        kc, vc = d.k_cache.clone(), d.v_cache.clone()
+        if fused:
+            mbe.refresh_gather_write(d.q, d.k_win, d.v_win, plan, kc, vc, out=outs)
+        else:
+            mbe.gather_rows_multi(list(zip((d.q, d.k_win, d.v_win), outs)), plan["src_row"],
+                                  rows_used=plan["count"][1:])
+            mbe.kv_window_write(outs[1], outs[2], kc, vc, plan["block_table"], plan["prefix_len"], plan["window_len"],
+                                plan["cu_window"], block_size=B, max_window=B)
+        st, flags = mbe.get_device_error()
+        assert flags == mbe.DEVERR_PAGE, flags
+        res.append(outs + (kc, vc))
+    for a, b in zip(*res):
+        assert torch.equal(a, b)
+    assert not torch.equal(res[0][3], d.k_cache)   # the other changed blocks were written
+
+
 def test_refresh_in_a_captured_graph_matches_eager():
     prob, old, changed, B = _refresh_problem(seed=22)
     eager = _gpu_refresh(prob, old, changed, B)
