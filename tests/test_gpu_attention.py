@@ -251,6 +251,25 @@ def test_long32k_workload_sampled():
         compare_attention(prob, out, lse, seqs=[0, 3], heads=[0, 9, 30])
 
 
+def test_stream_k_pieces_of_one_query_tile_slabs():
+    """Slabs of one length with a single query tile each (W G = 128 rows): the
+    plan cuts their concatenated key tiles at multiples of total / SMs, so split
+    pieces of units that run both TMEM chains on one query tile are merged by
+    log-sum-exp. Checked against the oracle on sampled sequences; the plan must
+    hold split groups."""
+    prob = wl.attention_problem([16384] * 8, [32] * 8, [wl.BIDIRECTIONAL] * 8, 32, 8, 128, 32, 32, seed=61,
+                                device=DEV)
+    out, lse = run_attention(prob)
+    need = mbe.window_attention_workspace_size(prob.batch, 32, 8, 128, prob.max_window, prob.max_prefix)
+    ws = torch.empty(need, dtype=torch.uint8, device=DEV)
+    mbe.window_attention_plan(prob.prefix_len, prob.window_len, prob.cu_window, prob.mask_mode,
+                              total_q_tokens=prob.total_tokens, num_q_heads=32, num_kv_heads=8, head_dim=128,
+                              block_size=32, max_window=prob.max_window, max_prefix=prob.max_prefix, workspace=ws)
+    n_units, n_groups = mbe.window_attention_plan_stats(ws)
+    assert n_groups > 0 and n_units > prob.batch * 8
+    compare_attention(prob, out, lse, seqs=[0, 5], heads=[0, 13, 31])
+
+
 def test_serving128_full_size_sampled():
     """Full per-layer shapes of the serving mix (2 of its 24 layers)."""
     w = wl.serving128(DEV, layers=2, vocab=8)
