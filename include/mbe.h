@@ -554,9 +554,10 @@ mbe_status mbe_gather_rows_multi(int32_t n_tensors, const void* const* srcs, con
  * max_pages_per_seq]). The result equals mbe_gather_rows_multi of the three
  * tensors followed by mbe_kv_window_write of k_out / v_out on the refresh
  * layout. Rows with src_row[k] < 0 become zero rows and write no cache slot;
- * src_row[k] >= src_rows gives a zero row and MBE_DEVERR_LENGTH; a position
- * past the block-table row sets MBE_DEVERR_LENGTH and a page id outside
- * [0, num_pages) MBE_DEVERR_PAGE (those rows write no cache slot). Rows from
+ * src_row[k] >= src_rows gives a zero row and MBE_DEVERR_LENGTH; a row outside
+ * every entry (k >= r_cu_window[num_entries]) or a position past the
+ * block-table row sets MBE_DEVERR_LENGTH and a page id outside [0, num_pages)
+ * MBE_DEVERR_PAGE (those rows write no cache slot). Rows from
  * *rows_used_or_null on are left as they are. All buffers are device memory,
  * 16-byte aligned, none overlapping.
  * Errors: MBE_ERR_INVALID_ARG (null or misaligned pointers, bad sizes),

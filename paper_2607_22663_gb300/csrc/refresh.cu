@@ -203,7 +203,8 @@ __global__ void __launch_bounds__(256) refresh_rows_kernel(
         const int64_t pos = static_cast<int64_t>(r_prefix[lo]) + (k - r_cu[lo]);
         const int64_t lp = pos / page_size;
         const int page = (lp >= 0 && lp < max_pages) ? r_bt[static_cast<int64_t>(lo) * max_pages + lp] : -2;
-        if (lp < 0 || lp >= max_pages) {
+        if (k < r_cu[lo] || k >= r_cu[lo + 1] || lp < 0 || lp >= max_pages) {
+          // a row outside every entry (row count and layout disagree) or past its block-table row
           atomicOr(&g_error_word, MBE_DEVERR_LENGTH);
         } else if (page < 0 || page >= num_pages) {
           atomicOr(&g_error_word, MBE_DEVERR_PAGE);

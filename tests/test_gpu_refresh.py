@@ -277,6 +277,32 @@ def test_refresh_gather_write_bad_page_flags_and_skips_like_separate_calls():
     assert not torch.equal(res[0][3], d.k_cache)   # the other changed blocks were written
 
 
+def test_refresh_gather_write_row_outside_every_entry_writes_no_slot():
+    """A row count larger than the layout (and a valid source row for the extra
+    row): that row is compacted but writes no cache slot, and the call sets
+    MBE_DEVERR_LENGTH; the caches equal those of the consistent call."""
+    prob, old, changed, B = _refresh_problem(seed=25)
+    d = prob.to(DEV)
+    plan = mbe.refresh_plan(changed.to(DEV), d.prefix_len, d.window_len, d.cu_window, d.block_table, block_size=B,
+                            max_window=max(prob.window_host), total_rows=int(prob.cu_window[-1]))
+    n = int(plan["count"][1])
+    assert n < plan["src_row"].numel()
+    res = []
+    for extra in (False, True):
+        p2 = {k: v.clone() for k, v in plan.items()}
+        if extra:
+            p2["src_row"][n] = 0
+            p2["count"][1] = n + 1
+        outs = tuple(torch.zeros_like(x) for x in (d.q, d.k_win, d.v_win))
+        kc, vc = d.k_cache.clone(), d.v_cache.clone()
+        mbe.refresh_gather_write(d.q, d.k_win, d.v_win, p2, kc, vc, out=outs)
+        st, flags = mbe.get_device_error()
+        assert flags == (mbe.DEVERR_LENGTH if extra else 0), flags
+        res.append((outs, kc, vc))
+    assert torch.equal(res[0][1], res[1][1]) and torch.equal(res[0][2], res[1][2])
+    assert torch.equal(res[1][0][0][n], d.q[0])   # the extra row itself is compacted
+
+
 def test_refresh_in_a_captured_graph_matches_eager():
     prob, old, changed, B = _refresh_problem(seed=22)
     eager = _gpu_refresh(prob, old, changed, B)
