@@ -736,20 +736,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto wait_item = [&](uint32_t n) { return mbar_wait(bar(bars.full[n % S::kSlots]), (n / S::kSlots) & 1, abort_flag, wait_ns); };
       auto release_item = [&](uint32_t n) { umma_commit(bar(bars.empty[n % S::kSlots])); };
       // S of chain i = Q tile qt times K (qt = i, or 0 for both chains of a split unit)
+      // descriptors of a tile: one built per operand, the K steps by constant adds
       auto issue_qk = [&](int i, uint32_t ka, int qt) {
-        const uint32_t qa = sbase + S::kQ + qt * S::kQTile;
+        const uint64_t qd = sdesc_sw128(sbase + S::kQ + qt * S::kQTile, 16, 1024), kd = sdesc_sw128(ka, 16, 1024);
 #pragma unroll
         for (int h = 0; h < S::kHalves; ++h)
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            umma_ss(tmem + kTmemS + 128 * i, sdesc_sw128(qa + h * S::kHalfBytes + k * 32, 16, 1024),
-                    sdesc_sw128(ka + h * S::kHalfBytes + k * 32, 16, 1024), idesc_qk, (h | k) ? 1u : 0u);
+            umma_ss(tmem + kTmemS + 128 * i, desc_add(qd, (h * S::kHalfBytes + k * 32) >> 4),
+                    desc_add(kd, (h * S::kHalfBytes + k * 32) >> 4), idesc_qk, (h | k) ? 1u : 0u);
       };
       auto issue_pv = [&](int i, uint32_t va, bool acc) {
+        const uint64_t vd = sdesc_sw128(va, S::kHalfBytes, 1024);
 #pragma unroll
         for (int kk = 0; kk < kTileKeys / 16; ++kk)
-          umma_ts(tmem + i * D, tmem + kTmemS + 128 * i + kk * 8, sdesc_sw128(va + kk * 16 * 128, S::kHalfBytes, 1024),
-                  idesc_pv, (acc || kk > 0) ? 1u : 0u);
+          umma_ts(tmem + i * D, tmem + kTmemS + 128 * i + kk * 8, desc_add(vd, (kk * 16 * 128) >> 4), idesc_pv,
+                  (acc || kk > 0) ? 1u : 0u);
       };
       for (;;) {
         const int slot = u_it & 1;

@@ -166,6 +166,15 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo_byt
   return d;
 }
 
+// The descriptor of base + off16 * 16 bytes from the descriptor of base: the start
+// address is the low 14-bit field (address / 16), and shared-memory addresses stay
+// below 256 KB, so the add never carries out of it. One 32-bit add instead of
+// rebuilding the descriptor keeps the single MMA-issuing thread's instruction count
+// low; it shares its sub-partition's issue slots with busy softmax or epilogue warps.
+__device__ __forceinline__ uint64_t desc_add(uint64_t d, uint32_t off16) {
+  return (d & 0xFFFFFFFF00000000ull) | static_cast<uint32_t>(static_cast<uint32_t>(d) + off16);
+}
+
 // Instruction descriptor, kind::f16 with bf16 A/B and fp32 accumulation.
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, bool a_mn_major, bool b_mn_major) {
   return (1u << 4)                                  // D = f32
