@@ -184,10 +184,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tc_fence_after();
             const uint32_t a = sbase + s * kStageBytes, b = a + kABytes;
+            const uint64_t ad = sdesc_sw128(a, 16, 1024), bd = sdesc_sw128(b, 16, 1024);
 #pragma unroll
             for (int k = 0; k < kBK / 16; ++k)
-              umma_ss(d_tmem, sdesc_sw128(a + k * 32, 16, 1024), sdesc_sw128(b + k * 32, 16, 1024), idesc,
-                      (kb | k) != 0);
+              umma_ss(d_tmem, desc_add(ad, (k * 32) >> 4), desc_add(bd, (k * 32) >> 4), idesc, (kb | k) != 0);
             umma_commit(bar(bars.empty[s]));
           }
           if (!ok) break;

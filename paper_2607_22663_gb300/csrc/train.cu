@@ -399,13 +399,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait(bar(bars.q_full[t % 3]), (t / 3) & 1, abort_flag, wait_ns)) return false;
         tc_fence_after();
         const uint32_t qa = sbase + kRingA + (t % 3) * kTileBytes;
+        const uint64_t kd = sdesc_sw128(sbase + kK, 16, 1024), qd = sdesc_sw128(qa, 16, 1024);
 #pragma unroll
         for (int h = 0; h < 2; ++h)
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
-            const uint32_t off = h * kHalf + k * 32;
-            umma_ss(tmem + kTmS, sdesc_sw128(sbase + kK + off, 16, 1024), sdesc_sw128(qa + off, 16, 1024), idesc_kk,
-                    (h | k) ? 1u : 0u);
+            const uint32_t off16 = (h * kHalf + k * 32) >> 4;
+            umma_ss(tmem + kTmS, desc_add(kd, off16), desc_add(qd, off16), idesc_kk, (h | k) ? 1u : 0u);
           }
         umma_commit(bar(bars.s_full));
         return true;
@@ -415,13 +415,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait(bar(bars.do_full[t & 1]), (t >> 1) & 1, abort_flag, wait_ns)) return false;
         tc_fence_after();
         const uint32_t da = sbase + kRingB + (t & 1) * kTileBytes;
+        const uint64_t vd = sdesc_sw128(sbase + kV, 16, 1024), dd = sdesc_sw128(da, 16, 1024);
 #pragma unroll
         for (int h = 0; h < 2; ++h)
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
-            const uint32_t off = h * kHalf + k * 32;
-            umma_ss(tmem + kTmDP, sdesc_sw128(sbase + kV + off, 16, 1024), sdesc_sw128(da + off, 16, 1024), idesc_kk,
-                    (h | k) ? 1u : 0u);
+            const uint32_t off16 = (h * kHalf + k * 32) >> 4;
+            umma_ss(tmem + kTmDP, desc_add(vd, off16), desc_add(dd, off16), idesc_kk, (h | k) ? 1u : 0u);
           }
         umma_commit(bar(bars.dp_full));
         return true;
@@ -448,20 +448,22 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           tc_fence_after();
+          const uint64_t dod = sdesc_sw128(da, kHalf, 1024);
 #pragma unroll
           for (int kk = 0; kk < kTile / 16; ++kk)
             // P^T of query columns 64 h .. 64 h + 63 sits packed at S region columns 64 h .. 64 h + 31
-            umma_ts(tmem + kTmDV, tmem + kTmS + (kk >> 2) * 64 + (kk & 3) * 8,
-                    sdesc_sw128(da + kk * 16 * 128, kHalf, 1024), idesc_tb, (j > 0 || kk > 0) ? 1u : 0u);
+            umma_ts(tmem + kTmDV, tmem + kTmS + (kk >> 2) * 64 + (kk & 3) * 8, desc_add(dod, (kk * 16 * 128) >> 4),
+                    idesc_tb, (j > 0 || kk > 0) ? 1u : 0u);
           umma_commit(bar(bars.do_empty[t & 1]));
           if (j + 1 < n_q && !issue_s(t + 1)) { ok = false; break; }
           // dK once dS^T is in TMEM (over dP^T), then the next tile's dP^T
           if (!mbar_wait(bar(bars.ds_full), t & 1, abort_flag, wait_ns)) { ok = false; break; }
           tc_fence_after();
+          const uint64_t qtd = sdesc_sw128(qa, kHalf, 1024);
 #pragma unroll
           for (int kk = 0; kk < kTile / 16; ++kk)
-            umma_ts(tmem + kTmDK, tmem + kTmDP + (kk >> 2) * 64 + (kk & 3) * 8,
-                    sdesc_sw128(qa + kk * 16 * 128, kHalf, 1024), idesc_tb, (j > 0 || kk > 0) ? 1u : 0u);
+            umma_ts(tmem + kTmDK, tmem + kTmDP + (kk >> 2) * 64 + (kk & 3) * 8, desc_add(qtd, (kk * 16 * 128) >> 4),
+                    idesc_tb, (j > 0 || kk > 0) ? 1u : 0u);
           umma_commit(bar(bars.q_empty[t % 3]));
           if (j + 1 < n_q && !issue_dp(t + 1)) { ok = false; break; }
         }
@@ -793,13 +795,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait(bar(bars.k_full[t % 3]), (t / 3) & 1, abort_flag, wait_ns)) return false;
         tc_fence_after();
         const uint32_t ka = sbase + kRingA + (t % 3) * kTileBytes;
+        const uint64_t qd = sdesc_sw128(sbase + kQ, 16, 1024), kd = sdesc_sw128(ka, 16, 1024);
 #pragma unroll
         for (int h = 0; h < 2; ++h)
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
-            const uint32_t off = h * kHalf + k * 32;
-            umma_ss(tmem + kTmQS + 128 * b, sdesc_sw128(sbase + kQ + off, 16, 1024), sdesc_sw128(ka + off, 16, 1024),
-                    idesc_kk, (h | k) ? 1u : 0u);
+            const uint32_t off16 = (h * kHalf + k * 32) >> 4;
+            umma_ss(tmem + kTmQS + 128 * b, desc_add(qd, off16), desc_add(kd, off16), idesc_kk, (h | k) ? 1u : 0u);
           }
         umma_commit(bar(bars.s_full[b]));
         return true;
@@ -810,13 +812,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait(bar(bars.v_full[t & 1]), (t >> 1) & 1, abort_flag, wait_ns)) return false;
         tc_fence_after();
         const uint32_t va = sbase + kRingB + (t & 1) * kTileBytes;
+        const uint64_t dod = sdesc_sw128(sbase + kDO, 16, 1024), vd = sdesc_sw128(va, 16, 1024);
 #pragma unroll
         for (int h = 0; h < 2; ++h)
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
-            const uint32_t off = h * kHalf + k * 32;
-            umma_ss(tmem + kTmQDP, sdesc_sw128(sbase + kDO + off, 16, 1024), sdesc_sw128(va + off, 16, 1024),
-                    idesc_kk, (h | k) ? 1u : 0u);
+            const uint32_t off16 = (h * kHalf + k * 32) >> 4;
+            umma_ss(tmem + kTmQDP, desc_add(dod, off16), desc_add(vd, off16), idesc_kk, (h | k) ? 1u : 0u);
           }
         umma_commit(bar(bars.dp_full));
         umma_commit(bar(bars.v_empty[t & 1]));
@@ -848,10 +850,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t ka = sbase + kRingA + (t % 3) * kTileBytes;
           // dQ += dS K_t: dS of key columns 64 h .. 64 h + 63 sits packed at S buffer columns
           // 64 h .. 64 h + 31 (A from TMEM); K_t [key][d] is an MN-major B
+          const uint64_t ktd = sdesc_sw128(ka, kHalf, 1024);
 #pragma unroll
           for (int kk = 0; kk < kTile / 16; ++kk)
             umma_ts(tmem + kTmQDQ, tmem + kTmQS + 128 * (t & 1) + (kk >> 2) * 64 + (kk & 3) * 8,
-                    sdesc_sw128(ka + kk * 16 * 128, kHalf, 1024), idesc_dq, (j > 0 || kk > 0) ? 1u : 0u);
+                    desc_add(ktd, (kk * 16 * 128) >> 4), idesc_dq, (j > 0 || kk > 0) ? 1u : 0u);
           umma_commit(bar(bars.k_empty[t % 3]));
           if (j + 2 < n_k && !issue_s(t + 2)) { ok = false; break; }
         }
