@@ -73,12 +73,12 @@ def edit_bytes(rows, vocab, elem):
 # (attn_kernel) of the serving workload, keyed by the first 16 hex digits of the
 # SHA-256 of the kernel source that was measured; a changed kernel gets no traffic
 # figure until it is measured again. Measured on a 64-sequence, one-layer case of
-# the same workload (2.3 GB of cache on the device), whose reads were 1.0089x its
+# the same workload (2.3 GB of cache on the device), whose reads were 1.0092x its
 # algorithmic Q + K/V bytes; scaled to the 128-sequence call by those bytes, plus
 # its output (the full call splits no key range, so it writes no partials).
 # Source: profiles/attn_kernel_dram_serving_b64.md.
 MEASURED_TRAFFIC = {
-    "dc01577b12386ae2": {"serving128": 4437382166 + 67108864},
+    "d2f0654adf59f35a": {"serving128": 4436701626 + 67108864},
 }
 
 
