@@ -40,6 +40,11 @@ RAGGED = [
     ([255, 700, 1], [64, 128, 8], [BIDIRECTIONAL, BLOCK_CAUSAL, BIDIRECTIONAL], 8, 2, 64, 32, 64),   # D = 64
     ([130, 90], [40, 24], [BLOCK_CAUSAL, BLOCK_CAUSAL], 4, 2, 128, 8, 8),            # page 8, odd windows
     ([4000], [256], [BLOCK_CAUSAL], 16, 4, 128, 32, 128),                          # 4 query slabs
+    # the other group sizes GQA packing allows: a 128-row tile holds 128 / G tokens
+    ([2100, 45], [96, 64], [BLOCK_CAUSAL, BIDIRECTIONAL], 8, 4, 128, 32, 32),       # G = 2
+    ([1500, 300], [32, 72], [BIDIRECTIONAL, BLOCK_CAUSAL], 32, 2, 128, 32, 32),     # G = 16
+    ([800], [64], [BLOCK_CAUSAL], 32, 1, 128, 16, 64),                             # G = 32: 4 tokens per tile
+    ([257, 30], [24, 40], [BLOCK_CAUSAL, BIDIRECTIONAL], 128, 1, 64, 8, 16),        # G = 128: 1 token per tile
 ]
 
 
