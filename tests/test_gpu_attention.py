@@ -45,6 +45,10 @@ RAGGED = [
     ([1500, 300], [32, 72], [BIDIRECTIONAL, BLOCK_CAUSAL], 32, 2, 128, 32, 32),     # G = 16
     ([800], [64], [BLOCK_CAUSAL], 32, 1, 128, 16, 64),                             # G = 32: 4 tokens per tile
     ([257, 30], [24, 40], [BLOCK_CAUSAL, BIDIRECTIONAL], 128, 1, 64, 8, 16),        # G = 128: 1 token per tile
+    # block sizes: 1 (block-causal is then causal), 48 (not a power of two), 128 > W
+    ([150], [40], [BLOCK_CAUSAL], 16, 4, 128, 1, 32),
+    ([500, 61], [96, 144], [BLOCK_CAUSAL, BLOCK_CAUSAL], 16, 4, 128, 48, 32),
+    ([700], [64], [BLOCK_CAUSAL], 16, 4, 128, 128, 64),
 ]
 
 

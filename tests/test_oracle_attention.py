@@ -80,6 +80,42 @@ def test_one_block_window_is_standard_block_diffusion_pass():
             np.testing.assert_allclose(out_c[t0:t0 + 32, h], ref.numpy(), rtol=0, atol=1e-12)
 
 
+def test_block_size_one_is_causal_attention():
+    """B = 1 (Sec. 2.2 with one-token blocks): each window query sees the prefix
+    and the window keys up to itself. Without a prefix that is torch's own causal
+    attention (is_causal); with one, the window part of the mask is a lower triangle."""
+    W, D = 24, 32
+    prob = attention_problem([0], [W], [BLOCK_CAUSAL], 4, 2, D, 1, 8, seed=41)
+    out, lse = oracle_attention(prob)
+    for h in range(4):
+        K, V = dense_keys(prob, 0, h // 2)
+        q = prob.q[:W, h].double()
+        ref = F.scaled_dot_product_attention(q[None, None], K[None, None], V[None, None], is_causal=True,
+                                             scale=1.0 / math.sqrt(D))[0, 0]
+        np.testing.assert_allclose(out[:W, h], ref.numpy(), rtol=0, atol=1e-12)
+    P = 37
+    prob = attention_problem([P], [W], [BLOCK_CAUSAL], 4, 2, D, 1, 8, seed=42)
+    out, lse = oracle_attention(prob)
+    mask = torch.cat([torch.ones(W, P, dtype=torch.bool), torch.ones(W, W, dtype=torch.bool).tril()], dim=1)
+    for h in range(4):
+        ref, ref_lse = _sdpa_reference(prob, 0, h, mask)
+        np.testing.assert_allclose(out[:W, h], ref.numpy(), rtol=0, atol=1e-12)
+        np.testing.assert_allclose(lse[:W, h], ref_lse.numpy(), rtol=0, atol=1e-12)
+
+
+def test_block_at_least_as_long_as_the_window_is_bidirectional():
+    """B >= W: the whole window is one block, so block-causal and bidirectional
+    attention (Eq. 5) coincide exactly."""
+    for B in (64, 128):
+        prob = attention_problem([70], [64], [BLOCK_CAUSAL], 4, 1, 32, B, 16, seed=43)
+        out_c, lse_c = oracle_attention(prob)
+        prob_b = AttnProblem(**{**prob.__dict__, "mask_mode": torch.tensor([BIDIRECTIONAL], dtype=torch.uint8),
+                                "mode_host": [BIDIRECTIONAL]})
+        out_b, lse_b = oracle_attention(prob_b)
+        np.testing.assert_array_equal(out_c, out_b)
+        np.testing.assert_array_equal(lse_c, lse_b)
+
+
 def test_block_causal_equals_sequential_single_block_passes():
     """k blocks in block-causal mode == decoding them one block at a time, each
     pass seeing the prefix plus the earlier window blocks as cached history."""
