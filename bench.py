@@ -862,6 +862,43 @@ def run_reference(args, rank, world):
     return res
 
 
+def run_profile_case(args):
+    """One extra on its own, for ncu captures of its kernels: the fused LM head
+    (--lm-rows x 131072 x 4096 on seeded random weights, beside cuBLAS) or the SFT
+    attention forward and backward (--sft-seqs sequences of 4 prompt blocks and
+    --sft-blocks noisy + clean blocks). Three warm-up calls, then the timed ones."""
+    from types import SimpleNamespace
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream()
+    peaks, _ = load_peaks()
+
+    def ev_time(fn, reps=3):
+        for _ in range(3):
+            fn()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    if args.profile_case == "lm_head":
+        R, V = args.lm_rows, 131072
+        g = torch.Generator(device=dev).manual_seed(5)
+        edit = SimpleNamespace(logits=torch.empty(R, V, dtype=torch.bfloat16, device=dev), tau=0.9,
+                               committed=torch.randint(0, V, (R,), generator=g, device=dev, dtype=torch.int32))
+        res = time_lm_head({"edit": edit}, dev, peaks, ev_time)
+    else:
+        res = time_sft_attention(dev, peaks, ev_time, batch=args.sft_seqs, n_blocks=args.sft_blocks)
+    from paper_2607_22663_gb300 import mbe
+    st, flags = mbe.get_device_error()
+    if st != 0:
+        raise RuntimeError(f"device error: status {st} flags {flags:#x}")
+    return {"profile_case": args.profile_case, **res}
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -879,9 +916,17 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extras", action="store_true", help="skip the end-to-end pass and the extras (for "
                     "profiling captures; not for bench lines)")
+    ap.add_argument("--profile-case", choices=["lm_head", "sft"], default=None,
+                    help="time one extra on its own and print its JSON (for profiling captures; not a bench line)")
+    ap.add_argument("--lm-rows", type=int, default=1024, help="rows of the --profile-case lm_head projection")
+    ap.add_argument("--sft-seqs", type=int, default=4, help="sequences of the --profile-case sft batch")
+    ap.add_argument("--sft-blocks", type=int, default=64, help="noisy (= clean) blocks per --profile-case sft sequence")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.profile_case is not None:
+        print(json.dumps(run_profile_case(args)), flush=True)
+        return
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
