@@ -862,6 +862,43 @@ def run_reference(args, rank, world):
     return res
 
 
+def run_edit_kv_case(dev, stream, peaks):
+    """Edit decision over the varlen64 (4992 x 65536) and serving128 (8192 x 131072)
+    logits, three calls each, then three KV window writes of one layer of the serving
+    mix at 32 sequences (1.15 GB of cache, so that a multi-pass ncu capture holds a few GB
+    at most); timed with CUDA events."""
+    from paper_2607_22663_gb300 import mbe
+    from paper_2607_22663_gb300 import workloads as wl
+    res = {"profile_case": "edit_kv"}
+    for rows, v in ((4992, 65536), (8192, 131072)):
+        g = torch.Generator(device=dev).manual_seed(3)
+        ep = wl.edit_problem(rows, v, torch.bfloat16, 3, dev, sd=2.0, peak_frac=0.6, peak_lo=2.0, peak_hi=10.0, tau=0.9,
+                             g=g)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        ev[0].record(stream)
+        for i in range(3):
+            mbe.edit_decide(ep.logits, ep.committed, tau=ep.tau, want_argmax=False)
+            ev[i + 1].record(stream)
+        torch.cuda.synchronize()
+        ms = statistics.median(ev[i].elapsed_time(ev[i + 1]) for i in range(3))
+        gbs = edit_bytes(rows, v, 2) / (ms * 1e-3) / 1e9
+        res[f"edit_decide_{rows}x{v}"] = {"ms": round(ms, 4), "gbs": round(gbs, 1),
+                                          "frac_hbm": round(gbs / peaks["hbm_gbs"], 4)}
+        del ep
+        torch.cuda.empty_cache()
+    a = build_workload("serving128", dev, 1, 32, 8)["attn"][0]
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    ev[0].record(stream)
+    for i in range(3):
+        mbe.kv_window_write(a.k_win, a.v_win, a.k_cache, a.v_cache, a.block_table, a.prefix_len, a.window_len,
+                            a.cu_window, block_size=a.block_size, max_window=a.max_window)
+        ev[i + 1].record(stream)
+    torch.cuda.synchronize()
+    res["kv_window_write_32_seqs_ms"] = round(statistics.median(ev[i].elapsed_time(ev[i + 1])
+                                                                      for i in range(3)), 4)
+    return res
+
+
 def run_profile_case(args):
     """One extra on its own, for ncu captures of its kernels: the fused LM head
     (--lm-rows x 131072 x 4096 on seeded random weights, beside cuBLAS) or the SFT
@@ -884,6 +921,8 @@ def run_profile_case(args):
         torch.cuda.synchronize()
         return e0.elapsed_time(e1) / reps
 
+    if args.profile_case == "edit_kv":
+        return run_edit_kv_case(dev, stream, peaks)
     if args.profile_case == "lm_head":
         R, V = args.lm_rows, 131072
         g = torch.Generator(device=dev).manual_seed(5)
@@ -916,7 +955,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extras", action="store_true", help="skip the end-to-end pass and the extras (for "
                     "profiling captures; not for bench lines)")
-    ap.add_argument("--profile-case", choices=["lm_head", "sft"], default=None,
+    ap.add_argument("--profile-case", choices=["lm_head", "sft", "edit_kv"], default=None,
                     help="time one extra on its own and print its JSON (for profiling captures; not a bench line)")
     ap.add_argument("--lm-rows", type=int, default=1024, help="rows of the --profile-case lm_head projection")
     ap.add_argument("--sft-seqs", type=int, default=4, help="sequences of the --profile-case sft batch")
