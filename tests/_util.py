@@ -21,6 +21,19 @@ def dense_keys(prob, s, g):
     return torch.cat([kp, kw]), torch.cat([vp, vw])
 
 
+def np_logsumexp(s, axis=-1):
+    """log(sum(exp(s))) along an axis in float64, shifted by the row maximum; rows
+    that are all -inf give -inf. numpy rather than torch.logsumexp: torch's CPU
+    kernel returned values up to 3e-10 off in some rows on the first call of a
+    process (about one process in thirty), while the scores it was given were exact."""
+    s = np.asarray(s, dtype=np.float64)
+    m = np.max(s, axis=axis, keepdims=True)
+    m_safe = np.where(np.isfinite(m), m, 0.0)
+    with np.errstate(divide="ignore"):
+        out = np.log(np.sum(np.exp(s - m_safe), axis=axis, keepdims=True)) + m_safe
+    return np.squeeze(out, axis=axis)
+
+
 def oracle_attention(prob, units=None, scale=None):
     import oracle
     return oracle.window_attention(bf16_bits(prob.q), bf16_bits(prob.k_win), bf16_bits(prob.v_win),
