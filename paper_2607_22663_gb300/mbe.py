@@ -155,6 +155,25 @@ def _need(t, name, dtype=None, cuda=True):
         raise ValueError(f"{name} must be contiguous")
 
 
+def _shape(t, name, shape):
+    """The C ABI takes plain pointers and trusts the lengths it is given, so every
+    array the call reads or writes is held to the shape those lengths imply."""
+    if t is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
+
+
+def _same_device(dev, stream, **tensors):
+    """Every tensor on `dev`, `dev` the current CUDA device (the library launches on
+    the current device) and an explicit stream on `dev` too."""
+    for name, t in tensors.items():
+        if t is not None and t.device != dev:
+            raise ValueError(f"{name} is on {t.device}, the call's tensors are on {dev}")
+    if dev.index != torch.cuda.current_device():
+        raise ValueError(f"the tensors are on {dev} but the current CUDA device is {torch.cuda.current_device()}")
+    if stream is not None and stream.device != dev:
+        raise ValueError(f"stream is on {stream.device}, the tensors on {dev}")
+
+
 def _check(fn, st):
     if st != MBE_OK:
         raise MbeError(fn, st)
@@ -163,6 +182,25 @@ def _check(fn, st):
 def window_attention_workspace_size(batch, num_q_heads, num_kv_heads, head_dim, max_window, max_prefix):
     return int(lib().mbe_window_attention_workspace_size(batch, num_q_heads, num_kv_heads, head_dim, max_window,
                                                          max_prefix))
+
+
+def _attention_shapes(q, k_win, v_win, k_cache, v_cache, block_table, prefix_len, window_len, cu_window, mask_mode):
+    """Shapes of a window-attention call (include/mbe.h): q [T, Hq, D], k_win and v_win
+    [T, Hkv, D], caches [num_pages, Hkv, page_size, D], block_table [batch, max_pages],
+    prefix_len / window_len / mask_mode [batch], cu_window [batch + 1]."""
+    if q.dim() != 3 or k_cache.dim() != 4 or block_table.dim() != 2:
+        raise ValueError("q must be [T, Hq, D], the caches [num_pages, Hkv, page_size, D], block_table [batch, pages]")
+    T, Hq, D = q.shape
+    num_pages, Hkv, page_size, _ = k_cache.shape
+    _shape(k_cache, "k_cache", (num_pages, Hkv, page_size, D))
+    _shape(v_cache, "v_cache", (num_pages, Hkv, page_size, D))
+    _shape(k_win, "k_win", (T, Hkv, D))
+    _shape(v_win, "v_win", (T, Hkv, D))
+    batch, max_pages = block_table.shape
+    for t, n in ((prefix_len, "prefix_len"), (window_len, "window_len"), (mask_mode, "mask_mode")):
+        _shape(t, n, (batch,))
+    _shape(cu_window, "cu_window", (batch + 1,))
+    return T, Hq, D, num_pages, Hkv, page_size, batch, max_pages
 
 
 def _attention(fn_name, q, k_win, v_win, k_cache, v_cache, block_table, prefix_len, window_len, cu_window, mask_mode, *,
@@ -174,18 +212,22 @@ def _attention(fn_name, q, k_win, v_win, k_cache, v_cache, block_table, prefix_l
                  (cu_window, "cu_window")):
         _need(t, n, torch.int32)
     _need(mask_mode, "mask_mode", torch.uint8)
-    T, Hq, D = q.shape
-    num_pages, Hkv, page_size, D2 = k_cache.shape
-    if D2 != D or tuple(k_win.shape) != (T, Hkv, D) or tuple(v_win.shape) != (T, Hkv, D) or v_cache.shape != k_cache.shape:
-        raise ValueError("inconsistent q/k/v shapes")
-    batch, max_pages = block_table.shape
+    T, Hq, D, num_pages, Hkv, page_size, batch, max_pages = _attention_shapes(
+        q, k_win, v_win, k_cache, v_cache, block_table, prefix_len, window_len, cu_window, mask_mode)
     if out is None:
         out = torch.empty_like(q)
     _need(out, "out", torch.bfloat16)
+    _shape(out, "out", (T, Hq, D))
     if return_lse and lse is None:
         lse = torch.empty((T, Hq), dtype=torch.float32, device=q.device)
     if lse is not None:
         _need(lse, "lse", torch.float32)
+        _shape(lse, "lse", (T, Hq))
+    if workspace is not None:
+        _need(workspace, "workspace", torch.uint8)
+    _same_device(q.device, stream, k_win=k_win, v_win=v_win, k_cache=k_cache, v_cache=v_cache,
+                 block_table=block_table, prefix_len=prefix_len, window_len=window_len, cu_window=cu_window,
+                 mask_mode=mask_mode, out=out, lse=lse, workspace=workspace)
     need = window_attention_workspace_size(batch, Hq, Hkv, D, max_window, max_prefix)
     if workspace is None or workspace.numel() < need:
         if fn_name == "mbe_window_attention_run":
@@ -213,7 +255,13 @@ def window_attention_plan(prefix_len, window_len, cu_window, mask_mode, *, total
     for t, n in ((prefix_len, "prefix_len"), (window_len, "window_len"), (cu_window, "cu_window")):
         _need(t, n, torch.int32)
     _need(mask_mode, "mask_mode", torch.uint8)
+    _need(workspace, "workspace", torch.uint8)
     batch = prefix_len.shape[0]
+    for t, n in ((prefix_len, "prefix_len"), (window_len, "window_len"), (mask_mode, "mask_mode")):
+        _shape(t, n, (batch,))
+    _shape(cu_window, "cu_window", (batch + 1,))
+    _same_device(prefix_len.device, stream, window_len=window_len, cu_window=cu_window, mask_mode=mask_mode,
+                 workspace=workspace)
     st = lib().mbe_window_attention_plan(_ptr(prefix_len), _ptr(window_len), _ptr(cu_window), _ptr(mask_mode), batch,
                                          total_q_tokens, num_q_heads, num_kv_heads, head_dim, block_size, max_window,
                                          max_prefix, _ptr(workspace), workspace.numel(), _stream(stream))
@@ -233,9 +281,22 @@ def window_attention_noalloc(q, k_win, v_win, k_cache, v_cache, block_table, pre
     """mbe_window_attention_noalloc: the attention with the library's static
     64 MiB scratch instead of a workspace, for callers that must not allocate.
     `out` (and `lse`, if wanted) must be given: this call allocates nothing."""
-    T, Hq, D = q.shape
-    num_pages, Hkv, page_size, _ = k_cache.shape
-    batch, max_pages = block_table.shape
+    for t, n in ((q, "q"), (k_win, "k_win"), (v_win, "v_win"), (k_cache, "k_cache"), (v_cache, "v_cache"),
+                 (out, "out")):
+        _need(t, n, torch.bfloat16)
+    for t, n in ((block_table, "block_table"), (prefix_len, "prefix_len"), (window_len, "window_len"),
+                 (cu_window, "cu_window")):
+        _need(t, n, torch.int32)
+    _need(mask_mode, "mask_mode", torch.uint8)
+    T, Hq, D, num_pages, Hkv, page_size, batch, max_pages = _attention_shapes(
+        q, k_win, v_win, k_cache, v_cache, block_table, prefix_len, window_len, cu_window, mask_mode)
+    _shape(out, "out", (T, Hq, D))
+    if lse is not None:
+        _need(lse, "lse", torch.float32)
+        _shape(lse, "lse", (T, Hq))
+    _same_device(q.device, stream, k_win=k_win, v_win=v_win, k_cache=k_cache, v_cache=v_cache,
+                 block_table=block_table, prefix_len=prefix_len, window_len=window_len, cu_window=cu_window,
+                 mask_mode=mask_mode, out=out, lse=lse)
     st = lib().mbe_window_attention_noalloc(_ptr(q), _ptr(k_win), _ptr(v_win), _ptr(k_cache), _ptr(v_cache),
                                             num_pages, _ptr(block_table), max_pages, _ptr(prefix_len),
                                             _ptr(window_len), _ptr(cu_window), _ptr(mask_mode), batch, T, Hq, Hkv,
@@ -263,10 +324,15 @@ def edit_decide(logits, committed, tau=0.0, tau_per_row=None, editable=None, *, 
     confidence = torch.empty(R, dtype=torch.float32, device=dev) if confidence is None else confidence
     if want_argmax and argmax is None:
         argmax = torch.empty(R, dtype=torch.int32, device=dev)
-    if tau_per_row is not None:
-        _need(tau_per_row, "tau_per_row", torch.float32)
-    if editable is not None:
-        _need(editable, "editable", torch.uint8)
+    for t, n, dtype in ((tau_per_row, "tau_per_row", torch.float32), (editable, "editable", torch.uint8),
+                        (new_tokens, "new_tokens", torch.int32), (edit_mask, "edit_mask", torch.uint8),
+                        (confidence, "confidence", torch.float32), (argmax, "argmax", torch.int32)):
+        if t is not None:
+            _need(t, n, dtype)
+            _shape(t, n, (R,))
+    _shape(committed, "committed", (R,))
+    _same_device(dev, stream, committed=committed, tau_per_row=tau_per_row, editable=editable, new_tokens=new_tokens,
+                 edit_mask=edit_mask, confidence=confidence, argmax=argmax)
     st = lib().mbe_edit_decide(_ptr(logits), dt, logits.stride(0), R, V, _ptr(committed), _ptr(tau_per_row),
                                float(tau), _ptr(editable), _ptr(new_tokens), _ptr(edit_mask), _ptr(confidence),
                                _ptr(argmax), _stream(stream))
@@ -291,8 +357,13 @@ def denoise_update(logits, tokens, cu_rows, *, block_size, mask_id, omega_mask, 
     _need(cu_rows, "cu_rows", torch.int32)
     if editable is not None:
         _need(editable, "editable", torch.uint8)
+        _shape(editable, "editable", (R,))
+    _shape(tokens, "tokens", (R,))
+    if cu_rows.dim() != 1 or cu_rows.numel() < 1:
+        raise ValueError("cu_rows must be [sequences + 1]")
     ns = cu_rows.shape[0] - 1
     dev = logits.device
+    _same_device(dev, stream, tokens=tokens, cu_rows=cu_rows, editable=editable)
     if out is not None:
         for k, dtype in (("new_tokens", torch.int32), ("kind", torch.uint8), ("confidence", torch.float32),
                          ("argmax", torch.int32)):
@@ -320,6 +391,7 @@ def denoise_update(logits, tokens, cu_rows, *, block_size, mask_id, omega_mask, 
                "entropy": torch.empty(R, dtype=torch.float32, device=dev) if want_entropy else None,
                "block_changed": torch.empty((ns, max_blocks), dtype=torch.uint8, device=dev) if want_blocks else None,
                "seq_changes": torch.empty(ns, dtype=torch.int32, device=dev) if want_blocks else None}
+    _same_device(dev, stream, **{k: v for k, v in out.items() if v is not None})
     st = lib().mbe_denoise_update(_ptr(logits), dt, logits.stride(0), V, _ptr(cu_rows), ns, R, block_size, max_blocks,
                                   _ptr(tokens), int(mask_id), float(omega_mask), float(omega_edit), _ptr(editable),
                                   _ptr(out["new_tokens"]), _ptr(out["kind"]), _ptr(out["confidence"]),
@@ -335,6 +407,8 @@ def tail_entropy_select(block_entropy, n_valid, *, rho, k_max, want_scores=True,
     _need(n_valid, "n_valid", torch.int32)
     S, H, B = block_entropy.shape
     dev = block_entropy.device
+    _shape(n_valid, "n_valid", (S,))
+    _same_device(dev, stream, n_valid=n_valid)
     best = torch.empty(S, dtype=torch.int32, device=dev)
     wb = torch.empty(S, dtype=torch.int32, device=dev)
     scores = torch.empty((S, H), dtype=torch.float32, device=dev) if want_scores else None
@@ -352,12 +426,24 @@ def kv_window_write(k_win, v_win, k_cache, v_cache, block_table, prefix_len, win
     for t, n in ((block_table, "block_table"), (prefix_len, "prefix_len"), (window_len, "window_len"),
                  (cu_window, "cu_window")):
         _need(t, n, torch.int32)
+    if k_cache.dim() != 4 or k_win.dim() != 3 or block_table.dim() != 2:
+        raise ValueError("k_win must be [T, Hkv, D], the caches [num_pages, Hkv, page_size, D], block_table [batch, pages]")
     num_pages, Hkv, page_size, D = k_cache.shape
+    _shape(v_cache, "v_cache", (num_pages, Hkv, page_size, D))
+    _shape(k_win, "k_win", (k_win.shape[0], Hkv, D))
+    _shape(v_win, "v_win", tuple(k_win.shape))
     batch, max_pages = block_table.shape
+    _shape(prefix_len, "prefix_len", (batch,))
+    _shape(window_len, "window_len", (batch,))
+    _shape(cu_window, "cu_window", (batch + 1,))
     max_blocks = 0
     if block_write_mask is not None:
         _need(block_write_mask, "block_write_mask", torch.uint8)
+        if block_write_mask.dim() != 2 or block_write_mask.shape[0] != batch:
+            raise ValueError("block_write_mask must be [batch, blocks]")
         max_blocks = block_write_mask.shape[1]
+    _same_device(k_win.device, stream, v_win=v_win, k_cache=k_cache, v_cache=v_cache, block_table=block_table,
+                 prefix_len=prefix_len, window_len=window_len, cu_window=cu_window, block_write_mask=block_write_mask)
     st = lib().mbe_kv_window_write(_ptr(k_win), _ptr(v_win), _ptr(k_cache), _ptr(v_cache), num_pages,
                                    _ptr(block_table), max_pages, _ptr(prefix_len), _ptr(window_len), _ptr(cu_window),
                                    _ptr(block_write_mask), max_blocks, batch, max_window, Hkv, D, block_size,
@@ -395,9 +481,20 @@ def lm_head_edit_decide(hidden, weight, committed, tau=0.0, tau_per_row=None, ed
         argmax = torch.empty(R, dtype=torch.int32, device=dev)
     if want_entropy and entropy is None:
         entropy = torch.empty(R, dtype=torch.float32, device=dev)
+    for t, n, dtype in ((tau_per_row, "tau_per_row", torch.float32), (editable, "editable", torch.uint8),
+                        (new_tokens, "new_tokens", torch.int32), (edit_mask, "edit_mask", torch.uint8),
+                        (confidence, "confidence", torch.float32), (argmax, "argmax", torch.int32),
+                        (entropy, "entropy", torch.float32)):
+        if t is not None:
+            _need(t, n, dtype)
+            _shape(t, n, (R,))
     need = lm_head_workspace_size(R, V)
     if workspace is None:
         workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
+    _need(workspace, "workspace", torch.uint8)
+    _same_device(dev, stream, weight=weight, committed=committed, tau_per_row=tau_per_row, editable=editable,
+                 new_tokens=new_tokens, edit_mask=edit_mask, confidence=confidence, argmax=argmax, entropy=entropy,
+                 workspace=workspace)
     st = lib().mbe_lm_head_edit_decide(_ptr(hidden), _ptr(weight), R, V, d, _ptr(committed), _ptr(tau_per_row),
                                        float(tau), _ptr(editable), _ptr(new_tokens), _ptr(edit_mask),
                                        _ptr(confidence), _ptr(argmax), _ptr(entropy), _ptr(workspace),
@@ -415,10 +512,29 @@ def sft_block_mask(n_prompt_blocks, n_blocks, K, mask_rows, mask_words=None, out
     if out is None:
         out = torch.empty((batch, mask_rows, mask_words), dtype=torch.int32, device=n_blocks.device)
     _need(out, "out", torch.int32)
+    _shape(n_prompt_blocks, "n_prompt_blocks", (batch,))
+    _shape(out, "out", (batch, mask_rows, mask_words))
+    _same_device(n_blocks.device, stream, n_prompt_blocks=n_prompt_blocks, out=out)
     st = lib().mbe_sft_block_mask(_ptr(n_prompt_blocks), _ptr(n_blocks), int(K), batch, mask_rows, mask_words,
                                   _ptr(out), _stream(stream))
     _check("mbe_sft_block_mask", st)
     return out
+
+
+def _block_mask_shapes(q, k, v, seq_len, cu_seqlens, mask):
+    """Shapes of a block-mask attention call (include/mbe.h): q [T, Hq, D], k and v
+    [T, Hkv, D], mask [batch, mask_rows, mask_words], seq_len [batch], cu_seqlens
+    [batch + 1]."""
+    if q.dim() != 3 or k.dim() != 3 or mask.dim() != 3:
+        raise ValueError("q must be [T, Hq, D], k and v [T, Hkv, D], mask [batch, rows, words]")
+    T, Hq, D = q.shape
+    Hkv = k.shape[1]
+    _shape(k, "k", (T, Hkv, D))
+    _shape(v, "v", (T, Hkv, D))
+    batch, mask_rows, mask_words = mask.shape
+    _shape(seq_len, "seq_len", (batch,))
+    _shape(cu_seqlens, "cu_seqlens", (batch + 1,))
+    return T, Hq, D, Hkv, batch, mask_rows, mask_words
 
 
 def block_mask_attention(q, k, v, seq_len, cu_seqlens, mask, *, block_size, max_seq_len, softmax_scale=0.0,
@@ -429,19 +545,22 @@ def block_mask_attention(q, k, v, seq_len, cu_seqlens, mask, *, block_size, max_
         _need(t, n, torch.bfloat16)
     for t, n in ((seq_len, "seq_len"), (cu_seqlens, "cu_seqlens"), (mask, "mask")):
         _need(t, n, torch.int32)
-    T, Hq, D = q.shape
-    Hkv = k.shape[1]
-    batch, mask_rows, mask_words = mask.shape
+    T, Hq, D, Hkv, batch, mask_rows, mask_words = _block_mask_shapes(q, k, v, seq_len, cu_seqlens, mask)
     if out is None:
         out = torch.empty_like(q)
     _need(out, "out", torch.bfloat16)
+    _shape(out, "out", (T, Hq, D))
     if return_lse and lse is None:
         lse = torch.empty((T, Hq), dtype=torch.float32, device=q.device)
     if lse is not None:
         _need(lse, "lse", torch.float32)
+        _shape(lse, "lse", (T, Hq))
     need = window_attention_workspace_size(batch, Hq, Hkv, D, max_seq_len, 0)
     if workspace is None:
         workspace = torch.empty(max(need, 1), dtype=torch.uint8, device=q.device)
+    _need(workspace, "workspace", torch.uint8)
+    _same_device(q.device, stream, k=k, v=v, seq_len=seq_len, cu_seqlens=cu_seqlens, mask=mask, out=out, lse=lse,
+                 workspace=workspace)
     st = lib().mbe_block_mask_attention(_ptr(q), _ptr(k), _ptr(v), _ptr(seq_len), _ptr(cu_seqlens), _ptr(mask),
                                         mask_rows, mask_words, batch, T, Hq, Hkv, D, block_size, max_seq_len,
                                         float(softmax_scale), _ptr(out), _ptr(lse), _ptr(workspace), workspace.numel(),
@@ -458,18 +577,23 @@ def block_mask_attention_bwd(q, k, v, out, dout, lse, seq_len, cu_seqlens, mask,
     _need(lse, "lse", torch.float32)
     for t, n in ((seq_len, "seq_len"), (cu_seqlens, "cu_seqlens"), (mask, "mask")):
         _need(t, n, torch.int32)
-    T, Hq, D = q.shape
-    Hkv = k.shape[1]
-    batch, mask_rows, mask_words = mask.shape
+    T, Hq, D, Hkv, batch, mask_rows, mask_words = _block_mask_shapes(q, k, v, seq_len, cu_seqlens, mask)
+    _shape(out, "out", (T, Hq, D))
+    _shape(dout, "dout", (T, Hq, D))
+    _shape(lse, "lse", (T, Hq))
     dev = q.device
     dq = torch.empty((T, Hq, D), dtype=torch.float32, device=dev) if dq is None else dq
     dk = torch.empty((T, Hkv, D), dtype=torch.float32, device=dev) if dk is None else dk
     dv = torch.empty((T, Hkv, D), dtype=torch.float32, device=dev) if dv is None else dv
-    for t, n in ((dq, "dq"), (dk, "dk"), (dv, "dv")):
+    for t, n, shp in ((dq, "dq", (T, Hq, D)), (dk, "dk", (T, Hkv, D)), (dv, "dv", (T, Hkv, D))):
         _need(t, n, torch.float32)
+        _shape(t, n, shp)
     need = int(lib().mbe_block_mask_attention_bwd_workspace_size(batch, T, Hq))
     if workspace is None:
         workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
+    _need(workspace, "workspace", torch.uint8)
+    _same_device(dev, stream, k=k, v=v, out=out, dout=dout, lse=lse, seq_len=seq_len, cu_seqlens=cu_seqlens,
+                 mask=mask, dq=dq, dk=dk, dv=dv, workspace=workspace)
     st = lib().mbe_block_mask_attention_bwd(_ptr(q), _ptr(k), _ptr(v), _ptr(out), _ptr(dout), _ptr(lse),
                                             _ptr(seq_len), _ptr(cu_seqlens), _ptr(mask), mask_rows, mask_words, batch,
                                             T, Hq, Hkv, D, block_size, max_seq_len, float(softmax_scale), _ptr(dq),
@@ -511,6 +635,8 @@ def refresh_plan(block_changed, prefix_len, window_len, cu_window, block_table, 
         if tuple(out[k].shape) != shp:
             raise ValueError(f"out[{k!r}] must have shape {shp}")
     _need(out["src_row"], "src_row", torch.int32)
+    _same_device(dev, stream, prefix_len=prefix_len, window_len=window_len, cu_window=cu_window,
+                 block_table=block_table, **{f"out_{k}": t for k, t in out.items()})
     st = lib().mbe_refresh_plan(_ptr(block_changed), max_blocks, _ptr(prefix_len), _ptr(window_len), _ptr(cu_window),
                                 _ptr(block_table), max_pages, batch, block_size, max_window, out["src_row"].numel(),
                                 _ptr(out["prefix_len"]), _ptr(out["window_len"]), _ptr(out["cu_window"]),
@@ -535,6 +661,7 @@ def gather_rows(src, src_row, out=None, rows_used=None, stream=None):
     row_bytes = (src[0].numel() if src.shape[0] else out[0].numel() if rows else 1) * src.element_size()
     if rows_used is not None:
         _need(rows_used, "rows_used", torch.int32)
+    _same_device(src.device, stream, src_row=src_row, out=out, rows_used=rows_used)
     st = lib().mbe_gather_rows(_ptr(src), src.shape[0], row_bytes, _ptr(src_row), rows,
                                _ptr(rows_used) if rows_used is not None else None, _ptr(out), _stream(stream))
     _check("mbe_gather_rows", st)
@@ -562,6 +689,8 @@ def gather_rows_multi(pairs, src_row, rows_used=None, stream=None):
         nbytes.append(max(1, (src[0].numel() if src_rows else out[0].numel() if rows else 1) * src.element_size()))
     if rows_used is not None:
         _need(rows_used, "rows_used", torch.int32)
+    _same_device(src_row.device, stream, rows_used=rows_used,
+                 **{f"{k}{i}": t for i, (a, b) in enumerate(pairs) for k, t in (("src", a), ("out", b))})
     n = len(pairs)
     c_src = (ctypes.c_void_p * n)(*srcs)
     c_dst = (ctypes.c_void_p * n)(*dsts)
@@ -580,13 +709,23 @@ def refresh_gather_write(q, k_win, v_win, plan, k_cache, v_cache, *, out, stream
     for t, n in ((q, "q"), (k_win, "k_win"), (v_win, "v_win"), (k_cache, "k_cache"), (v_cache, "v_cache"),
                  (q_out, "q_out"), (k_out, "k_out"), (v_out, "v_out")):
         _need(t, n, torch.bfloat16)
+    if q.dim() != 3 or k_win.dim() != 3 or k_cache.dim() != 4:
+        raise ValueError("q must be [rows, Hq, D], k_win and v_win [rows, Hkv, D], the caches [pages, Hkv, page, D]")
     src_rows, Hq, D = q.shape
     Hkv = k_win.shape[1]
+    _shape(k_win, "k_win", (src_rows, Hkv, D))
+    _shape(v_win, "v_win", (src_rows, Hkv, D))
     num_pages, _, page_size, _ = k_cache.shape
+    _shape(k_cache, "k_cache", (num_pages, Hkv, page_size, D))
+    _shape(v_cache, "v_cache", (num_pages, Hkv, page_size, D))
     rows = plan["src_row"].numel()
     if q_out.shape[0] < rows or k_out.shape[0] < rows or v_out.shape[0] < rows:
         raise ValueError("the outputs must hold every refresh row of the plan")
+    if tuple(q_out.shape[1:]) != (Hq, D) or tuple(k_out.shape[1:]) != (Hkv, D) or tuple(v_out.shape[1:]) != (Hkv, D):
+        raise ValueError("q_out must be [rows, Hq, D] and k_out, v_out [rows, Hkv, D]")
     E, max_pages = plan["block_table"].shape
+    _same_device(q.device, stream, k_win=k_win, v_win=v_win, k_cache=k_cache, v_cache=v_cache, q_out=q_out,
+                 k_out=k_out, v_out=v_out, **{f"plan_{k}": t for k, t in plan.items()})
     st = lib().mbe_refresh_gather_write(_ptr(q), _ptr(k_win), _ptr(v_win), src_rows, Hq, Hkv, D, _ptr(plan["src_row"]),
                                         _ptr(plan["count"][1:]), rows, _ptr(plan["prefix_len"]),
                                         _ptr(plan["cu_window"]), _ptr(plan["block_table"]), E, max_pages,
