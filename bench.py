@@ -321,17 +321,36 @@ def run_gpu(args, rank, world):
     return res
 
 
-def time_extras(w, a0, dev, stream, peaks, reps=10):
-    """Entry points around the editing pass, timed outside the step: the full
-    Eq. 2 update of a standard decoding step over the same logits (a third of
-    the rows masked) and the tail-entropy window choice for every sequence."""
+def time_denoise_select(w, a0, dev, peaks, ev_time):
+    """The full Eq. 2 update of a standard decoding step over the pass's logits (a
+    third of the rows masked) and the tail-entropy window choice for every sequence."""
     from paper_2607_22663_gb300 import mbe
     ep = w["edit"]
     R, V = ep.logits.shape
     mask_id = V - 1
     tokens = ep.committed.clone()
     tokens[torch.arange(R, device=dev) % 3 == 0] = mask_id
-    cu = a0.cu_window
+    # max_blocks from the host-side window lengths and the outputs of a first call
+    # reused, as in a captured pass: the timed calls hold no host synchronisation
+    B = a0.block_size
+    kw = dict(block_size=B, mask_id=mask_id, omega_mask=0.5, omega_edit=0.0)
+    out = mbe.denoise_update(ep.logits, tokens, a0.cu_window, max_blocks=(max(a0.window_host) + B - 1) // B, **kw)
+    ms = ev_time(lambda: mbe.denoise_update(ep.logits, tokens, a0.cu_window, out=out, **kw))
+    byts = R * V * ep.logits.element_size() + R * (4 + 4 + 1 + 4 + 4 + 4)
+    ent = torch.rand(a0.batch, 3, a0.block_size, device=dev)
+    nv = torch.full((a0.batch,), 3, dtype=torch.int32, device=dev)
+    ms_sel = ev_time(lambda: mbe.tail_entropy_select(ent, nv, rho=0.25, k_max=4))
+    return {"denoise_update": {"ms": round(ms, 4), "gbs": round(byts / (ms * 1e-3) / 1e9, 1),
+                               "frac_hbm": round(byts / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"], 4),
+                               "rows": R, "vocab": V},
+            "tail_entropy_select": {"us": round(ms_sel * 1e3, 2), "sequences": a0.batch, "k_max": 4, "rho": 0.25}}
+
+
+def time_extras(w, a0, dev, stream, peaks, reps=10):
+    """Entry points around the editing pass, timed outside the step: the full Eq. 2
+    update and the tail-entropy choice, the other workloads, the fused LM head, the
+    SFT attention, the targeted refresh and the graph pass loop."""
+    from paper_2607_22663_gb300 import mbe
 
     def ev_time(fn):
         for _ in range(3):
@@ -344,12 +363,7 @@ def time_extras(w, a0, dev, stream, peaks, reps=10):
         torch.cuda.synchronize()
         return e0.elapsed_time(e1) / reps
 
-    ms = ev_time(lambda: mbe.denoise_update(ep.logits, tokens, cu, block_size=a0.block_size, mask_id=mask_id,
-                                            omega_mask=0.5, omega_edit=0.0))
-    byts = R * V * ep.logits.element_size() + R * (4 + 4 + 1 + 4 + 4 + 4)
-    ent = torch.rand(a0.batch, 3, a0.block_size, device=dev)
-    nv = torch.full((a0.batch,), 3, dtype=torch.int32, device=dev)
-    ms_sel = ev_time(lambda: mbe.tail_entropy_select(ent, nv, rho=0.25, k_max=4))
+    denoise = time_denoise_select(w, a0, dev, peaks, ev_time)
     workloads = time_workloads(dev, stream, peaks)
     lm_head = time_lm_head(w, dev, peaks, ev_time)
     sft = time_sft_attention(dev, peaks, ev_time)
@@ -358,12 +372,8 @@ def time_extras(w, a0, dev, stream, peaks, reps=10):
     st, flags = mbe.get_device_error()
     if st != 0:
         raise RuntimeError(f"device error in extras: status {st} flags {flags:#x}")
-    return {"denoise_update": {"ms": round(ms, 4), "gbs": round(byts / (ms * 1e-3) / 1e9, 1),
-                               "frac_hbm": round(byts / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"], 4),
-                               "rows": R, "vocab": V},
-            "tail_entropy_select": {"us": round(ms_sel * 1e3, 2), "sequences": a0.batch, "k_max": 4, "rho": 0.25},
-            "lm_head_edit_decide": lm_head, "sft_attention": sft, "refresh": refresh, "pass_loop": loop,
-            **workloads}
+    return {**denoise, "lm_head_edit_decide": lm_head, "sft_attention": sft, "refresh": refresh,
+            "pass_loop": loop, **workloads}
 
 
 def time_workloads(dev, stream, peaks, reps=10):
@@ -901,9 +911,11 @@ def run_edit_kv_case(dev, stream, peaks):
 
 def run_profile_case(args):
     """One extra on its own, for ncu captures of its kernels: the fused LM head
-    (--lm-rows x 131072 x 4096 on seeded random weights, beside cuBLAS) or the SFT
+    (--lm-rows x 131072 x 4096 on seeded random weights, beside cuBLAS), the SFT
     attention forward and backward (--sft-seqs sequences of 4 prompt blocks and
-    --sft-blocks noisy + clean blocks). Three warm-up calls, then the timed ones."""
+    --sft-blocks noisy + clean blocks), edit-decide and the KV write, or the Eq. 2
+    update, tail-entropy choice and targeted refresh of the serving mix (--batch,
+    --layers). Three warm-up calls, then the timed ones."""
     from types import SimpleNamespace
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
@@ -923,13 +935,21 @@ def run_profile_case(args):
 
     if args.profile_case == "edit_kv":
         return run_edit_kv_case(dev, stream, peaks)
-    if args.profile_case == "lm_head":
+    if args.profile_case == "refresh":
+        # the serving mix at --batch sequences (default 128) and --layers layers
+        # (default 2): the Eq. 2 update and the tail-entropy choice over its
+        # logits, then one targeted refresh pass of a seeded eighth of the blocks
+        w = build_workload("serving128", dev, args.layers or 2, args.batch, args.vocab)
+        res = {**time_denoise_select(w, w["attn"][0], dev, peaks, ev_time),
+               "refresh": time_refresh(w, dev, stream, peaks, ev_time),
+               "config": workload_config(w)}
+    elif args.profile_case == "lm_head":
         R, V = args.lm_rows, 131072
         g = torch.Generator(device=dev).manual_seed(5)
         edit = SimpleNamespace(logits=torch.empty(R, V, dtype=torch.bfloat16, device=dev), tau=0.9,
                                committed=torch.randint(0, V, (R,), generator=g, device=dev, dtype=torch.int32))
         res = time_lm_head({"edit": edit}, dev, peaks, ev_time)
-    else:
+    elif args.profile_case == "sft":
         res = time_sft_attention(dev, peaks, ev_time, batch=args.sft_seqs, n_blocks=args.sft_blocks)
     from paper_2607_22663_gb300 import mbe
     st, flags = mbe.get_device_error()
@@ -955,7 +975,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extras", action="store_true", help="skip the end-to-end pass and the extras (for "
                     "profiling captures; not for bench lines)")
-    ap.add_argument("--profile-case", choices=["lm_head", "sft", "edit_kv"], default=None,
+    ap.add_argument("--profile-case", choices=["lm_head", "sft", "edit_kv", "refresh"], default=None,
                     help="time one extra on its own and print its JSON (for profiling captures; not a bench line)")
     ap.add_argument("--lm-rows", type=int, default=1024, help="rows of the --profile-case lm_head projection")
     ap.add_argument("--sft-seqs", type=int, default=4, help="sequences of the --profile-case sft batch")
